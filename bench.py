@@ -1,0 +1,440 @@
+#!/usr/bin/env python3
+"""Benchmark of the gradient-coding hot path on one GB300 (or N replicas).
+
+Workload: logistic regression, m = N = 20 workers/chunks, cyclic assignment
+with delta = 4 chunks per worker, d = 4096, 512 points per chunk (X is 168 MB,
+larger than L2), 10^4 shifted-exponential straggler realizations per step,
+communication factor l = 2.
+
+One step (every row of the hot path once):
+  1. chunk gradients g_{D_i} at the current w            (gc_chunk_grads)
+  2. Algorithm 1 for all 10^4 patterns -> decode matrix C,
+     coefficient error and estimate                       (gc_find_encoding_coeff)
+  3. batched decode-combine Ghat = C . G (10^4 decoded
+     gradients written) with the fused gradient MSE       (gc_decode_combine)
+  4. the live realization: worker encoding (eq. 2), PS
+     decode of the transmissions, and the SGD update      (gc_encode, gc_decode_tx, gc_sgd_step)
+Each stage is captured once in a CUDA graph; CUDA events between the graph
+replays time every stage live inside the timed region.
+
+Metric: decoded gradients per second (whole job).  `e2e` repeats the timed
+loop through the same C-ABI calls with the step's inputs (the pattern batch
+and the live pattern) copied from pinned host memory and the per-pattern
+results (coefficient error, estimate, gradient MSE, loss) copied back every
+step.  `--impl reference` times the fp64 CPU oracle on the host cores instead.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "decoded gradients/sec (logistic m=N=20, delta=4, d=4096, 10^4 realizations, l=2)"
+UNIT = "decoded gradients/s"
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--impl", choices=["gc", "reference"], default="gc")
+    ap.add_argument("--ell", type=int, default=2)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--min-warm-seconds", type=float, default=1.5,
+                    help="keep warming up at least this long (steady clocks, clock samples)")
+    return ap.parse_args()
+
+
+def peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return d, "measured"
+    return FALLBACK_PEAKS, "fallback"
+
+
+# ------------------------------------------------------------------ clocks
+class Clocks:
+    """nvidia-smi samples every 200 ms while the GPU is under load."""
+    Q = ("index,uuid,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, uuid: str | None):
+        self.uuid = uuid
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        try:
+            fd, self.path = tempfile.mkstemp(suffix=".csv")
+            os.close(fd)
+            cmd = ["nvidia-smi", f"--query-gpu={self.Q}", "--format=csv,noheader,nounits", "-lms", "200"]
+            if self.uuid:
+                cmd += ["-i", self.uuid]
+            self.proc = subprocess.Popen(cmd, stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+
+    def stop(self) -> dict:
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        sm, mx, reasons, power = [], [], set(), []
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        with open(self.path) as f:
+            for line in f:
+                parts = [x.strip() for x in line.split(",")]
+                if len(parts) < 10:
+                    continue
+                try:
+                    sm.append(float(parts[2]))
+                    mx.append(float(parts[3]))
+                    power.append(float(parts[4]))
+                except ValueError:
+                    continue
+                for n, v in zip(names, parts[6:10]):
+                    if v.lower().startswith("active"):
+                        reasons.add(n)
+        os.unlink(self.path)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "samples": len(sm),
+                "power_w_max": max(power) if power else None, "reasons": sorted(reasons)}
+
+
+# ------------------------------------------------------------------ oracle timing
+def oracle_step_rate(cfg, data_cpu, ell, n_sample, seed_stream):
+    """Time the fp64 oracle on this host: one full chunk-gradient pass plus
+    `n_sample` realizations through Algorithm 1, encode and decode; returns
+    (decoded gradients/s extrapolated to the full batch, seconds used)."""
+    import oracle as O
+    from workloads import make_patterns, make_R
+
+    N, m, delta = cfg.N, cfg.m, cfg.delta
+    order = O.cyclic_order(N, m, delta)
+    R = make_R(cfg, ell)
+    X, y, w = data_cpu["X"].numpy(), data_cpu["y"].numpy(), data_cpu["w"].numpy()
+    t0 = time.perf_counter()
+    G = O.chunk_gradients(X, y, w, N, cfg.n_c, O.LOGISTIC)
+    t_cg = time.perf_counter() - t0
+    psi = make_patterns(cfg, npat=n_sample, stream=seed_stream)
+    t1 = time.perf_counter()
+    for b in range(n_sample):
+        O.run_pattern(R, order, psi[b], N, G, want_transmit=True)
+    t_pat = (time.perf_counter() - t1) / n_sample
+    step = t_cg + cfg.npat * t_pat
+    return cfg.npat / step, time.perf_counter() - t0, t_cg, t_pat
+
+
+def reference_arm(args, rank, world):
+    from workloads import get, make_data
+
+    if rank != 0:
+        return
+    cfg = get("logistic")
+    data = make_data(cfg, "cpu")
+    n_sample = 64
+    for t in range(args.warmup):
+        oracle_step_rate(cfg, data, args.ell, 8, 10_000 + t)
+    rates, t_all = [], time.perf_counter()
+    for t in range(args.steps):
+        r, _, _, _ = oracle_step_rate(cfg, data, args.ell, n_sample, 20_000 + t)
+        rates.append(r)
+    wall = time.perf_counter() - t_all
+    value = statistics.median(rates)
+    cores = os.cpu_count()
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * cfg.npat / value,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic",
+        "config": {"workload": "logistic m=N=20 delta=4 d=4096 n_c=512 npat=10000 ell=%d" % args.ell,
+                   "l2": "inputs larger than L2 (X 168 MB)"},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
+                         "sample": f"each step: full fp64 chunk-gradient pass + {n_sample} realizations "
+                                   "(Algorithm 1 per worker, eq. 2 encode, decode), extrapolated to 10^4; "
+                                   "pattern loop single-threaded NumPy"},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+        "wall_s": wall,
+    }
+    print(json.dumps(line), flush=True)
+
+
+# ------------------------------------------------------------------ GPU arm
+def _src_hash(names):
+    h = hashlib.sha256()
+    for n in names:
+        with open(os.path.join(ROOT, "paper_2405_19509_gb300", "csrc", n), "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()[:16]
+
+
+def _traffic(kernel, src_files):
+    """dram bytes per launch from a committed ncu summary, if it was taken
+    on the current kernel source (else None)."""
+    p = os.path.join(ROOT, "profiles", "traffic.json")
+    if not os.path.exists(p):
+        return None
+    with open(p) as f:
+        d = json.load(f)
+    e = d.get(kernel)
+    if not e or e.get("src_hash") != _src_hash(src_files):
+        return None
+    return e.get("dram_bytes_per_launch")
+
+
+def gpu_arm(args, rank, world, local_rank):
+    import torch
+
+    import paper_2405_19509_gb300 as gc
+    from workloads import get, make_data, make_patterns, make_R
+
+    dev = torch.device("cuda", local_rank)
+    torch.cuda.set_device(dev)
+    cfg = get("logistic")
+    N, m, delta, d, n_c, ell, npat = cfg.N, cfg.m, cfg.delta, cfg.d, cfg.n_c, args.ell, cfg.npat
+    L = -(-d // ell)
+    data_cpu = make_data(cfg, "cpu")
+    X = data_cpu["X"].to(dev)
+    y = data_cpu["y"].to(dev)
+    w = data_cpu["w"].to(dev).clone()
+    _, order, _ = gc.gc_make_assignment(N, m, delta, gc.GC_CYCLIC)
+    Rd = torch.from_numpy(make_R(cfg, ell)).to(dev)
+    od = torch.from_numpy(order).to(dev)
+    S = args.warmup + args.steps
+    # realizations: each rank draws its own batches (replicas over independent patterns)
+    base = 1_000_000 * rank
+    psi_host = np.stack([make_patterns(cfg, stream=base + t) for t in range(S)])
+    live_host = np.stack([make_patterns(cfg, npat=1, stream=base + 500_000 + t) for t in range(S)])
+    psi_all = torch.from_numpy(psi_host).to(dev)
+    live_all = torch.from_numpy(live_host).to(dev)
+    # static buffers
+    psi_s = torch.empty(npat, m, dtype=torch.int32, device=dev)
+    live_s = torch.empty(1, m, dtype=torch.int32, device=dev)
+    G_s = torch.empty(N, d, dtype=torch.float32, device=dev)
+    loss_s = torch.zeros(1, dtype=torch.float64, device=dev)
+    C_s = torch.empty(npat, ell, N * ell, dtype=torch.float32, device=dev)
+    ce_s = torch.empty(npat, dtype=torch.float64, device=dev)
+    est_s = torch.empty(npat, dtype=torch.float64, device=dev)
+    Gh_s = torch.empty(npat, d, dtype=torch.float32, device=dev)
+    mse_s = torch.empty(npat, dtype=torch.float64, device=dev)
+    T_s = torch.empty(1, m, L, dtype=torch.float32, device=dev)
+    gh_s = torch.empty(1, d, dtype=torch.float32, device=dev)
+    wsA, wsB, wsC, wsD = (gc.Workspace(dev) for _ in range(4))
+
+    def stage_a():
+        gc.gc_chunk_grads(X, y, w, N, n_c, gc.GC_LOGISTIC, G=G_s, loss_out=loss_s, ws=wsA)
+
+    def stage_b():
+        gc.gc_find_encoding_coeff(Rd, ell, od, N, m, delta, psi_s, E=False, C=C_s, delta_out=False,
+                                  support=False, coef_err=ce_s, est=est_s, ws=wsB)
+
+    def stage_c():
+        gc.gc_decode_combine(C_s, ell, N, G_s, Ghat=Gh_s, grad_mse=mse_s, ws=wsC)
+
+    def stage_d():
+        gc.gc_encode(Rd, ell, od, N, m, delta, live_s, G_s, T=T_s, ws=wsD)
+        gc.gc_decode_tx(Rd, ell, m, T_s, d, ghat=gh_s)
+        gc.gc_sgd_step(w, gh_s[0], cfg.lr, cfg.Ntil)
+
+    stages = [stage_a, stage_b, stage_c, stage_d]
+    # eager run: allocates workspaces, checks the device status words
+    psi_s.copy_(psi_all[0])
+    live_s.copy_(live_all[0])
+    for f in stages:
+        f()
+    for ws in (wsA, wsB, wsC, wsD):
+        gc.gc_status(ws)
+    torch.cuda.synchronize()
+    # capture each stage in its own graph
+    n0 = gc.gc_kernel_launches()
+    graphs = []
+    cap_stream = torch.cuda.Stream(dev)
+    for f in stages:
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=cap_stream):
+            f()
+        graphs.append(g)
+    launches_per_step = gc.gc_kernel_launches() - n0
+    torch.cuda.synchronize()
+
+    stream = torch.cuda.current_stream(dev)
+
+    def run_step(t, evs=None):
+        psi_s.copy_(psi_all[t], non_blocking=True)
+        live_s.copy_(live_all[t], non_blocking=True)
+        if evs is not None:
+            evs[0].record(stream)
+        for k, g in enumerate(graphs):
+            g.replay()
+            if evs is not None:
+                evs[k + 1].record(stream)
+
+    import torch.distributed as tdist
+
+    def barrier():
+        if world > 1:
+            tdist.barrier()
+
+    props = torch.cuda.get_device_properties(dev)
+    uuid = getattr(props, "uuid", None)
+    clocks = Clocks(f"GPU-{uuid}" if uuid is not None else None)
+    clocks.start()
+    # warm-up: at least W steps and at least --min-warm-seconds
+    t_w = time.perf_counter()
+    t = 0
+    while t < args.warmup or time.perf_counter() - t_w < args.min_warm_seconds:
+        run_step(t % S)
+        t += 1
+        if t % 64 == 0:
+            torch.cuda.synchronize()
+    torch.cuda.synchronize()
+
+    K = args.steps
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(5)] for _ in range(K)]
+    barrier()
+    torch.cuda.synchronize()
+    t_start = torch.cuda.Event(enable_timing=True)
+    t_end = torch.cuda.Event(enable_timing=True)
+    wall0 = time.perf_counter()
+    t_start.record(stream)
+    for k in range(K):
+        run_step(args.warmup + k if args.warmup + k < S else k % S, evs[k])
+    t_end.record(stream)
+    torch.cuda.synchronize()
+    barrier()
+    wall = time.perf_counter() - wall0
+    clk = clocks.stop()
+    total_ms = t_start.elapsed_time(t_end)
+    stage_ms = np.zeros(4)
+    for k in range(K):
+        for s in range(4):
+            stage_ms[s] += evs[k][s].elapsed_time(evs[k][s + 1])
+    stage_ms /= K
+    for ws in (wsA, wsB, wsC, wsD):
+        gc.gc_status(ws)
+
+    # ---- end to end through the C-ABI with host buffers
+    pin_psi = torch.from_numpy(psi_host).pin_memory()
+    pin_live = torch.from_numpy(live_host).pin_memory()
+    out_ce = torch.empty(K, npat, dtype=torch.float64).pin_memory()
+    out_est = torch.empty(K, npat, dtype=torch.float64).pin_memory()
+    out_mse = torch.empty(K, npat, dtype=torch.float64).pin_memory()
+    out_loss = torch.empty(K, 1, dtype=torch.float64).pin_memory()
+    barrier()
+    torch.cuda.synchronize()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for k in range(K):
+        t = (args.warmup + k) % S
+        psi_s.copy_(pin_psi[t], non_blocking=True)
+        live_s.copy_(pin_live[t], non_blocking=True)
+        for g in graphs:
+            g.replay()
+        out_ce[k].copy_(ce_s, non_blocking=True)
+        out_est[k].copy_(est_s, non_blocking=True)
+        out_mse[k].copy_(mse_s, non_blocking=True)
+        out_loss[k].copy_(loss_s, non_blocking=True)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    barrier()
+    e2e_ms = e0.elapsed_time(e1)
+    assert np.all(np.isfinite(out_mse.numpy())) and np.all(out_est.numpy() >= 0)
+
+    # ---- max over ranks
+    times = torch.tensor([total_ms, e2e_ms], dtype=torch.float64, device=dev)
+    if world > 1:
+        tdist.all_reduce(times, op=tdist.ReduceOp.MAX)
+    total_ms, e2e_ms = times.tolist()
+    value = world * npat * K / (total_ms / 1e3)
+    e2e_value = world * npat * K / (e2e_ms / 1e3)
+
+    # ---- roofline of the dominant stage
+    pk, pk_src = peaks()
+    hbm = float(pk["hbm_gbs"])
+    names = ["k_chunkgrad", "k_patterns", "k_combine_simt", "encode+decode_tx+sgd"]
+    alg_bytes = [
+        cfg.Ntil * d * 4 + cfg.Ntil * 4 + N * d * 4,                          # X, y read; G written
+        npat * m * 4 + npat * ell * N * ell * 4 + 2 * npat * 8,               # psi read; C, errors written
+        npat * d * 4 + npat * ell * N * ell * 4 + N * d * 4 + npat * 8,       # Ghat written; C, G read
+        N * d * 4 + m * L * 4 * 2 + d * 4 * 3,                                # G read; T; ghat; w
+    ]
+    srcs = [["k_chunkgrad.cu"], ["k_solve.cu"], ["k_combine.cu"], ["k_encode.cu"]]
+    dom = int(np.argmax(stage_ms))
+    achieved = alg_bytes[dom] / (stage_ms[dom] / 1e3) / 1e9
+    roofline = {"kernel": names[dom], "bound": "hbm", "achieved": achieved, "peak": hbm,
+                "unit": "GB/s", "frac": achieved / hbm, "peak_source": f"{pk_src} hbm_gbs",
+                "traffic": _traffic(names[dom], srcs[dom]),
+                "timing": "CUDA events around the stage's graph (kernel plus its small helpers), "
+                          "averaged over the timed steps",
+                "stage_ms": {n: float(v) for n, v in zip(names, stage_ms)},
+                "stage_frac_of_hbm": {n: float(b / (t / 1e3) / 1e9 / hbm) for n, b, t in
+                                      zip(names, alg_bytes, stage_ms)}}
+
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K,
+        "warmup": args.warmup, "ms_per_step": total_ms / K, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+        "config": {"workload": "logistic m=N=20 delta=4 d=4096 n_c=512 npat=10000 ell=%d" % ell,
+                   "l2": "inputs larger than L2 (X 168 MB, Ghat 164 MB per step)",
+                   "parallelism": f"replicas x{world} (independent realization batches)"},
+        "roofline": roofline,
+        "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": int(npat * m * 4 + m * 4),
+                "d2h_bytes_per_step": int(3 * npat * 8 + 8)},
+        "gpu_launches": int(launches_per_step * K),
+        "clocks": clk,
+        "wall_s_timed": wall,
+    }
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        rate, used, t_cg, t_pat = oracle_step_rate(cfg, data_cpu, ell, 256, 7_777)
+        line["cpu_baseline"] = {
+            "value": rate, "unit": UNIT, "cores": os.cpu_count(), "kind": "oracle",
+            "sample": f"full fp64 chunk-gradient pass ({t_cg:.3f} s, BLAS threads) + 256 realizations "
+                      f"({1e3 * t_pat:.2f} ms each, single-threaded NumPy), extrapolated to 10^4; "
+                      f"{used:.1f} s of CPU work"}
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+
+
+def main():
+    args = parse()
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+    if args.impl == "reference":
+        reference_arm(args, rank, world)
+        return
+    if world > 1:
+        import torch
+        import torch.distributed as tdist
+        torch.cuda.set_device(local_rank)
+        tdist.init_process_group("nccl", device_id=torch.device("cuda", local_rank))
+    gpu_arm(args, rank, world, local_rank)
+    if world > 1:
+        import torch.distributed as tdist
+        tdist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,218 @@
+/*
+ * gc.h -- C ABI of the GB300 gradient-coding library (libgc.so).
+ *
+ * Implements the data-parallel hot path of the partial-straggler
+ * gradient-coding protocol of "Leveraging partial stragglers within gradient
+ * coding" (Ramamoorthy, Meng, Girimaji): chunk gradients (Sec. I), the
+ * encoding coefficients of Algorithm 1, worker encoding (eq. 2), PS decoding
+ * (Sec. II-B), batched over many straggler patterns, and the error measures
+ * of Sec. II-A / Sec. IV.  Workers and the PS are simulated on one device.
+ *
+ * Notation: N chunks, m workers, delta chunks per worker (load), ell the
+ * communication factor, d the parameter dimension, L = ceil(d / ell) the block
+ * length, n_c points per chunk, N~ = N * n_c, npat straggler patterns.
+ *
+ * Conventions shared by every entry point
+ *  - Return value: GC_OK (0) or a negative GC_ERR_* code.  On error,
+ *    gc_last_error() returns a thread-local message.  No C++ exception
+ *    crosses this boundary.
+ *  - Ownership: every buffer belongs to the caller.  The library never
+ *    allocates device or host memory and never frees caller memory.
+ *    Pointers without the _h suffix are DEVICE pointers; *_h are host pointers.
+ *  - Scratch: an entry point that needs scratch takes (ws, ws_bytes), a
+ *    device buffer of at least the size its gc_*_workspace() function
+ *    returns, 256-byte aligned.  The first 256 bytes are a status header
+ *    that kernels set when they detect bad data on the device (a psi entry
+ *    outside [0, delta], a rank-deficient least-squares system, a bounded
+ *    wait that expired).  The header is sticky: it must be zeroed once
+ *    before first use (gc_workspace_init) and is read and cleared by
+ *    gc_status().
+ *  - Streams: `stream` is a cudaStream_t (NULL = legacy default stream).
+ *    All device entry points are asynchronous on it; gc_make_assignment is
+ *    host-only and synchronous.
+ *  - Layouts are row-major and dense unless stated.
+ *  - Validation of sizes and pointers happens on the host before any
+ *    launch; nothing is launched when a check fails.
+ */
+#ifndef GC_H_
+#define GC_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* ---- status codes ---------------------------------------------------- */
+#define GC_OK 0
+#define GC_ERR_ARG (-1)         /* null pointer, out-of-range enum or scalar */
+#define GC_ERR_SHAPE (-2)       /* inconsistent or out-of-range sizes        */
+#define GC_ERR_UNSUPPORTED (-3) /* valid but not supported (ell > 8, delta > 32, ...) */
+#define GC_ERR_CUDA (-4)        /* a CUDA runtime call failed                */
+#define GC_ERR_TIMEOUT (-5)     /* a bounded device wait expired             */
+#define GC_ERR_WORKSPACE (-6)   /* workspace missing, too small or misaligned */
+#define GC_ERR_DATA (-7)        /* device-detected bad data (see gc_status)   */
+
+/* ---- enums ----------------------------------------------------------- */
+#define GC_CYCLIC 0   /* W_j holds chunks j, j+1, ..., j+delta-1 (mod N)   */
+#define GC_EXPLICIT 1 /* orders given by the caller                        */
+
+#define GC_F32 0  /* X element type: float32                              */
+#define GC_BF16 1 /* X element type: bfloat16                             */
+
+#define GC_LSQ 0      /* l = (x^T w - y)^2 / 2                             */
+#define GC_LOGISTIC 1 /* l = log(1 + exp(-y x^T w)), y in {-1, +1}          */
+
+/* Limits of this build. */
+#define GC_MAX_ELL 8      /* communication factor ell                        */
+#define GC_MAX_DELTA 32   /* chunks per worker                               */
+#define GC_MAX_REPL 32    /* copies of one chunk in the cluster (gamma_i)    */
+
+/* ---- library ---------------------------------------------------------- */
+/* Thread-local text of the last error raised on this thread ("" if none). */
+const char* gc_last_error(void);
+
+/* Version as 10000*major + 100*minor + patch. */
+int gc_version(void);
+
+/* Number of CUDA kernels this library has launched since it was loaded
+ * (launches recorded into a CUDA graph count once, at capture). */
+uint64_t gc_kernel_launches(void);
+
+/* Zero the status header of a workspace (asynchronous on `stream`). */
+int gc_workspace_init(void* ws, size_t ws_bytes, void* stream);
+
+/* Synchronise `stream`, read and clear the workspace status header.
+ * Returns GC_OK, GC_ERR_DATA (bad psi / singular system) or GC_ERR_TIMEOUT;
+ * the message names what was found. */
+int gc_status(void* ws, void* stream);
+
+/* ---- assignment (Sec. I assignment matrix A; Sec. III ordering matrix O) --
+ * Host only.  kind = GC_CYCLIC: requires N == m; W_j processes chunks
+ * (j + p) mod N for p = 0..delta-1 top to bottom (the cyclic assignment that
+ * Sec. III shows optimal for the Q_max metric).  kind = GC_EXPLICIT: the
+ * m x delta int32 array explicit_order_h lists, per worker, its chunks in
+ * processing order, -1 marking an empty slot (empty slots only at the end
+ * of a row); a chunk may appear at most once per worker and at most
+ * GC_MAX_REPL times overall.
+ * Outputs (host, caller-owned, any may be NULL):
+ *   A_h      N x m uint8, A[i][j] = 1 iff D_i is assigned to W_j.
+ *   order_h  m x delta int32, the processing order (copy of the input for
+ *            GC_EXPLICIT).
+ *   O_h      N x m uint8, O[i][j] = position (1-based) of D_i in W_j, 0 if
+ *            not assigned.
+ */
+int gc_make_assignment(int N, int m, int delta, int kind, const int32_t* explicit_order_h,
+                       uint8_t* A_h, int32_t* order_h, uint8_t* O_h);
+
+/* ---- chunk gradients (Sec. I: g_{D_j} = sum_{i in D_j} grad l) --------
+ * X        N~ x d, element type x_dtype, row-major, 16-byte aligned; chunk i
+ *          is rows [i*n_c, (i+1)*n_c).
+ * y        N~ float32 labels (+-1 for GC_LOGISTIC).
+ * w        d float32 parameter vector.
+ * G        N x d float32 output: G[i] = X_i^T (f(X_i w) - y01_i), f = identity
+ *          (GC_LSQ, y01 = y) or the logistic sigmoid (GC_LOGISTIC,
+ *          y01 = (y + 1) / 2).  Un-normalised sums, as in Sec. I.
+ * loss_out NULL or one device double: L = (1/N~) sum_i l(x_i, y_i, w).
+ * Requires d >= 1, n_c >= 1, N >= 1.  One pass over X.
+ */
+size_t gc_chunk_grads_workspace(int N, int n_c, int d, int x_dtype);
+int gc_chunk_grads(const void* X, int x_dtype, const float* y, const float* w, int N, int n_c,
+                   int d, int loss, float* G, double* loss_out, void* ws, size_t ws_bytes,
+                   void* stream);
+
+/* ---- Algorithm 1, Find-Encoding-Coeff, batched over patterns ----------
+ * R      ell x m float64, the PS's Gaussian matrix (Sec. II).
+ * order  m x delta int32 device copy of the processing order (-1 = empty).
+ * psi    npat x m int32 state vectors: psi[b][j] = chunks W_j processed in
+ *        pattern b, 0 <= psi <= delta (checked on the device: bad entries
+ *        are treated as 0 and raise GC_ERR_DATA in the status header).
+ * For every pattern b and chunk i, S_i = workers that processed D_i and
+ * Delta_i = |S_i|; the block column B^(i) restricted to rows S_i is the
+ * minimum-norm least-squares solution X^+ of eq. (6), X = R[:, S_i]
+ * (computed in float64).  Outputs (each may be NULL):
+ *   E         npat x m x delta x ell float64: E[b][j][p][k] = the coefficient
+ *             W_j applies to g_{D_{order[j][p]}}[k] (eps_j of Algorithm 1 in
+ *             processing order), 0 for p >= psi[b][j].
+ *   C         npat x ell x (N*ell) float32: the decode matrix R B, i.e.
+ *             C[b][k][i*ell + k'] = (R_{S_i} X^+)[k][k'] (a projector; the
+ *             identity when Delta_i >= ell, Sec. II-A).
+ *   delta_out npat x N uint8: Delta_i.
+ *   support   npat x N x m uint8: 1 iff W_j processed D_i (supports of
+ *             eqs. 3 and 8).
+ *   coef_err  npat float64: || (1_N (x) I_ell)^T - R B ||_F^2.
+ *   est       npat float64: sum_i max(0, ell - Delta_i) (eq. 7).
+ */
+size_t gc_coeff_workspace(int N, int m, int delta, int ell, int npat);
+int gc_find_encoding_coeff(const double* R, int ell, const int32_t* order, int N, int m, int delta,
+                           const int32_t* psi, int npat, double* E, float* C, uint8_t* delta_out,
+                           uint8_t* support, double* coef_err, double* est, void* ws,
+                           size_t ws_bytes, void* stream);
+
+/* ---- worker encoding (eq. 2) ------------------------------------------
+ * Runs Algorithm 1 for every pattern, then each worker's transmission
+ *   T[b][j] = sum_{p < psi[b][j]} sum_k E[b][j][p][k] g_{D_order[j][p]}[k],
+ * where g[k] = g[k*L : (k+1)*L] zero-padded to length L.
+ * G  N x d float32 chunk gradients; T npat x m x L float32 output.
+ */
+size_t gc_encode_workspace(int N, int m, int delta, int ell, int npat, int d);
+int gc_encode(const double* R, int ell, const int32_t* order, int N, int m, int delta,
+              const int32_t* psi, int npat, const float* G, int d, float* T, void* ws,
+              size_t ws_bytes, void* stream);
+
+/* ---- PS decoding of received transmissions (Sec. II-B) ----------------
+ * ghat[b][k*L + c] = sum_j R[k][j] T[b][j][c] for k*L + c < d.
+ * T npat x m x L float32; ghat npat x d float32.  No workspace.
+ */
+int gc_decode_tx(const double* R, int ell, int m, const float* T, int npat, int d, float* ghat,
+                 void* stream);
+
+/* ---- batched decode-combine -------------------------------------------
+ * The composition of encode and decode for many patterns at once, using the
+ * identity sum_j R[k][j] T[b][j] = sum_i sum_k' (R B_b)[k][i*ell+k'] g_{D_i}[k']:
+ *   Ghat (npat*ell x L) = C (npat*ell x N*ell) . G (N*ell x L),
+ * with C from Algorithm 1 (above) and G viewed as N*ell blocks of length L.
+ * G     N x d float32 chunk gradients.
+ * Ghat  NULL or npat x d float32 decoded gradients.
+ * coef_err, est   NULL or npat float64 (as gc_find_encoding_coeff).
+ * grad_mse        NULL or npat float64: ||ghat_b - sum_i g_{D_i}||^2 / d,
+ *                 reduced in a fixed order (deterministic).
+ * At least one of Ghat / grad_mse must be non-NULL.
+ */
+size_t gc_decode_batch_workspace(int N, int m, int delta, int ell, int npat, int d);
+int gc_decode_batch(const double* R, int ell, const int32_t* order, int N, int m, int delta,
+                    const int32_t* psi, int npat, const float* G, int d, float* Ghat,
+                    double* coef_err, double* est, double* grad_mse, void* ws, size_t ws_bytes,
+                    void* stream);
+
+/* ---- decode-combine alone ----------------------------------------------
+ * The GEMM step of gc_decode_batch for a decode matrix the caller already
+ * has (e.g. from gc_find_encoding_coeff):
+ *   Ghat (npat*ell x L) = C (npat*ell x N*ell) . G (N*ell x L).
+ * C     npat x ell x (N*ell) float32 (layout of gc_find_encoding_coeff's C).
+ * G     N x d float32; Ghat NULL or npat x d float32; grad_mse NULL or npat
+ *       float64 (||ghat_b - sum_i g_{D_i}||^2 / d).  One of the two non-NULL.
+ */
+size_t gc_decode_combine_workspace(int N, int ell, int npat, int d);
+int gc_decode_combine(const float* C, int ell, int N, int npat, const float* G, int d,
+                      float* Ghat, double* grad_mse, void* ws, size_t ws_bytes, void* stream);
+
+/* ---- error measures only (Sec. II-A eq. 7, Sec. IV) -------------------
+ * gc_decode_batch with Ghat = NULL: coef_err, est and grad_mse per pattern;
+ * the decoded gradients are reduced on chip and never written.
+ */
+size_t gc_mse_workspace(int N, int m, int delta, int ell, int npat, int d);
+int gc_mse(const double* R, int ell, const int32_t* order, int N, int m, int delta,
+           const int32_t* psi, int npat, const float* G, int d, double* coef_err, double* est,
+           double* grad_mse, void* ws, size_t ws_bytes, void* stream);
+
+/* ---- parameter update (Sec. I: w_{t+1} from grad L = (1/N~) sum g) ----
+ * w[c] -= lr * ghat[c] / Ntil for c < d.  w, ghat float32 device vectors.
+ */
+int gc_sgd_step(float* w, const float* ghat, int d, float lr, int64_t Ntil, void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* GC_H_ */

@@ -173,8 +173,9 @@ def unblock(gb: np.ndarray, d: int) -> np.ndarray:
 # The state vector psi and the support of B (Sec. II)
 # --------------------------------------------------------------------------
 def processed_chunks(order: np.ndarray, psi, j: int) -> list[int]:
-    """Chunks W_j has processed: the first psi_j entries of its order."""
-    return [int(c) for c in order[j, : int(psi[j])]]
+    """Chunks W_j has processed: the first psi_j entries of its order (an
+    empty slot, -1, holds no chunk)."""
+    return [int(c) for c in order[j, : int(psi[j])] if c >= 0]
 
 
 def completed_sets(order: np.ndarray, psi, N: int) -> list[list[int]]:

@@ -1,0 +1,340 @@
+"""ctypes binding of libgc.so (argument marshalling only).
+
+Tensors passed to device entry points must be contiguous CUDA tensors of the
+dtype the C header states; outputs not supplied by the caller are allocated
+with torch.  Calls are asynchronous on torch's current stream, like the C
+functions; gc_status() synchronises and reports device-detected data errors.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+import numpy as np
+import torch  # loads the CUDA runtime libgc.so links against
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+library_path = os.path.join(_HERE, "libgc.so")
+if not os.path.exists(library_path):
+    raise ImportError(
+        f"{library_path} is missing: build it with `python -c 'import __graft_entry__ as g; g.build()'`"
+        " (the gradient-coding path has no fallback without the CUDA library)")
+lib = ctypes.CDLL(library_path)
+
+GC_CYCLIC, GC_EXPLICIT = 0, 1
+GC_F32, GC_BF16 = 0, 1
+GC_LSQ, GC_LOGISTIC = 0, 1
+
+_i, _sz, _p, _d, _f, _i64 = (ctypes.c_int, ctypes.c_size_t, ctypes.c_void_p, ctypes.c_double,
+                             ctypes.c_float, ctypes.c_int64)
+
+
+def _sig(name, res, *args):
+    fn = getattr(lib, name)
+    fn.restype = res
+    fn.argtypes = list(args)
+    return fn
+
+
+_sig("gc_last_error", ctypes.c_char_p)
+_sig("gc_version", _i)
+_sig("gc_kernel_launches", ctypes.c_uint64)
+_sig("gc_workspace_init", _i, _p, _sz, _p)
+_sig("gc_status", _i, _p, _p)
+_sig("gc_make_assignment", _i, _i, _i, _i, _i, _p, _p, _p, _p)
+_sig("gc_chunk_grads_workspace", _sz, _i, _i, _i, _i)
+_sig("gc_chunk_grads", _i, _p, _i, _p, _p, _i, _i, _i, _i, _p, _p, _p, _sz, _p)
+_sig("gc_coeff_workspace", _sz, _i, _i, _i, _i, _i)
+_sig("gc_find_encoding_coeff", _i, _p, _i, _p, _i, _i, _i, _p, _i, _p, _p, _p, _p, _p, _p, _p,
+     _sz, _p)
+_sig("gc_encode_workspace", _sz, _i, _i, _i, _i, _i, _i)
+_sig("gc_encode", _i, _p, _i, _p, _i, _i, _i, _p, _i, _p, _i, _p, _p, _sz, _p)
+_sig("gc_decode_tx", _i, _p, _i, _i, _p, _i, _i, _p, _p)
+_sig("gc_decode_batch_workspace", _sz, _i, _i, _i, _i, _i, _i)
+_sig("gc_decode_batch", _i, _p, _i, _p, _i, _i, _i, _p, _i, _p, _i, _p, _p, _p, _p, _p, _sz, _p)
+_sig("gc_decode_combine_workspace", _sz, _i, _i, _i, _i)
+_sig("gc_decode_combine", _i, _p, _i, _i, _i, _p, _i, _p, _p, _p, _sz, _p)
+_sig("gc_mse_workspace", _sz, _i, _i, _i, _i, _i, _i)
+_sig("gc_mse", _i, _p, _i, _p, _i, _i, _i, _p, _i, _p, _i, _p, _p, _p, _p, _sz, _p)
+_sig("gc_sgd_step", _i, _p, _p, _i, _f, _i64, _p)
+
+
+class GCError(RuntimeError):
+    def __init__(self, code: int, msg: str):
+        super().__init__(f"gc error {code}: {msg}")
+        self.code = code
+
+
+def gc_last_error() -> str:
+    return lib.gc_last_error().decode()
+
+
+def gc_version() -> int:
+    return lib.gc_version()
+
+
+def _check(rc: int) -> None:
+    if rc != 0:
+        raise GCError(rc, gc_last_error())
+
+
+def block_length(d: int, ell: int) -> int:
+    return -(-d // ell)
+
+
+def _stream() -> int:
+    return torch.cuda.current_stream().cuda_stream
+
+
+def _dev(t, dtype, name, shape=None):
+    """Device pointer of a contiguous CUDA tensor of the given dtype (None -> NULL)."""
+    if t is None:
+        return None
+    if not isinstance(t, torch.Tensor) or not t.is_cuda:
+        raise TypeError(f"{name} must be a CUDA tensor")
+    if t.dtype != dtype:
+        raise TypeError(f"{name} must be {dtype}, got {t.dtype}")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    if shape is not None and tuple(t.shape) != tuple(shape):
+        raise ValueError(f"{name} has shape {tuple(t.shape)}, expected {tuple(shape)}")
+    return t.data_ptr()
+
+
+class Workspace:
+    """Reusable device scratch buffer; grows on demand.  Its 256-byte status
+    header is zeroed whenever a new buffer is allocated."""
+
+    def __init__(self, device=None):
+        self.device = torch.device(device) if device is not None else torch.device("cuda")
+        self.buf = None
+
+    def get(self, nbytes: int):
+        nbytes = max(int(nbytes), 256)
+        if self.buf is None or self.buf.numel() < nbytes:
+            self.buf = None
+            self.buf = torch.empty(nbytes, dtype=torch.uint8, device=self.device)
+            _check(lib.gc_workspace_init(self.buf.data_ptr(), nbytes, _stream()))
+        return self.buf.data_ptr(), self.buf.numel()
+
+    def status(self) -> None:
+        if self.buf is not None:
+            _check(lib.gc_status(self.buf.data_ptr(), _stream()))
+
+
+def _ws(ws, nbytes, device):
+    if ws is None:
+        ws = Workspace(device)
+    return ws, ws.get(nbytes)
+
+
+def gc_status(ws: Workspace) -> None:
+    """Synchronise and raise GCError if a kernel flagged bad data or a timeout."""
+    ws.status()
+
+
+# ---------------------------------------------------------------- assignment
+def gc_make_assignment(N: int, m: int, delta: int, kind: int = GC_CYCLIC, explicit_order=None):
+    """Host-only: (A N x m uint8, order m x delta int32, O N x m uint8) numpy arrays."""
+    A = np.zeros((N, m), dtype=np.uint8)
+    O = np.zeros((N, m), dtype=np.uint8)
+    order = np.zeros((m, delta), dtype=np.int32)
+    ex = None
+    if explicit_order is not None:
+        ex = np.ascontiguousarray(explicit_order, dtype=np.int32)
+        if ex.shape != (m, delta):
+            raise ValueError("explicit_order must be m x delta")
+    _check(lib.gc_make_assignment(N, m, delta, kind, None if ex is None else ex.ctypes.data,
+                                  A.ctypes.data, order.ctypes.data, O.ctypes.data))
+    return A, order, O
+
+
+# ---------------------------------------------------------------- chunk gradients
+def gc_chunk_grads_workspace(N, n_c, d, x_dtype):
+    return lib.gc_chunk_grads_workspace(N, n_c, d, x_dtype)
+
+
+def gc_chunk_grads(X, y, w, N: int, n_c: int, loss: int, G=None, loss_out=None,
+                   ws: Workspace | None = None):
+    """G (N x d float32) = per-chunk gradients; loss_out (1 float64) optional."""
+    d = X.shape[1]
+    x_dtype = GC_BF16 if X.dtype == torch.bfloat16 else GC_F32
+    if X.dtype not in (torch.float32, torch.bfloat16):
+        raise TypeError("X must be float32 or bfloat16")
+    if X.shape[0] != N * n_c:
+        raise ValueError("X must have N * n_c rows")
+    if G is None:
+        G = torch.empty(N, d, dtype=torch.float32, device=X.device)
+    ws, (wp, wn) = _ws(ws, gc_chunk_grads_workspace(N, n_c, d, x_dtype), X.device)
+    _check(lib.gc_chunk_grads(_dev(X, X.dtype, "X"), x_dtype, _dev(y, torch.float32, "y", (N * n_c,)),
+                              _dev(w, torch.float32, "w", (d,)), N, n_c, d, loss,
+                              _dev(G, torch.float32, "G", (N, d)),
+                              _dev(loss_out, torch.float64, "loss_out"), wp, wn, _stream()))
+    return G
+
+
+# ---------------------------------------------------------------- Algorithm 1
+def gc_coeff_workspace(N, m, delta, ell, npat):
+    return lib.gc_coeff_workspace(N, m, delta, ell, npat)
+
+
+def gc_find_encoding_coeff(R, ell, order, N, m, delta, psi, E=True, C=True, delta_out=True,
+                           support=False, coef_err=True, est=True, ws: Workspace | None = None):
+    """Batched Algorithm 1.  Boolean arguments request an output (allocated
+    here); tensors are used as given.  Returns a dict of the outputs."""
+    npat = psi.shape[0]
+    dev = psi.device
+
+    def out(flag, shape, dtype):
+        if isinstance(flag, torch.Tensor):
+            return flag
+        return torch.empty(shape, dtype=dtype, device=dev) if flag else None
+
+    res = {
+        "E": out(E, (npat, m, delta, ell), torch.float64),
+        "C": out(C, (npat, ell, N * ell), torch.float32),
+        "delta": out(delta_out, (npat, N), torch.uint8),
+        "support": out(support, (npat, N, m), torch.uint8),
+        "coef_err": out(coef_err, (npat,), torch.float64),
+        "est": out(est, (npat,), torch.float64),
+    }
+    ws, (wp, wn) = _ws(ws, gc_coeff_workspace(N, m, delta, ell, npat), dev)
+    _check(lib.gc_find_encoding_coeff(
+        _dev(R, torch.float64, "R", (ell, m)), ell, _dev(order, torch.int32, "order", (m, delta)),
+        N, m, delta, _dev(psi, torch.int32, "psi", (npat, m)), npat,
+        _dev(res["E"], torch.float64, "E"), _dev(res["C"], torch.float32, "C"),
+        _dev(res["delta"], torch.uint8, "delta_out"), _dev(res["support"], torch.uint8, "support"),
+        _dev(res["coef_err"], torch.float64, "coef_err"), _dev(res["est"], torch.float64, "est"),
+        wp, wn, _stream()))
+    return res
+
+
+# ---------------------------------------------------------------- encode / decode
+def gc_encode_workspace(N, m, delta, ell, npat, d):
+    return lib.gc_encode_workspace(N, m, delta, ell, npat, d)
+
+
+def gc_encode(R, ell, order, N, m, delta, psi, G, T=None, ws: Workspace | None = None):
+    """Worker transmissions T (npat x m x L float32), eq. (2)."""
+    npat = psi.shape[0]
+    d = G.shape[1]
+    L = block_length(d, ell)
+    if T is None:
+        T = torch.empty(npat, m, L, dtype=torch.float32, device=G.device)
+    ws, (wp, wn) = _ws(ws, gc_encode_workspace(N, m, delta, ell, npat, d), G.device)
+    _check(lib.gc_encode(_dev(R, torch.float64, "R", (ell, m)), ell,
+                         _dev(order, torch.int32, "order", (m, delta)), N, m, delta,
+                         _dev(psi, torch.int32, "psi", (npat, m)), npat,
+                         _dev(G, torch.float32, "G", (N, d)), d,
+                         _dev(T, torch.float32, "T", (npat, m, L)), wp, wn, _stream()))
+    return T
+
+
+def gc_decode_tx(R, ell, m, T, d, ghat=None):
+    """PS decode of transmissions: ghat (npat x d float32)."""
+    npat = T.shape[0]
+    L = block_length(d, ell)
+    if ghat is None:
+        ghat = torch.empty(npat, d, dtype=torch.float32, device=T.device)
+    _check(lib.gc_decode_tx(_dev(R, torch.float64, "R", (ell, m)), ell, m,
+                            _dev(T, torch.float32, "T", (npat, m, L)), npat, d,
+                            _dev(ghat, torch.float32, "ghat", (npat, d)), _stream()))
+    return ghat
+
+
+def gc_decode_batch_workspace(N, m, delta, ell, npat, d):
+    return lib.gc_decode_batch_workspace(N, m, delta, ell, npat, d)
+
+
+def gc_decode_batch(R, ell, order, N, m, delta, psi, G, Ghat=True, coef_err=True, est=True,
+                    grad_mse=True, ws: Workspace | None = None):
+    """Batched decode-combine.  Returns dict with Ghat (npat x d float32 or
+    None), coef_err, est, grad_mse (npat float64 or None)."""
+    npat = psi.shape[0]
+    d = G.shape[1]
+    dev = G.device
+
+    def out(flag, shape, dtype):
+        if isinstance(flag, torch.Tensor):
+            return flag
+        return torch.empty(shape, dtype=dtype, device=dev) if flag else None
+
+    res = {
+        "Ghat": out(Ghat, (npat, d), torch.float32),
+        "coef_err": out(coef_err, (npat,), torch.float64),
+        "est": out(est, (npat,), torch.float64),
+        "grad_mse": out(grad_mse, (npat,), torch.float64),
+    }
+    ws, (wp, wn) = _ws(ws, gc_decode_batch_workspace(N, m, delta, ell, npat, d), dev)
+    _check(lib.gc_decode_batch(
+        _dev(R, torch.float64, "R", (ell, m)), ell, _dev(order, torch.int32, "order", (m, delta)),
+        N, m, delta, _dev(psi, torch.int32, "psi", (npat, m)), npat,
+        _dev(G, torch.float32, "G", (N, d)), d, _dev(res["Ghat"], torch.float32, "Ghat", (npat, d)),
+        _dev(res["coef_err"], torch.float64, "coef_err"), _dev(res["est"], torch.float64, "est"),
+        _dev(res["grad_mse"], torch.float64, "grad_mse"), wp, wn, _stream()))
+    return res
+
+
+def gc_kernel_launches() -> int:
+    return int(lib.gc_kernel_launches())
+
+
+def gc_decode_combine_workspace(N, ell, npat, d):
+    return lib.gc_decode_combine_workspace(N, ell, npat, d)
+
+
+def gc_decode_combine(C, ell, N, G, Ghat=True, grad_mse=True, ws: Workspace | None = None):
+    """Ghat (npat x d) = C . G for a decode matrix C (npat x ell x N*ell) from
+    gc_find_encoding_coeff; grad_mse optional."""
+    npat = C.shape[0]
+    d = G.shape[1]
+    dev = G.device
+    if not isinstance(Ghat, torch.Tensor):
+        Ghat = torch.empty(npat, d, dtype=torch.float32, device=dev) if Ghat else None
+    if not isinstance(grad_mse, torch.Tensor):
+        grad_mse = torch.empty(npat, dtype=torch.float64, device=dev) if grad_mse else None
+    ws, (wp, wn) = _ws(ws, gc_decode_combine_workspace(N, ell, npat, d), dev)
+    _check(lib.gc_decode_combine(_dev(C, torch.float32, "C", (npat, ell, N * ell)), ell, N, npat,
+                                 _dev(G, torch.float32, "G", (N, d)), d,
+                                 _dev(Ghat, torch.float32, "Ghat", (npat, d)),
+                                 _dev(grad_mse, torch.float64, "grad_mse"), wp, wn, _stream()))
+    return {"Ghat": Ghat, "grad_mse": grad_mse}
+
+
+def gc_mse_workspace(N, m, delta, ell, npat, d):
+    return lib.gc_mse_workspace(N, m, delta, ell, npat, d)
+
+
+def gc_mse(R, ell, order, N, m, delta, psi, G, coef_err=True, est=True, grad_mse=True,
+           ws: Workspace | None = None):
+    """Error measures only; decoded gradients are never written."""
+    npat = psi.shape[0]
+    d = G.shape[1]
+    dev = G.device
+
+    def out(flag, shape, dtype):
+        if isinstance(flag, torch.Tensor):
+            return flag
+        return torch.empty(shape, dtype=dtype, device=dev) if flag else None
+
+    res = {
+        "coef_err": out(coef_err, (npat,), torch.float64),
+        "est": out(est, (npat,), torch.float64),
+        "grad_mse": out(grad_mse, (npat,), torch.float64),
+    }
+    ws, (wp, wn) = _ws(ws, gc_mse_workspace(N, m, delta, ell, npat, d), dev)
+    _check(lib.gc_mse(
+        _dev(R, torch.float64, "R", (ell, m)), ell, _dev(order, torch.int32, "order", (m, delta)),
+        N, m, delta, _dev(psi, torch.int32, "psi", (npat, m)), npat,
+        _dev(G, torch.float32, "G", (N, d)), d, _dev(res["coef_err"], torch.float64, "coef_err"),
+        _dev(res["est"], torch.float64, "est"), _dev(res["grad_mse"], torch.float64, "grad_mse"),
+        wp, wn, _stream()))
+    return res
+
+
+def gc_sgd_step(w, ghat, lr: float, Ntil: int):
+    """w -= lr * ghat / N~ in place."""
+    d = w.shape[0]
+    _check(lib.gc_sgd_step(_dev(w, torch.float32, "w", (d,)), _dev(ghat, torch.float32, "ghat", (d,)),
+                           d, float(lr), int(Ntil), _stream()))
+    return w

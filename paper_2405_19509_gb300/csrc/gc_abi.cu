@@ -1,0 +1,345 @@
+// extern "C" entry points of libgc.so: validation, workspace layout, launches.
+// Every entry point validates on the host before launching anything and
+// returns a GC_* status; the text of the last error is thread-local.
+#include <stdarg.h>
+#include <stdio.h>
+#include <string.h>
+
+#include <algorithm>
+#include <atomic>
+#include <vector>
+
+#include "gc_internal.cuh"
+
+namespace gc {
+
+static thread_local char g_err[512] = "";
+
+int fail(int code, const char* fmt, ...) {
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(g_err, sizeof(g_err), fmt, ap);
+  va_end(ap);
+  return code;
+}
+
+int cuda_check(cudaError_t e, const char* what) {
+  if (e == cudaSuccess) return GC_OK;
+  return fail(GC_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
+}
+
+static std::atomic<uint64_t> g_launches{0};
+void count_launches(int n) { g_launches.fetch_add((uint64_t)n, std::memory_order_relaxed); }
+
+int device_sm_count() {
+  int dev = 0, n = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return 152;
+  if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0)
+    return 152;
+  return n;
+}
+
+namespace {
+
+cudaStream_t as_stream(void* s) { return static_cast<cudaStream_t>(s); }
+
+int check_ws(void* ws, size_t ws_bytes, size_t need) {
+  if (!ws) return fail(GC_ERR_WORKSPACE, "workspace is NULL (need %zu bytes)", need);
+  if (reinterpret_cast<uintptr_t>(ws) % 256 != 0)
+    return fail(GC_ERR_WORKSPACE, "workspace must be 256-byte aligned");
+  if (ws_bytes < need)
+    return fail(GC_ERR_WORKSPACE, "workspace too small: %zu < %zu bytes", ws_bytes, need);
+  return GC_OK;
+}
+
+int check_dims(int N, int m, int delta, int ell, int npat) {
+  if (N < 1 || m < 1) return fail(GC_ERR_SHAPE, "N=%d and m=%d must be >= 1", N, m);
+  if (m > 32767) return fail(GC_ERR_UNSUPPORTED, "m=%d exceeds 32767", m);
+  if (delta < 1) return fail(GC_ERR_SHAPE, "delta=%d must be >= 1", delta);
+  if (delta > GC_MAX_DELTA) return fail(GC_ERR_UNSUPPORTED, "delta=%d exceeds %d", delta, GC_MAX_DELTA);
+  if (ell < 1) return fail(GC_ERR_SHAPE, "ell=%d must be >= 1", ell);
+  if (ell > GC_MAX_ELL) return fail(GC_ERR_UNSUPPORTED, "ell=%d exceeds %d", ell, GC_MAX_ELL);
+  if (npat < 0) return fail(GC_ERR_SHAPE, "npat=%d must be >= 0", npat);
+  if ((long long)N * ell > (1LL << 30)) return fail(GC_ERR_UNSUPPORTED, "N*ell too large");
+  return GC_OK;
+}
+
+// Workspace layout of the pattern solve: holders, then the memo table.
+struct SolveWs {
+  Holders h;
+  void* table;
+  int bits;
+};
+SolveWs carve_solve(Carve& c, int N, int m, int delta, int ell, int npat) {
+  SolveWs s;
+  s.h = carve_holders(c, N);
+  s.bits = solve_table_bits(N, m, delta, npat);
+  const size_t tb = solve_table_bytes(N, ell, s.bits);
+  s.table = tb ? c.take<char>(tb) : nullptr;
+  return s;
+}
+
+uint32_t* status_of(void* ws) { return static_cast<uint32_t*>(ws); }
+
+}  // namespace
+}  // namespace gc
+
+using namespace gc;
+
+extern "C" {
+
+const char* gc_last_error(void) { return g_err; }
+
+int gc_version(void) { return 100; }
+
+uint64_t gc_kernel_launches(void) { return g_launches.load(); }
+
+int gc_workspace_init(void* ws, size_t ws_bytes, void* stream) {
+  if (!ws || ws_bytes < kHeaderBytes) return fail(GC_ERR_WORKSPACE, "workspace missing or < 256 bytes");
+  GC_CUDA(cudaMemsetAsync(ws, 0, kHeaderBytes, as_stream(stream)));
+  return GC_OK;
+}
+
+int gc_status(void* ws, void* stream) {
+  if (!ws) return fail(GC_ERR_WORKSPACE, "workspace is NULL");
+  WsHeader h{};
+  GC_CUDA(cudaStreamSynchronize(as_stream(stream)));
+  GC_CUDA(cudaMemcpy(&h, ws, sizeof(h), cudaMemcpyDeviceToHost));
+  GC_CUDA(cudaMemset(ws, 0, sizeof(h)));
+  if (h.status & ST_TIMEOUT)
+    return fail(GC_ERR_TIMEOUT, "a bounded device wait expired (status 0x%x)", h.status);
+  if (h.status & (ST_BAD_PSI | ST_SINGULAR | ST_BAD_ORDER)) {
+    return fail(GC_ERR_DATA, "device reported:%s%s%s", (h.status & ST_BAD_PSI) ? " psi outside [0, delta];" : "",
+                (h.status & ST_SINGULAR) ? " rank-deficient least-squares system;" : "",
+                (h.status & ST_BAD_ORDER) ? " invalid order entry or too many copies of a chunk;" : "");
+  }
+  return GC_OK;
+}
+
+int gc_make_assignment(int N, int m, int delta, int kind, const int32_t* explicit_order_h,
+                       uint8_t* A_h, int32_t* order_h, uint8_t* O_h) {
+  if (N < 1 || m < 1 || delta < 1) return fail(GC_ERR_SHAPE, "N, m, delta must be >= 1");
+  if (delta > GC_MAX_DELTA) return fail(GC_ERR_UNSUPPORTED, "delta=%d exceeds %d", delta, GC_MAX_DELTA);
+  if (delta > N) return fail(GC_ERR_SHAPE, "delta=%d exceeds N=%d", delta, N);
+  std::vector<int32_t> order((size_t)m * delta, -1);
+  if (kind == GC_CYCLIC) {
+    if (N != m) return fail(GC_ERR_SHAPE, "cyclic assignment needs N == m (N=%d, m=%d)", N, m);
+    for (int j = 0; j < m; ++j)
+      for (int p = 0; p < delta; ++p) order[(size_t)j * delta + p] = (j + p) % N;
+  } else if (kind == GC_EXPLICIT) {
+    if (!explicit_order_h) return fail(GC_ERR_ARG, "explicit_order_h is NULL");
+    std::vector<int> copies(N, 0);
+    std::vector<char> seen(N, 0);
+    for (int j = 0; j < m; ++j) {
+      std::fill(seen.begin(), seen.end(), 0);
+      bool ended = false;
+      for (int p = 0; p < delta; ++p) {
+        const int v = explicit_order_h[(size_t)j * delta + p];
+        if (v == -1) {
+          ended = true;
+          continue;
+        }
+        if (v < -1 || v >= N) return fail(GC_ERR_ARG, "order[%d][%d]=%d outside [-1, N)", j, p, v);
+        if (ended) return fail(GC_ERR_ARG, "order[%d]: chunk after an empty slot", j);
+        if (seen[v]) return fail(GC_ERR_ARG, "order[%d]: chunk %d twice", j, v);
+        seen[v] = 1;
+        if (++copies[v] > GC_MAX_REPL)
+          return fail(GC_ERR_UNSUPPORTED, "chunk %d has more than %d copies", v, GC_MAX_REPL);
+        order[(size_t)j * delta + p] = v;
+      }
+    }
+  } else {
+    return fail(GC_ERR_ARG, "unknown assignment kind %d", kind);
+  }
+  if (A_h) memset(A_h, 0, (size_t)N * m);
+  if (O_h) memset(O_h, 0, (size_t)N * m);
+  for (int j = 0; j < m; ++j)
+    for (int p = 0; p < delta; ++p) {
+      const int v = order[(size_t)j * delta + p];
+      if (v < 0) continue;
+      if (A_h) A_h[(size_t)v * m + j] = 1;
+      if (O_h) O_h[(size_t)v * m + j] = (uint8_t)(p + 1);
+    }
+  if (order_h) memcpy(order_h, order.data(), order.size() * sizeof(int32_t));
+  return GC_OK;
+}
+
+// ---------------------------------------------------------------- chunk grads
+size_t gc_chunk_grads_workspace(int N, int n_c, int d, int x_dtype) {
+  if (N < 1 || n_c < 1 || d < 1) return 0;
+  return kHeaderBytes + chunkgrad_ws_bytes(N, n_c, d, x_dtype);
+}
+
+int gc_chunk_grads(const void* X, int x_dtype, const float* y, const float* w, int N, int n_c,
+                   int d, int loss, float* G, double* loss_out, void* ws, size_t ws_bytes,
+                   void* stream) {
+  if (!X || !y || !w || !G) return fail(GC_ERR_ARG, "X, y, w and G must be non-NULL");
+  if (x_dtype != GC_F32 && x_dtype != GC_BF16) return fail(GC_ERR_ARG, "x_dtype=%d", x_dtype);
+  if (loss != GC_LSQ && loss != GC_LOGISTIC) return fail(GC_ERR_ARG, "loss=%d", loss);
+  if (N < 1 || n_c < 1 || d < 1) return fail(GC_ERR_SHAPE, "N, n_c, d must be >= 1");
+  if ((long long)N * n_c > (1LL << 40)) return fail(GC_ERR_SHAPE, "N*n_c too large");
+  int rc = check_ws(ws, ws_bytes, gc_chunk_grads_workspace(N, n_c, d, x_dtype));
+  if (rc) return rc;
+  Carve c(ws);
+  return launch_chunkgrad(X, x_dtype, y, w, N, n_c, d, loss, G, loss_out, c, status_of(ws),
+                          as_stream(stream));
+}
+
+// ---------------------------------------------------------------- Algorithm 1
+size_t gc_coeff_workspace(int N, int m, int delta, int ell, int npat) {
+  if (check_dims(N, m, delta, ell, npat)) return 0;
+  Carve c(nullptr);
+  carve_solve(c, N, m, delta, ell, npat);
+  return c.bytes();
+}
+
+int gc_find_encoding_coeff(const double* R, int ell, const int32_t* order, int N, int m, int delta,
+                           const int32_t* psi, int npat, double* E, float* C, uint8_t* delta_out,
+                           uint8_t* support, double* coef_err, double* est, void* ws,
+                           size_t ws_bytes, void* stream) {
+  int rc = check_dims(N, m, delta, ell, npat);
+  if (rc) return rc;
+  if (!R || !order || (!psi && npat > 0)) return fail(GC_ERR_ARG, "R, order and psi must be non-NULL");
+  rc = check_ws(ws, ws_bytes, gc_coeff_workspace(N, m, delta, ell, npat));
+  if (rc) return rc;
+  if (npat == 0) return GC_OK;
+  cudaStream_t s = as_stream(stream);
+  Carve c(ws);
+  SolveWs sw = carve_solve(c, N, m, delta, ell, npat);
+  launch_holders(order, N, m, delta, sw.h, status_of(ws), s);
+  SolveOut out{E, C, delta_out, support, coef_err, est};
+  return launch_solve_impl(R, ell, psi, sw.h, N, m, delta, npat, out, sw.table, sw.bits,
+                           status_of(ws), s);
+}
+
+// ---------------------------------------------------------------- encode
+size_t gc_encode_workspace(int N, int m, int delta, int ell, int npat, int d) {
+  if (check_dims(N, m, delta, ell, npat) || d < 1) return 0;
+  Carve c(nullptr);
+  carve_solve(c, N, m, delta, ell, npat);
+  c.take<double>((size_t)npat * m * delta * ell);
+  return c.bytes();
+}
+
+int gc_encode(const double* R, int ell, const int32_t* order, int N, int m, int delta,
+              const int32_t* psi, int npat, const float* G, int d, float* T, void* ws,
+              size_t ws_bytes, void* stream) {
+  int rc = check_dims(N, m, delta, ell, npat);
+  if (rc) return rc;
+  if (d < 1) return fail(GC_ERR_SHAPE, "d=%d must be >= 1", d);
+  if (!R || !order || !G || !T || (!psi && npat > 0))
+    return fail(GC_ERR_ARG, "R, order, psi, G and T must be non-NULL");
+  rc = check_ws(ws, ws_bytes, gc_encode_workspace(N, m, delta, ell, npat, d));
+  if (rc) return rc;
+  if (npat == 0) return GC_OK;
+  cudaStream_t s = as_stream(stream);
+  Carve c(ws);
+  SolveWs sw = carve_solve(c, N, m, delta, ell, npat);
+  double* E = c.take<double>((size_t)npat * m * delta * ell);
+  launch_holders(order, N, m, delta, sw.h, status_of(ws), s);
+  SolveOut out{E, nullptr, nullptr, nullptr, nullptr, nullptr};
+  rc = launch_solve_impl(R, ell, psi, sw.h, N, m, delta, npat, out, sw.table, sw.bits,
+                         status_of(ws), s);
+  if (rc) return rc;
+  return launch_encode(E, order, psi, N, m, delta, ell, npat, G, d, T, s);
+}
+
+int gc_decode_tx(const double* R, int ell, int m, const float* T, int npat, int d, float* ghat,
+                 void* stream) {
+  if (!R || !T || !ghat) return fail(GC_ERR_ARG, "R, T and ghat must be non-NULL");
+  if (m < 1 || npat < 0 || d < 1) return fail(GC_ERR_SHAPE, "m, d >= 1 and npat >= 0 required");
+  if (ell < 1) return fail(GC_ERR_SHAPE, "ell=%d must be >= 1", ell);
+  if (ell > GC_MAX_ELL) return fail(GC_ERR_UNSUPPORTED, "ell=%d exceeds %d", ell, GC_MAX_ELL);
+  return launch_decode_tx(R, ell, m, T, npat, d, ghat, as_stream(stream));
+}
+
+// ---------------------------------------------------------------- decode batch / mse
+size_t gc_decode_batch_workspace(int N, int m, int delta, int ell, int npat, int d) {
+  if (check_dims(N, m, delta, ell, npat) || d < 1) return 0;
+  Carve c(nullptr);
+  carve_solve(c, N, m, delta, ell, npat);
+  c.take<float>((size_t)npat * ell * N * ell);  // C
+  c.take<float>((size_t)d);                      // sum of chunk gradients
+  c.take<char>(combine_ws_bytes(N, ell, npat, d));
+  return c.bytes();
+}
+
+int gc_decode_batch(const double* R, int ell, const int32_t* order, int N, int m, int delta,
+                    const int32_t* psi, int npat, const float* G, int d, float* Ghat,
+                    double* coef_err, double* est, double* grad_mse, void* ws, size_t ws_bytes,
+                    void* stream) {
+  int rc = check_dims(N, m, delta, ell, npat);
+  if (rc) return rc;
+  if (d < 1) return fail(GC_ERR_SHAPE, "d=%d must be >= 1", d);
+  if (!R || !order || !G || (!psi && npat > 0))
+    return fail(GC_ERR_ARG, "R, order, psi and G must be non-NULL");
+  if (npat == 0) return GC_OK;
+  if (!Ghat && !grad_mse) return fail(GC_ERR_ARG, "Ghat and grad_mse are both NULL");
+  rc = check_ws(ws, ws_bytes, gc_decode_batch_workspace(N, m, delta, ell, npat, d));
+  if (rc) return rc;
+  if (npat == 0) return GC_OK;
+  cudaStream_t s = as_stream(stream);
+  Carve c(ws);
+  SolveWs sw = carve_solve(c, N, m, delta, ell, npat);
+  float* C = c.take<float>((size_t)npat * ell * N * ell);
+  float* gsum = c.take<float>((size_t)d);
+  launch_holders(order, N, m, delta, sw.h, status_of(ws), s);
+  SolveOut out{nullptr, C, nullptr, nullptr, coef_err, est};
+  rc = launch_solve_impl(R, ell, psi, sw.h, N, m, delta, npat, out, sw.table, sw.bits,
+                         status_of(ws), s);
+  if (rc) return rc;
+  if (grad_mse) {
+    rc = launch_colsum(G, N, d, gsum, s);
+    if (rc) return rc;
+  }
+  return launch_combine(C, G, gsum, N, ell, npat, d, Ghat, grad_mse, c, status_of(ws), s);
+}
+
+size_t gc_decode_combine_workspace(int N, int ell, int npat, int d) {
+  if (N < 1 || ell < 1 || ell > GC_MAX_ELL || npat < 0 || d < 1) return 0;
+  Carve c(nullptr);
+  c.take<float>((size_t)d);
+  c.take<char>(combine_ws_bytes(N, ell, npat, d));
+  return c.bytes();
+}
+
+int gc_decode_combine(const float* C, int ell, int N, int npat, const float* G, int d,
+                      float* Ghat, double* grad_mse, void* ws, size_t ws_bytes, void* stream) {
+  if (N < 1 || npat < 0 || d < 1) return fail(GC_ERR_SHAPE, "N, d >= 1 and npat >= 0 required");
+  if (ell < 1) return fail(GC_ERR_SHAPE, "ell=%d must be >= 1", ell);
+  if (ell > GC_MAX_ELL) return fail(GC_ERR_UNSUPPORTED, "ell=%d exceeds %d", ell, GC_MAX_ELL);
+  if ((long long)N * ell > (1LL << 30)) return fail(GC_ERR_UNSUPPORTED, "N*ell too large");
+  if (!C || !G) return fail(GC_ERR_ARG, "C and G must be non-NULL");
+  if (npat == 0) return GC_OK;
+  if (!Ghat && !grad_mse) return fail(GC_ERR_ARG, "Ghat and grad_mse are both NULL");
+  int rc = check_ws(ws, ws_bytes, gc_decode_combine_workspace(N, ell, npat, d));
+  if (rc) return rc;
+  cudaStream_t s = as_stream(stream);
+  Carve c(ws);
+  float* gsum = c.take<float>((size_t)d);
+  if (grad_mse) {
+    rc = launch_colsum(G, N, d, gsum, s);
+    if (rc) return rc;
+  }
+  return launch_combine(C, G, gsum, N, ell, npat, d, Ghat, grad_mse, c, status_of(ws), s);
+}
+
+size_t gc_mse_workspace(int N, int m, int delta, int ell, int npat, int d) {
+  return gc_decode_batch_workspace(N, m, delta, ell, npat, d);
+}
+
+int gc_mse(const double* R, int ell, const int32_t* order, int N, int m, int delta,
+           const int32_t* psi, int npat, const float* G, int d, double* coef_err, double* est,
+           double* grad_mse, void* ws, size_t ws_bytes, void* stream) {
+  if (!grad_mse && npat > 0) return fail(GC_ERR_ARG, "grad_mse must be non-NULL");
+  return gc_decode_batch(R, ell, order, N, m, delta, psi, npat, G, d, nullptr, coef_err, est,
+                         grad_mse, ws, ws_bytes, stream);
+}
+
+int gc_sgd_step(float* w, const float* ghat, int d, float lr, int64_t Ntil, void* stream) {
+  if (!w || !ghat) return fail(GC_ERR_ARG, "w and ghat must be non-NULL");
+  if (d < 1 || Ntil < 1) return fail(GC_ERR_SHAPE, "d and Ntil must be >= 1");
+  return launch_sgd(w, ghat, d, lr, Ntil, as_stream(stream));
+}
+
+}  // extern "C"

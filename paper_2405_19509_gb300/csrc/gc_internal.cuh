@@ -1,0 +1,104 @@
+// Internal declarations shared by the translation units of libgc.so.
+#pragma once
+
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "gc.h"
+
+namespace gc {
+
+// ---- status header at the start of every workspace ----------------------
+enum : uint32_t {
+  ST_BAD_PSI = 1u,     // psi outside [0, delta]
+  ST_SINGULAR = 2u,    // a least-squares system was numerically rank deficient
+  ST_TIMEOUT = 4u,     // a bounded mbarrier wait expired
+  ST_BAD_ORDER = 8u,   // order entry outside [-1, N) or a chunk with > GC_MAX_REPL copies
+};
+constexpr size_t kHeaderBytes = 256;
+
+struct WsHeader {
+  uint32_t status;
+  uint32_t info;
+};
+
+// ---- error reporting (thread-local, host) --------------------------------
+int fail(int code, const char* fmt, ...);
+int cuda_check(cudaError_t e, const char* what);
+#define GC_CUDA(call)                                   \
+  do {                                                  \
+    cudaError_t e_ = (call);                            \
+    if (e_ != cudaSuccess) return ::gc::cuda_check(e_, #call); \
+  } while (0)
+
+inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+// Linear carving of a caller workspace into 256-byte aligned pieces.
+struct Carve {
+  char* base;
+  size_t off;
+  explicit Carve(void* b) : base(static_cast<char*>(b)), off(kHeaderBytes) {}
+  template <typename T>
+  T* take(size_t count) {
+    T* p = base ? reinterpret_cast<T*>(base + off) : nullptr;
+    off = align_up(off + count * sizeof(T), 256);
+    return p;
+  }
+  size_t bytes() const { return off; }
+};
+
+int device_sm_count();
+
+// Launch accounting for gc_kernel_launches().
+void count_launches(int n);
+
+// ---- holder table: copies of every chunk, sorted by worker --------------
+// hold_w[i*GC_MAX_REPL + h], hold_p[...]: worker and slot of the h-th holder of
+// chunk i (workers ascending, then slot); hold_cnt[i] holders.
+struct Holders {
+  int32_t* cnt;
+  int16_t* w;
+  int8_t* p;
+};
+Holders carve_holders(Carve& c, int N);
+void launch_holders(const int32_t* order, int N, int m, int delta, Holders h, uint32_t* status,
+                    cudaStream_t s);
+
+// ---- Algorithm 1 batched (k_solve.cu) -----------------------------------
+struct SolveOut {
+  double* E;          // npat x m x delta x ell (nullable)
+  float* C;           // npat x ell x N*ell (nullable)
+  uint8_t* delta_out; // npat x N (nullable)
+  uint8_t* support;   // npat x N x m (nullable)
+  double* coef_err;   // npat (nullable)
+  double* est;        // npat (nullable)
+};
+// Memo table of every holder subset (bits = masks per chunk in log2, -1 = none).
+int solve_table_bits(int N, int m, int delta, int npat);
+size_t solve_table_bytes(int N, int ell, int bits);
+int launch_solve_impl(const double* R, int ell, const int32_t* psi, Holders h, int N, int m,
+                      int delta, int npat, SolveOut out, void* table_mem, int bits,
+                      uint32_t* status, cudaStream_t s);
+
+// ---- chunk gradients (k_chunkgrad.cu) -----------------------------------
+size_t chunkgrad_ws_bytes(int N, int n_c, int d, int x_dtype);
+int launch_chunkgrad(const void* X, int x_dtype, const float* y, const float* w, int N, int n_c,
+                     int d, int loss, float* G, double* loss_out, Carve& ws, uint32_t* status,
+                     cudaStream_t s);
+
+// ---- encode / decode / update (k_encode.cu) -----------------------------
+int launch_encode(const double* E, const int32_t* order, const int32_t* psi, int N, int m,
+                  int delta, int ell, int npat, const float* G, int d, float* T, cudaStream_t s);
+int launch_decode_tx(const double* R, int ell, int m, const float* T, int npat, int d, float* ghat,
+                     cudaStream_t s);
+int launch_sgd(float* w, const float* ghat, int d, float lr, int64_t Ntil, cudaStream_t s);
+int launch_colsum(const float* G, int N, int d, float* gsum, cudaStream_t s);
+
+// ---- batched decode-combine (k_combine.cu) ------------------------------
+size_t combine_ws_bytes(int N, int ell, int npat, int d);
+int launch_combine(const float* C, const float* G, const float* gsum, int N, int ell, int npat,
+                   int d, float* Ghat, double* grad_mse, Carve& ws, uint32_t* status,
+                   cudaStream_t s);
+
+}  // namespace gc

@@ -1,0 +1,126 @@
+// Worker encoding (eq. 2), PS decoding of transmissions (Sec. II-B), the
+// parameter update (Sec. I) and the sum of chunk gradients.
+//
+// All four are HBM-bound streaming kernels with coalesced accesses along the
+// block coordinate c (consecutive threads, consecutive columns).
+#include "gc_internal.cuh"
+
+namespace gc {
+
+// T[b][j][c] = sum_{p < psi[b][j]} sum_k E[b][j][p][k] * g_{order[j][p]}[k*L + c]
+// (g zero past d).  One thread per (b, j, c).
+__global__ void k_encode(const double* __restrict__ E, const int32_t* __restrict__ order,
+                         const int32_t* __restrict__ psi, int N, int m, int delta, int ell,
+                         int npat, const float* __restrict__ G, int d, int L,
+                         float* __restrict__ T) {
+  const long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+  const long long tot = (long long)npat * m * L;
+  if (idx >= tot) return;
+  const int c = (int)(idx % L);
+  const long long bj = idx / L;
+  const int j = (int)(bj % m);
+  const int b = (int)(bj / m);
+  int np = psi[(size_t)b * m + j];
+  np = np < 0 ? 0 : (np > delta ? delta : np);  // bad values are flagged by the solve
+  const double* Ej = E + ((size_t)b * m + j) * delta * ell;
+  float acc = 0.f;
+  for (int p = 0; p < np; ++p) {
+    const int i = order[(size_t)j * delta + p];
+    if (i < 0 || i >= N) continue;
+    const float* gi = G + (size_t)i * d;
+    for (int k = 0; k < ell; ++k) {
+      const int col = k * L + c;
+      if (col < d) acc = fmaf((float)Ej[p * ell + k], __ldg(gi + col), acc);
+    }
+  }
+  T[idx] = acc;
+}
+
+int launch_encode(const double* E, const int32_t* order, const int32_t* psi, int N, int m,
+                  int delta, int ell, int npat, const float* G, int d, float* T, cudaStream_t s) {
+  const int L = (d + ell - 1) / ell;
+  const long long tot = (long long)npat * m * L;
+  if (tot == 0) return GC_OK;
+  const int threads = 256;
+  k_encode<<<(unsigned)((tot + threads - 1) / threads), threads, 0, s>>>(E, order, psi, N, m,
+                                                                         delta, ell, npat, G, d, L,
+                                                                         T);
+  count_launches(1);
+  return cuda_check(cudaGetLastError(), "k_encode");
+}
+
+// ghat[b][k*L + c] = sum_j R[k][j] * T[b][j][c].  One thread per (b, c).
+template <int ELL>
+__global__ void k_decode_tx(const double* __restrict__ R, int m, const float* __restrict__ T,
+                            int npat, int d, int L, float* __restrict__ ghat) {
+  const long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+  if (idx >= (long long)npat * L) return;
+  const int c = (int)(idx % L);
+  const int b = (int)(idx / L);
+  float acc[ELL];
+#pragma unroll
+  for (int k = 0; k < ELL; ++k) acc[k] = 0.f;
+  const float* Tb = T + (size_t)b * m * L + c;
+  for (int j = 0; j < m; ++j) {
+    const float t = __ldg(Tb + (size_t)j * L);
+#pragma unroll
+    for (int k = 0; k < ELL; ++k) acc[k] = fmaf((float)__ldg(R + (size_t)k * m + j), t, acc[k]);
+  }
+#pragma unroll
+  for (int k = 0; k < ELL; ++k) {
+    const int col = k * L + c;
+    if (col < d) ghat[(size_t)b * d + col] = acc[k];
+  }
+}
+
+int launch_decode_tx(const double* R, int ell, int m, const float* T, int npat, int d, float* ghat,
+                     cudaStream_t s) {
+  const int L = (d + ell - 1) / ell;
+  const long long tot = (long long)npat * L;
+  if (tot == 0) return GC_OK;
+  const int threads = 256;
+  const unsigned blocks = (unsigned)((tot + threads - 1) / threads);
+  switch (ell) {
+    case 1: k_decode_tx<1><<<blocks, threads, 0, s>>>(R, m, T, npat, d, L, ghat); break;
+    case 2: k_decode_tx<2><<<blocks, threads, 0, s>>>(R, m, T, npat, d, L, ghat); break;
+    case 3: k_decode_tx<3><<<blocks, threads, 0, s>>>(R, m, T, npat, d, L, ghat); break;
+    case 4: k_decode_tx<4><<<blocks, threads, 0, s>>>(R, m, T, npat, d, L, ghat); break;
+    case 5: k_decode_tx<5><<<blocks, threads, 0, s>>>(R, m, T, npat, d, L, ghat); break;
+    case 6: k_decode_tx<6><<<blocks, threads, 0, s>>>(R, m, T, npat, d, L, ghat); break;
+    case 7: k_decode_tx<7><<<blocks, threads, 0, s>>>(R, m, T, npat, d, L, ghat); break;
+    case 8: k_decode_tx<8><<<blocks, threads, 0, s>>>(R, m, T, npat, d, L, ghat); break;
+    default: return fail(GC_ERR_UNSUPPORTED, "ell=%d exceeds GC_MAX_ELL", ell);
+  }
+  count_launches(1);
+  return cuda_check(cudaGetLastError(), "k_decode_tx");
+}
+
+// w[c] -= lr * ghat[c] / N~
+__global__ void k_sgd(float* __restrict__ w, const float* __restrict__ ghat, int d, float scale) {
+  const int c = blockIdx.x * blockDim.x + threadIdx.x;
+  if (c < d) w[c] = fmaf(-scale, ghat[c], w[c]);
+}
+
+int launch_sgd(float* w, const float* ghat, int d, float lr, int64_t Ntil, cudaStream_t s) {
+  const float scale = (float)((double)lr / (double)Ntil);
+  k_sgd<<<(d + 255) / 256, 256, 0, s>>>(w, ghat, d, scale);
+  count_launches(1);
+  return cuda_check(cudaGetLastError(), "k_sgd");
+}
+
+// gsum[c] = sum_i G[i][c], chunks in increasing order.
+__global__ void k_colsum(const float* __restrict__ G, int N, int d, float* __restrict__ gsum) {
+  const int c = blockIdx.x * blockDim.x + threadIdx.x;
+  if (c >= d) return;
+  float s = 0.f;
+  for (int i = 0; i < N; ++i) s += __ldg(G + (size_t)i * d + c);
+  gsum[c] = s;
+}
+
+int launch_colsum(const float* G, int N, int d, float* gsum, cudaStream_t s) {
+  k_colsum<<<(d + 255) / 256, 256, 0, s>>>(G, N, d, gsum);
+  count_launches(1);
+  return cuda_check(cudaGetLastError(), "k_colsum");
+}
+
+}  // namespace gc

@@ -1,0 +1,564 @@
+// Algorithm 1 (Find-Encoding-Coeff), batched over straggler patterns.
+//
+// For a pattern psi and chunk D_i, S_i is the set of workers that processed
+// D_i and X = R[:, S_i] (ell x Delta_i).  The block column B^(i) restricted to
+// the rows S_i is the minimum-norm least-squares solution X^+ of eq. (6); it
+// separates column by column (Frobenius norm), and every holder of D_i
+// computes the same block (Sec. II).  The decode matrix block is
+// Pi_i = R_{S_i} X^+ = X X^+, the orthogonal projector onto range(X): the
+// identity when Delta_i >= ell (exact recovery, Sec. II-A), rank Delta_i
+// otherwise (approximate GC, eq. 7).
+//
+// Numerics (fp64 throughout):
+//  * Delta >= ell (X has full row rank): X^+ = X^T Lambda with
+//    Lambda = (X X^T)^{-1} from a Cholesky factorisation, followed by one step
+//    of iterative refinement driven by the true residual e_k - X b_k, so the
+//    error is O(eps * kappa(X)) instead of O(eps * kappa^2).
+//  * 0 < Delta < ell (X has full column rank): QR of X by classical
+//    Gram-Schmidt with re-orthogonalisation (CGS2); X^+ = R^{-1} Q^T.
+//  * Delta = 0: X^+ is empty and Pi = 0.
+//
+// GB300 has a low fp64 rate, and Algorithm 1's result for chunk i depends
+// only on (R, S_i), i.e. on which of the chunk's holders finished.  When the
+// number of holder subsets is small compared with the number of (pattern,
+// chunk) problems, every subset is solved once into a table (in the caller's
+// workspace) and each pattern gathers from it; the values are bit-identical
+// to solving the pattern directly, since the same function runs on the same
+// inputs.
+#include <math.h>
+
+#include "gc_internal.cuh"
+
+namespace gc {
+
+// ---------------------------------------------------------------------------
+// Holder table
+// ---------------------------------------------------------------------------
+Holders carve_holders(Carve& c, int N) {
+  Holders h;
+  h.cnt = c.take<int32_t>(N);
+  h.w = c.take<int16_t>((size_t)N * GC_MAX_REPL);
+  h.p = c.take<int8_t>((size_t)N * GC_MAX_REPL);
+  return h;
+}
+
+// One CTA per chunk: scan order[] in (worker, slot) order and compact the
+// matches, which keeps holders sorted by worker then slot.
+__global__ void k_holders(const int32_t* __restrict__ order, int N, int m, int delta, Holders h,
+                          uint32_t* status) {
+  const int i = blockIdx.x;
+  __shared__ int s_warp[32];
+  __shared__ int s_base;
+  if (threadIdx.x == 0) s_base = 0;
+  __syncthreads();
+  const int total = m * delta;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nwarp = blockDim.x >> 5;
+  for (int t0 = 0; t0 < total; t0 += blockDim.x) {
+    const int t = t0 + threadIdx.x;
+    int v = -1;
+    if (t < total) {
+      v = order[t];
+      if ((v < -1 || v >= N) && i == 0) atomicOr(status, ST_BAD_ORDER);
+    }
+    const bool hit = (t < total) && v == i;
+    const unsigned bal = __ballot_sync(0xffffffffu, hit);
+    if (lane == 0) s_warp[warp] = __popc(bal);
+    __syncthreads();
+    int off = s_base;
+    for (int w = 0; w < warp; ++w) off += s_warp[w];
+    off += __popc(bal & ((1u << lane) - 1u));
+    if (hit) {
+      if (off < GC_MAX_REPL) {
+        h.w[(size_t)i * GC_MAX_REPL + off] = (int16_t)(t / delta);
+        h.p[(size_t)i * GC_MAX_REPL + off] = (int8_t)(t % delta);
+      } else {
+        atomicOr(status, ST_BAD_ORDER);
+      }
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      int s = 0;
+      for (int w = 0; w < nwarp; ++w) s += s_warp[w];
+      s_base += s;
+    }
+    __syncthreads();
+  }
+  if (threadIdx.x == 0) h.cnt[i] = s_base < GC_MAX_REPL ? s_base : GC_MAX_REPL;
+}
+
+void launch_holders(const int32_t* order, int N, int m, int delta, Holders h, uint32_t* status,
+                    cudaStream_t s) {
+  k_holders<<<N, 256, 0, s>>>(order, N, m, delta, h, status);
+  count_launches(1);
+}
+
+// ---------------------------------------------------------------------------
+// One least-squares block: chunk i, completion mask over its holders.
+// emit(h, k, v) receives X^+ row of holder h (0 for holders not in S_i).
+// Returns Delta; Pi (ell x ell) and err = ||I - Pi||_F^2 by reference.
+// ---------------------------------------------------------------------------
+template <int ELL, typename Emit>
+__device__ __forceinline__ int solve_block(const double* __restrict__ R, int m, int cnt,
+                                           const int16_t* __restrict__ hw, uint32_t mask,
+                                           double (&Pi)[ELL][ELL], double& err, uint32_t* status,
+                                           Emit emit) {
+  const int D = __popc(mask);
+#pragma unroll
+  for (int a = 0; a < ELL; ++a)
+#pragma unroll
+    for (int k = 0; k < ELL; ++k) Pi[a][k] = 0.0;
+
+  if (D >= ELL) {
+    // Gram matrix M = X X^T (lower triangle) and its Cholesky factor.
+    double Lc[ELL][ELL];
+#pragma unroll
+    for (int a = 0; a < ELL; ++a)
+#pragma unroll
+      for (int c = 0; c < ELL; ++c) Lc[a][c] = 0.0;
+    for (int h = 0; h < cnt; ++h) {
+      if (!((mask >> h) & 1u)) continue;
+      const int j = hw[h];
+      double x[ELL];
+#pragma unroll
+      for (int a = 0; a < ELL; ++a) x[a] = __ldg(R + (size_t)a * m + j);
+#pragma unroll
+      for (int a = 0; a < ELL; ++a)
+#pragma unroll
+        for (int c = 0; c <= a; ++c) Lc[a][c] = fma(x[a], x[c], Lc[a][c]);
+    }
+    bool bad = false;
+#pragma unroll
+    for (int a = 0; a < ELL; ++a) {
+      double s = Lc[a][a];
+#pragma unroll
+      for (int c = 0; c < a; ++c) s -= Lc[a][c] * Lc[a][c];
+      const double ref = Lc[a][a];
+      if (!(s > 1e-26 * ref) || !isfinite(s)) {
+        bad = true;
+        s = ref > 0.0 ? 1e-26 * ref : 1e-300;
+      }
+      const double piv = sqrt(s);
+      Lc[a][a] = piv;
+#pragma unroll
+      for (int r = a + 1; r < ELL; ++r) {
+        double t = Lc[r][a];
+#pragma unroll
+        for (int c = 0; c < a; ++c) t -= Lc[r][c] * Lc[a][c];
+        Lc[r][a] = t / piv;
+      }
+    }
+    if (bad) atomicOr(status, ST_SINGULAR);
+    // Cholesky solve of M Y = Bm in place (column by column).
+    auto chol_solve = [&](double (&Bm)[ELL][ELL]) {
+#pragma unroll
+      for (int k = 0; k < ELL; ++k) {
+        double yv[ELL];
+#pragma unroll
+        for (int a = 0; a < ELL; ++a) {
+          double t = Bm[a][k];
+#pragma unroll
+          for (int c = 0; c < a; ++c) t -= Lc[a][c] * yv[c];
+          yv[a] = t / Lc[a][a];
+        }
+#pragma unroll
+        for (int a = ELL - 1; a >= 0; --a) {
+          double t = yv[a];
+#pragma unroll
+          for (int c = a + 1; c < ELL; ++c) t -= Lc[c][a] * Bm[c][k];
+          Bm[a][k] = t / Lc[a][a];
+        }
+      }
+    };
+    double Lam[ELL][ELL];
+#pragma unroll
+    for (int a = 0; a < ELL; ++a)
+#pragma unroll
+      for (int k = 0; k < ELL; ++k) Lam[a][k] = (a == k) ? 1.0 : 0.0;
+    chol_solve(Lam);
+    // One refinement step on the residual of X b_k = e_k, b_k = X^T Lambda e_k.
+    double Res[ELL][ELL];
+#pragma unroll
+    for (int a = 0; a < ELL; ++a)
+#pragma unroll
+      for (int k = 0; k < ELL; ++k) Res[a][k] = (a == k) ? 1.0 : 0.0;
+    for (int h = 0; h < cnt; ++h) {
+      if (!((mask >> h) & 1u)) continue;
+      const int j = hw[h];
+      double x[ELL];
+#pragma unroll
+      for (int a = 0; a < ELL; ++a) x[a] = __ldg(R + (size_t)a * m + j);
+#pragma unroll
+      for (int k = 0; k < ELL; ++k) {
+        double bk = 0.0;
+#pragma unroll
+        for (int c = 0; c < ELL; ++c) bk = fma(x[c], Lam[c][k], bk);
+#pragma unroll
+        for (int a = 0; a < ELL; ++a) Res[a][k] = fma(-x[a], bk, Res[a][k]);
+      }
+    }
+    chol_solve(Res);
+#pragma unroll
+    for (int a = 0; a < ELL; ++a)
+#pragma unroll
+      for (int k = 0; k < ELL; ++k) Lam[a][k] += Res[a][k];
+    // Coefficients and the projector Pi = X X^+.
+    for (int h = 0; h < cnt; ++h) {
+      if (!((mask >> h) & 1u)) {
+#pragma unroll
+        for (int k = 0; k < ELL; ++k) emit(h, k, 0.0);
+        continue;
+      }
+      const int j = hw[h];
+      double x[ELL];
+#pragma unroll
+      for (int a = 0; a < ELL; ++a) x[a] = __ldg(R + (size_t)a * m + j);
+#pragma unroll
+      for (int k = 0; k < ELL; ++k) {
+        double bk = 0.0;
+#pragma unroll
+        for (int c = 0; c < ELL; ++c) bk = fma(x[c], Lam[c][k], bk);
+        emit(h, k, bk);
+#pragma unroll
+        for (int a = 0; a < ELL; ++a) Pi[a][k] = fma(x[a], bk, Pi[a][k]);
+      }
+    }
+  } else if (D > 0) {
+    constexpr int MQ = ELL > 1 ? ELL - 1 : 1;
+    int jq[MQ];
+    {
+      int q = 0;
+      for (int h = 0; h < cnt; ++h) {
+        if (!((mask >> h) & 1u)) continue;
+#pragma unroll
+        for (int qq = 0; qq < MQ; ++qq)
+          if (qq == q) jq[qq] = hw[h];
+        ++q;
+      }
+    }
+    double Xc[MQ][ELL], Q[MQ][ELL], Rr[MQ][MQ], Xp[MQ][ELL];
+#pragma unroll
+    for (int qq = 0; qq < MQ; ++qq) {
+#pragma unroll
+      for (int r = 0; r < MQ; ++r) Rr[r][qq] = 0.0;
+#pragma unroll
+      for (int a = 0; a < ELL; ++a) {
+        Xc[qq][a] = (qq < D) ? __ldg(R + (size_t)a * m + jq[qq]) : 0.0;
+        Q[qq][a] = 0.0;
+        Xp[qq][a] = 0.0;
+      }
+    }
+    bool bad = false;
+#pragma unroll
+    for (int qq = 0; qq < MQ; ++qq) {
+      if (qq < D) {
+        double v[ELL];
+        double n0 = 0.0;
+#pragma unroll
+        for (int a = 0; a < ELL; ++a) {
+          v[a] = Xc[qq][a];
+          n0 = fma(v[a], v[a], n0);
+        }
+#pragma unroll
+        for (int pass = 0; pass < 2; ++pass) {
+#pragma unroll
+          for (int r = 0; r < MQ; ++r) {
+            if (r < qq) {
+              double dot = 0.0;
+#pragma unroll
+              for (int a = 0; a < ELL; ++a) dot = fma(Q[r][a], v[a], dot);
+#pragma unroll
+              for (int a = 0; a < ELL; ++a) v[a] = fma(-dot, Q[r][a], v[a]);
+              Rr[r][qq] += dot;
+            }
+          }
+        }
+        double nn = 0.0;
+#pragma unroll
+        for (int a = 0; a < ELL; ++a) nn = fma(v[a], v[a], nn);
+        if (!(nn > 1e-26 * n0) || !isfinite(nn)) {
+          bad = true;
+          nn = n0 > 0.0 ? 1e-26 * n0 : 1e-300;
+        }
+        const double nrm = sqrt(nn);
+        Rr[qq][qq] = nrm;
+#pragma unroll
+        for (int a = 0; a < ELL; ++a) Q[qq][a] = v[a] / nrm;
+      }
+    }
+    if (bad) atomicOr(status, ST_SINGULAR);
+    // X^+ = Rr^{-1} Q^T by back substitution.
+#pragma unroll
+    for (int qq = MQ - 1; qq >= 0; --qq) {
+      if (qq < D) {
+#pragma unroll
+        for (int k = 0; k < ELL; ++k) {
+          double t = Q[qq][k];
+#pragma unroll
+          for (int r = qq + 1; r < MQ; ++r)
+            if (r < D) t -= Rr[qq][r] * Xp[r][k];
+          Xp[qq][k] = t / Rr[qq][qq];
+        }
+      }
+    }
+    // Pi = X X^+
+#pragma unroll
+    for (int qq = 0; qq < MQ; ++qq)
+      if (qq < D) {
+#pragma unroll
+        for (int a = 0; a < ELL; ++a)
+#pragma unroll
+          for (int k = 0; k < ELL; ++k) Pi[a][k] = fma(Xc[qq][a], Xp[qq][k], Pi[a][k]);
+      }
+    int q = 0;
+    for (int h = 0; h < cnt; ++h) {
+      const bool in = (mask >> h) & 1u;
+#pragma unroll
+      for (int k = 0; k < ELL; ++k) {
+        double v = 0.0;
+        if (in) {
+#pragma unroll
+          for (int qq = 0; qq < MQ; ++qq)
+            if (qq == q) v = Xp[qq][k];
+        }
+        emit(h, k, v);
+      }
+      if (in) ++q;
+    }
+  } else {
+    for (int h = 0; h < cnt; ++h)
+#pragma unroll
+      for (int k = 0; k < ELL; ++k) emit(h, k, 0.0);
+  }
+  double e = 0.0;
+#pragma unroll
+  for (int a = 0; a < ELL; ++a)
+#pragma unroll
+    for (int k = 0; k < ELL; ++k) {
+      const double t = ((a == k) ? 1.0 : 0.0) - Pi[a][k];
+      e = fma(t, t, e);
+    }
+  err = e;
+  return D;
+}
+
+// ---------------------------------------------------------------------------
+// Table of every holder subset: entry (i, mask) holds X^+ (cnt x ell), Pi and err.
+// ---------------------------------------------------------------------------
+struct Table {
+  int bits;     // masks per chunk = 1 << bits
+  double* xp;   // [N][1<<bits][bits][ell]
+  double* pi;   // [N][1<<bits][ell][ell]
+  double* err;  // [N][1<<bits]
+};
+
+template <int ELL>
+__global__ void __launch_bounds__(128) k_table(const double* __restrict__ R, Holders hd, int N,
+                                              int m, Table tb, uint32_t* status) {
+  const long long e = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+  const long long nent = (long long)N << tb.bits;
+  if (e >= nent) return;
+  const int i = (int)(e >> tb.bits);
+  const uint32_t mask = (uint32_t)(e & ((1LL << tb.bits) - 1));
+  const int cnt = hd.cnt[i];
+  if (cnt > tb.bits) return;  // such chunks are solved directly per pattern
+  if (mask >> cnt) return;    // masks beyond this chunk's holders never occur
+  double Pi[ELL][ELL];
+  double err;
+  double* xp = tb.xp + (size_t)e * tb.bits * ELL;
+  solve_block<ELL>(R, m, cnt, hd.w + (size_t)i * GC_MAX_REPL, mask, Pi, err, status,
+                   [&](int h, int k, double v) { xp[h * ELL + k] = v; });
+  double* pi = tb.pi + (size_t)e * ELL * ELL;
+#pragma unroll
+  for (int a = 0; a < ELL; ++a)
+#pragma unroll
+    for (int k = 0; k < ELL; ++k) pi[a * ELL + k] = Pi[a][k];
+  tb.err[e] = err;
+}
+
+// ---------------------------------------------------------------------------
+// Per (pattern, chunk): completion mask, Delta, then table lookup or direct
+// solve; per-pattern error sums reduced in a fixed order.
+// ---------------------------------------------------------------------------
+template <int ELL, bool TABLE>
+__global__ void __launch_bounds__(256) k_patterns(const double* __restrict__ R,
+                                                 const int32_t* __restrict__ psi, Holders hd,
+                                                 int N, int m, int delta, int npat, int ppb,
+                                                 Table tb, SolveOut out, uint32_t* status) {
+  __shared__ double s_err[256];
+  __shared__ int s_def[256];
+  const int tid = threadIdx.x;
+  int b, i, istep;
+  bool active;
+  if (ppb > 0) {  // N <= 256: ppb patterns per block, one chunk per thread
+    const int lp = tid / N;
+    b = blockIdx.x * ppb + lp;
+    i = tid - lp * N;
+    istep = N;  // single iteration
+    active = (lp < ppb) && (b < npat);
+  } else {  // one pattern per block, threads stride over chunks
+    b = blockIdx.x;
+    i = tid;
+    istep = 256;
+    active = b < npat;
+  }
+  double my_err = 0.0;
+  int my_def = 0;
+  if (active) {
+    const int32_t* ps = psi + (size_t)b * m;
+    for (; i < N; i += istep) {
+      const int cnt = hd.cnt[i];
+      const int16_t* hw = hd.w + (size_t)i * GC_MAX_REPL;
+      const int8_t* hp = hd.p + (size_t)i * GC_MAX_REPL;
+      uint32_t mask = 0;
+      for (int h = 0; h < cnt; ++h) {
+        int v = ps[hw[h]];
+        if (v < 0 || v > delta) {
+          atomicOr(status, ST_BAD_PSI);
+          v = 0;
+        }
+        if (hp[h] < v) mask |= 1u << h;
+      }
+      double Pi[ELL][ELL];
+      double err;
+      int D;
+      double* E = out.E;
+      auto emit = [&](int h, int k, double v) {
+        if (E) E[(((size_t)b * m + hw[h]) * delta + hp[h]) * ELL + k] = v;
+      };
+      if (TABLE && cnt <= tb.bits) {
+        const size_t e = ((size_t)i << tb.bits) | mask;
+        const double* pi = tb.pi + e * ELL * ELL;
+#pragma unroll
+        for (int a = 0; a < ELL; ++a)
+#pragma unroll
+          for (int k = 0; k < ELL; ++k) Pi[a][k] = pi[a * ELL + k];
+        err = tb.err[e];
+        D = __popc(mask);
+        if (E) {
+          const double* xp = tb.xp + e * tb.bits * ELL;
+          for (int h = 0; h < cnt; ++h)
+#pragma unroll
+            for (int k = 0; k < ELL; ++k) emit(h, k, xp[h * ELL + k]);
+        }
+      } else {
+        D = solve_block<ELL>(R, m, cnt, hw, mask, Pi, err, status, emit);
+      }
+      if (out.C) {
+        float* Cb = out.C + (size_t)b * ELL * N * ELL + (size_t)i * ELL;
+#pragma unroll
+        for (int a = 0; a < ELL; ++a)
+#pragma unroll
+          for (int k = 0; k < ELL; ++k) Cb[(size_t)a * N * ELL + k] = (float)Pi[a][k];
+      }
+      if (out.delta_out) out.delta_out[(size_t)b * N + i] = (uint8_t)D;
+      if (out.support) {
+        uint8_t* row = out.support + ((size_t)b * N + i) * m;
+        for (int j = 0; j < m; ++j) row[j] = 0;
+        for (int h = 0; h < cnt; ++h)
+          if ((mask >> h) & 1u) row[hw[h]] = 1;
+      }
+      my_err += err;
+      my_def += D < ELL ? ELL - D : 0;
+    }
+  }
+  s_err[tid] = my_err;
+  s_def[tid] = my_def;
+  __syncthreads();
+  if (!(out.coef_err || out.est)) return;
+  if (ppb > 0) {
+    const int lp = tid / N;
+    if (active && tid - lp * N == 0) {
+      double se = 0.0;
+      int sd = 0;
+      for (int t = 0; t < N; ++t) {
+        se += s_err[tid + t];
+        sd += s_def[tid + t];
+      }
+      if (out.coef_err) out.coef_err[b] = se;
+      if (out.est) out.est[b] = (double)sd;
+    }
+  } else if (tid == 0 && active) {
+    double se = 0.0;
+    int sd = 0;
+    for (int t = 0; t < 256; ++t) {
+      se += s_err[t];
+      sd += s_def[t];
+    }
+    if (out.coef_err) out.coef_err[b] = se;
+    if (out.est) out.est[b] = (double)sd;
+  }
+}
+
+// Table width: masks over the first `bits` holders, bits = delta (the holder
+// count of every chunk under N == m uniform loads).  Chunks with more holders
+// than `bits` (possible with explicit orders) are solved directly.  The table
+// is used when it has no more entries than there are (pattern, chunk)
+// problems and at most 2^14 masks per chunk.
+int solve_table_bits(int N, int m, int delta, int npat) {
+  (void)m;
+  const int bits = delta;
+  if (bits > 14) return -1;
+  if (((long long)N << bits) > (long long)npat * N) return -1;
+  return bits;
+}
+
+size_t solve_table_bytes(int N, int ell, int bits) {
+  if (bits < 0) return 0;
+  const size_t ent = (size_t)N << bits;
+  return align_up(ent * bits * ell * sizeof(double), 256) +
+         align_up(ent * ell * ell * sizeof(double), 256) + align_up(ent * sizeof(double), 256);
+}
+
+template <int ELL>
+static void run_solve(const double* R, const int32_t* psi, Holders h, int N, int m, int delta,
+                      int npat, SolveOut out, Table tb, bool use_table, uint32_t* status,
+                      cudaStream_t s) {
+  if (use_table) {
+    const long long nent = (long long)N << tb.bits;
+    const int blocks = (int)((nent + 127) / 128);
+    k_table<ELL><<<blocks, 128, 0, s>>>(R, h, N, m, tb, status);
+    count_launches(1);
+  }
+  int ppb = N <= 256 ? 256 / N : 0;
+  const int grid = ppb > 0 ? (npat + ppb - 1) / ppb : npat;
+  count_launches(1);
+  if (use_table)
+    k_patterns<ELL, true><<<grid, 256, 0, s>>>(R, psi, h, N, m, delta, npat, ppb, tb, out, status);
+  else
+    k_patterns<ELL, false><<<grid, 256, 0, s>>>(R, psi, h, N, m, delta, npat, ppb, tb, out, status);
+}
+
+// The table region is carved by the caller right after the holders.
+int launch_solve_impl(const double* R, int ell, const int32_t* psi, Holders h, int N, int m,
+                      int delta, int npat, SolveOut out, void* table_mem, int bits,
+                      uint32_t* status, cudaStream_t s) {
+  Table tb{bits < 0 ? 0 : bits, nullptr, nullptr, nullptr};
+  const bool use_table = bits >= 0 && table_mem != nullptr;
+  if (use_table) {
+    const size_t ent = (size_t)N << bits;
+    char* p = static_cast<char*>(table_mem);
+    tb.xp = reinterpret_cast<double*>(p);
+    p += align_up(ent * bits * ell * sizeof(double), 256);
+    tb.pi = reinterpret_cast<double*>(p);
+    p += align_up(ent * ell * ell * sizeof(double), 256);
+    tb.err = reinterpret_cast<double*>(p);
+  }
+  if (out.E) {
+    cudaError_t e = cudaMemsetAsync(out.E, 0, (size_t)npat * m * delta * ell * sizeof(double), s);
+    if (e != cudaSuccess) return cuda_check(e, "cudaMemsetAsync(E)");
+  }
+  switch (ell) {
+    case 1: run_solve<1>(R, psi, h, N, m, delta, npat, out, tb, use_table, status, s); break;
+    case 2: run_solve<2>(R, psi, h, N, m, delta, npat, out, tb, use_table, status, s); break;
+    case 3: run_solve<3>(R, psi, h, N, m, delta, npat, out, tb, use_table, status, s); break;
+    case 4: run_solve<4>(R, psi, h, N, m, delta, npat, out, tb, use_table, status, s); break;
+    case 5: run_solve<5>(R, psi, h, N, m, delta, npat, out, tb, use_table, status, s); break;
+    case 6: run_solve<6>(R, psi, h, N, m, delta, npat, out, tb, use_table, status, s); break;
+    case 7: run_solve<7>(R, psi, h, N, m, delta, npat, out, tb, use_table, status, s); break;
+    case 8: run_solve<8>(R, psi, h, N, m, delta, npat, out, tb, use_table, status, s); break;
+    default: return fail(GC_ERR_UNSUPPORTED, "ell=%d exceeds GC_MAX_ELL", ell);
+  }
+  return cuda_check(cudaGetLastError(), "solve kernels");
+}
+
+}  // namespace gc

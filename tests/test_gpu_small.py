@@ -1,0 +1,272 @@
+"""GPU vs oracle parity on small inputs: the 6-worker workload brute-forced
+over every straggler pattern, ragged and degenerate shapes, explicit
+(non-uniform) orders, every cluster width of the chunk-gradient kernel, and
+device-detected bad data.  All calls go through the C-ABI (ctypes binding)."""
+import json
+import os
+
+import numpy as np
+import pytest
+import torch
+
+import oracle as O
+from _parity import (COEF_RTOL, assert_grad_close, assert_mse_close, dev_tensors, rel_inf, to_np)
+from workloads import all_patterns, get, make_data, make_patterns, make_R
+
+pytestmark = pytest.mark.gpu
+
+HERE = os.path.dirname(os.path.abspath(__file__))
+
+
+@pytest.fixture(scope="module")
+def gc():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    import paper_2405_19509_gb300 as m
+    return m
+
+
+def _tiny_patterns(cfg):
+    return np.concatenate([all_patterns(cfg.m, cfg.delta), make_patterns(cfg)])
+
+
+# ------------------------------------------------------------------ Algorithm 1
+@pytest.mark.parametrize("ell", [1, 2, 3])
+def test_tiny_coefficients_all_patterns(gc, ell):
+    """Every psi in {0..3}^6 plus the 256 seeded ones: Delta and the supports
+    bit-exact, E (Algorithm 1) to 1e-9, C = R B, coefficient error and
+    estimate, through both the memo-table path and the direct path."""
+    cfg = get("tiny")
+    N, m, delta = cfg.N, cfg.m, cfg.delta
+    order = O.cyclic_order(N, m, delta)
+    R = make_R(cfg, ell)
+    psi = _tiny_patterns(cfg)
+    Rd, od, pd = dev_tensors(R, order, psi)
+    big = gc.gc_find_encoding_coeff(Rd, ell, od, N, m, delta, pd, support=True)   # table path
+    ws = gc.Workspace()
+    small = gc.gc_find_encoding_coeff(Rd, ell, od, N, m, delta, pd[:3], support=True, ws=ws)  # direct
+    gc.gc_status(ws)
+    for k in ("E", "C", "coef_err", "delta"):
+        assert torch.equal(small[k], big[k][:3]), f"table and direct paths differ in {k}"
+    E, C, D, S = to_np(big["E"]), to_np(big["C"]), to_np(big["delta"]), to_np(big["support"])
+    ce, est = to_np(big["coef_err"]), to_np(big["est"])
+    for b in range(psi.shape[0]):
+        r = O.run_pattern(R, order, psi[b], N)
+        assert np.array_equal(D[b], r.Delta), b
+        assert np.array_equal(S[b], r.support), b
+        assert rel_inf(E[b], r.E) <= COEF_RTOL, b
+        assert np.max(np.abs(C[b] - r.C)) <= 2e-6, b
+        assert abs(ce[b] - r.coef_err) <= 1e-9, b
+        assert est[b] == r.est, b
+
+
+def test_worked_example_explicit_order(gc):
+    """Sec. II-B's five-worker example (non-uniform loads, a failed worker,
+    -1 slots): supports of eqs. (3) and (8) and the coefficients."""
+    with open(os.path.join(HERE, "golden", "worked_example.json")) as f:
+        g = json.load(f)
+    ex = np.array(g["order"], dtype=np.int32)
+    N, m, ell = g["N"], g["m"], g["ell"]
+    delta = ex.shape[1]
+    A, order, Om = gc.gc_make_assignment(N, m, delta, gc.GC_EXPLICIT, ex)
+    R = np.random.default_rng(31).standard_normal((ell, m))
+    psi = np.array([c["psi"] for c in g["cases"]], dtype=np.int32)
+    Rd, od, pd = dev_tensors(R, order, psi)
+    res = gc.gc_find_encoding_coeff(Rd, ell, od, N, m, delta, pd, support=True)
+    for b, case in enumerate(g["cases"]):
+        assert np.array_equal(to_np(res["support"][b]).T, np.array(case["B_support_worker_by_chunk"]))
+        assert list(to_np(res["delta"][b])) == case["Delta"]
+        assert res["est"][b].item() == case["estimate"]
+        r = O.run_pattern(R, order, psi[b], N)
+        assert rel_inf(to_np(res["E"][b]), r.E) <= COEF_RTOL
+        assert abs(res["coef_err"][b].item() - r.coef_err) <= 1e-9
+
+
+# ------------------------------------------------------------------ decode paths
+@pytest.mark.parametrize("ell", [1, 2, 3])
+def test_tiny_decode_batch_and_transmit_all_patterns(gc, ell):
+    """Batched decode-combine and the worker-encode / PS-decode path against
+    the oracle's transmit path, every pattern; l = 3 does not divide d = 64
+    (zero-padded last block)."""
+    cfg = get("tiny")
+    N, m, delta, d = cfg.N, cfg.m, cfg.delta, cfg.d
+    order = O.cyclic_order(N, m, delta)
+    R = make_R(cfg, ell)
+    psi = _tiny_patterns(cfg)
+    data = make_data(cfg)
+    G64 = O.chunk_gradients(data["X"].numpy(), data["y"].numpy(), data["w"].numpy(), N, cfg.n_c, O.LSQ)
+    G32 = G64.astype(np.float32)
+    Gref = G32.astype(np.float64)
+    Rd, od, pd = dev_tensors(R, order, psi)
+    Gd = torch.from_numpy(G32).cuda()
+    res = gc.gc_decode_batch(Rd, ell, od, N, m, delta, pd, Gd)
+    T = gc.gc_encode(Rd, ell, od, N, m, delta, pd, Gd)
+    gh = gc.gc_decode_tx(Rd, ell, m, T, d)
+    Gh, Tn, ghn = to_np(res["Ghat"]), to_np(T), to_np(gh)
+    mse = to_np(res["grad_mse"])
+    gsum = Gref.sum(axis=0)
+    floor = 1e-8 * float(gsum @ gsum) / d
+    for b in range(psi.shape[0]):
+        r = O.run_pattern(R, order, psi[b], N, Gref, want_transmit=True)
+        assert_grad_close(Gh[b], r.ghat, f"combine b={b}")
+        assert_grad_close(ghn[b], r.ghat, f"transmit b={b}")
+        if np.max(np.abs(r.T)) > 0:
+            assert rel_inf(Tn[b], r.T) <= 1e-4, b
+        else:
+            assert np.all(Tn[b] == 0)
+        assert_mse_close(mse[b], r.grad_mse, floor, f"mse b={b}")
+
+
+def test_degenerate_shapes(gc):
+    """d < ell (empty trailing blocks), psi all zero (nothing decoded), all
+    finished (baseline gradient), npat = 0 (no launch)."""
+    rng = np.random.default_rng(3)
+    N = m = 5
+    delta = 3
+    order = O.cyclic_order(N, m, delta)
+    for d, ell in [(2, 3), (5, 4), (1, 1), (7, 8)]:
+        if ell > 8:
+            continue
+        R = rng.standard_normal((ell, m))
+        G = rng.standard_normal((N, d)).astype(np.float32)
+        psi = np.array([[0] * m, [delta] * m, [1, 0, 3, 2, 1]], dtype=np.int32)
+        Rd, od, pd = dev_tensors(R, order, psi)
+        res = gc.gc_decode_batch(Rd, ell, od, N, m, delta, pd, torch.from_numpy(G).cuda())
+        Gh = to_np(res["Ghat"])
+        assert np.all(Gh[0] == 0.0)
+        for b in range(3):
+            r = O.run_pattern(R, order, psi[b], N, G.astype(np.float64))
+            assert_grad_close(Gh[b], r.ghat, f"d={d} ell={ell} b={b}")
+            assert res["est"][b].item() == r.est
+    # npat = 0: nothing to do, outputs untouched
+    R = rng.standard_normal((2, m))
+    Rd, od, pd = dev_tensors(R, order, np.zeros((0, m), dtype=np.int32))
+    res = gc.gc_decode_batch(Rd, 2, od, N, m, delta, pd, torch.zeros(N, 8, device="cuda"))
+    assert res["Ghat"].shape == (0, 8)
+
+
+def test_large_ell_and_explicit_uneven(gc):
+    """l = 8 (the build's maximum) with delta = 8, and an explicit order with
+    N != m and uneven replication."""
+    rng = np.random.default_rng(4)
+    N = m = 16
+    delta, ell, d = 8, 8, 40
+    order = O.cyclic_order(N, m, delta)
+    R = rng.standard_normal((ell, m))
+    G = rng.standard_normal((N, d)).astype(np.float32)
+    psi = rng.integers(0, delta + 1, size=(40, m)).astype(np.int32)
+    psi[0] = delta
+    Rd, od, pd = dev_tensors(R, order, psi)
+    res = gc.gc_decode_batch(Rd, ell, od, N, m, delta, pd, torch.from_numpy(G).cuda())
+    for b in range(psi.shape[0]):
+        r = O.run_pattern(R, order, psi[b], N, G.astype(np.float64), want_transmit=False)
+        assert_grad_close(to_np(res["Ghat"][b]), r.ghat, f"ell=8 b={b}")
+        assert abs(res["coef_err"][b].item() - r.coef_err) <= 1e-8
+    # explicit: 4 chunks, 6 workers, ragged loads
+    ex = np.array([[0, 1, 2], [1, 3, -1], [2, -1, -1], [3, 0, 1], [0, -1, -1], [2, 3, 0]],
+                  dtype=np.int32)
+    N2, m2, dl2 = 4, 6, 3
+    _, order2, _ = gc.gc_make_assignment(N2, m2, dl2, gc.GC_EXPLICIT, ex)
+    ell = 2
+    R2 = rng.standard_normal((ell, m2))
+    G2 = rng.standard_normal((N2, 10)).astype(np.float32)
+    psi2 = np.array([[3, 2, 1, 3, 1, 3], [1, 1, 0, 2, 0, 1], [0, 0, 0, 0, 0, 0], [2, 2, 1, 1, 1, 2]],
+                    dtype=np.int32)
+    Rd, od, pd = dev_tensors(R2, order2, psi2)
+    res = gc.gc_decode_batch(Rd, ell, od, N2, m2, dl2, pd, torch.from_numpy(G2).cuda())
+    for b in range(psi2.shape[0]):
+        r = O.run_pattern(R2, order2, psi2[b], N2, G2.astype(np.float64))
+        assert_grad_close(to_np(res["Ghat"][b]), r.ghat, f"explicit b={b}")
+        assert res["est"][b].item() == r.est
+
+
+# ------------------------------------------------------------------ chunk gradients
+@pytest.mark.parametrize("d,n_c,N,dtype,loss", [
+    (64, 32, 6, torch.float32, 0),       # tiny
+    (65, 7, 3, torch.float32, 1),        # ragged d (no TMA), odd n_c
+    (8, 1, 5, torch.float32, 0),         # one row per chunk
+    (4096, 16, 2, torch.float32, 1),     # one CTA per row
+    (16384, 8, 3, torch.float32, 0),     # cluster of 2
+    (32768, 4, 2, torch.float32, 1),     # cluster of 4
+    (65536, 4, 2, torch.float32, 0),     # cluster of 8
+    (65536, 8, 2, torch.bfloat16, 0),    # bf16, cluster of 4
+    (100, 6, 4, torch.bfloat16, 1),      # bf16 ragged (no TMA)
+    (1024, 2048, 1, torch.float32, 1),   # one chunk spanning many clusters
+])
+def test_chunk_grads_shapes(gc, d, n_c, N, dtype, loss):
+    g = torch.Generator().manual_seed(d * 7 + n_c)
+    X = torch.randn(N * n_c, d, generator=g)
+    if loss == 1:
+        X /= d ** 0.5
+        y = torch.where(torch.rand(N * n_c, generator=g) < 0.5, 1.0, -1.0)
+    else:
+        y = torch.randn(N * n_c, generator=g)
+    w = (torch.randn(d, generator=g) / d ** 0.5).float()
+    X = X.to(dtype)
+    Xd, yd, wd = X.cuda(), y.cuda(), w.cuda()
+    lo = torch.zeros(1, dtype=torch.float64, device="cuda")
+    ws = gc.Workspace()
+    G = gc.gc_chunk_grads(Xd, yd, wd, N, n_c, loss, loss_out=lo, ws=ws)
+    gc.gc_status(ws)
+    Go = O.chunk_gradients(X, y.numpy(), w.numpy(), N, n_c, loss)
+    for i in range(N):
+        assert_grad_close(to_np(G[i]), Go[i], f"chunk {i}")
+    Lo = O.full_loss(X, y.numpy(), w.numpy(), N * n_c, 4096, loss)
+    assert abs(lo.item() - Lo) <= 1e-5 * abs(Lo)
+
+
+def test_chunk_grads_unaligned_X(gc):
+    """An X view starting 4 bytes past a 16-byte boundary takes the plain-load path."""
+    N, n_c, d = 3, 8, 256
+    base = torch.randn(N * n_c * d + 1, generator=torch.Generator().manual_seed(9))
+    X = base[1:].view(N * n_c, d)
+    y = torch.randn(N * n_c, generator=torch.Generator().manual_seed(10))
+    w = torch.randn(d, generator=torch.Generator().manual_seed(11)) / 16
+    Xd = base.cuda()[1:].view(N * n_c, d)
+    assert Xd.data_ptr() % 16 != 0
+    G = gc.gc_chunk_grads(Xd, y.cuda(), w.cuda(), N, n_c, 0)
+    Go = O.chunk_gradients(X, y.numpy(), w.numpy(), N, n_c, 0)
+    assert_grad_close(to_np(G), Go, "unaligned")
+
+
+def test_sgd_step(gc):
+    d = 1000
+    w = torch.randn(d, generator=torch.Generator().manual_seed(1))
+    gh = torch.randn(d, generator=torch.Generator().manual_seed(2))
+    wd = w.cuda()
+    gc.gc_sgd_step(wd, gh.cuda(), 0.1, 4096)
+    ref = O.sgd_step(w.numpy(), gh.numpy(), 0.1, 4096)
+    assert np.max(np.abs(to_np(wd) - ref)) <= 1e-6 * (1 + np.max(np.abs(ref)))
+
+
+# ------------------------------------------------------------------ device-detected bad data
+def test_bad_psi_flagged(gc):
+    N = m = 6
+    delta, ell = 3, 2
+    order = O.cyclic_order(N, m, delta)
+    R = make_R(get("tiny"), ell)
+    psi = np.array([[0, 1, 2, 3, 4, 0], [-1, 0, 0, 0, 0, 0]], dtype=np.int32)   # 4 > delta, -1 < 0
+    Rd, od, pd = dev_tensors(R, order, psi)
+    ws = gc.Workspace()
+    gc.gc_find_encoding_coeff(Rd, ell, od, N, m, delta, pd, ws=ws)
+    with pytest.raises(gc.GCError) as ei:
+        gc.gc_status(ws)
+    assert ei.value.code == -7 and "psi" in str(ei.value)
+    gc.gc_status(ws)  # cleared
+
+
+def test_singular_R_flagged(gc):
+    """Two identical columns of R make X = R[:, S] rank deficient for a chunk
+    held by exactly those two workers."""
+    N = m = 6
+    delta, ell = 3, 2
+    order = O.cyclic_order(N, m, delta)
+    R = make_R(get("tiny"), ell)
+    R[:, 1] = R[:, 0]
+    psi = np.array([[2, 1, 0, 0, 0, 0]], dtype=np.int32)  # chunk 1 done by workers 0 and 1 only
+    Rd, od, pd = dev_tensors(R, order, psi)
+    ws = gc.Workspace()
+    gc.gc_find_encoding_coeff(Rd, ell, od, N, m, delta, pd, ws=ws)
+    with pytest.raises(gc.GCError) as ei:
+        gc.gc_status(ws)
+    assert ei.value.code == -7 and "rank" in str(ei.value)
