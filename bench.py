@@ -373,14 +373,14 @@ def gpu_arm(args, rank, world, local_rank):
     # ---- roofline of the dominant stage
     pk, pk_src = peaks()
     hbm = float(pk["hbm_gbs"])
-    names = ["k_chunkgrad", "k_patterns", "k_combine_simt", "encode+decode_tx+sgd"]
+    names = ["k_chunkgrad", "k_patterns", "k_combine_tc", "encode+decode_tx+sgd"]
     alg_bytes = [
         cfg.Ntil * d * 4 + cfg.Ntil * 4 + N * d * 4,                          # X, y read; G written
         npat * m * 4 + npat * ell * N * ell * 4 + 2 * npat * 8,               # psi read; C, errors written
         npat * d * 4 + npat * ell * N * ell * 4 + N * d * 4 + npat * 8,       # Ghat written; C, G read
         N * d * 4 + m * L * 4 * 2 + d * 4 * 3,                                # G read; T; ghat; w
     ]
-    srcs = [["k_chunkgrad.cu"], ["k_solve.cu"], ["k_combine.cu"], ["k_encode.cu"]]
+    srcs = [["k_chunkgrad.cu"], ["k_solve.cu"], ["k_combine_tc.cu"], ["k_encode.cu"]]
     dom = int(np.argmax(stage_ms))
     achieved = alg_bytes[dom] / (stage_ms[dom] / 1e3) / 1e9
     roofline = {"kernel": names[dom], "bound": "hbm", "achieved": achieved, "peak": hbm,

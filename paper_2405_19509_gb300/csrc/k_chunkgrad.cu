@@ -132,6 +132,7 @@ struct CGArgs {
   int S;          // stages
   int maxt;       // chunk slots per cluster in `parts`
   int loss;
+  int want_loss;
   int use_tma;
   float* parts;        // [clusters][maxt][d]
   double* loss_parts;  // [clusters]
@@ -304,29 +305,40 @@ __global__ void __launch_bounds__(NT, 1) k_chunkgrad(CGArgs a) {
         z[r] = t;
       }
     }
-    // ---- residuals (and the loss)
+    // ---- residuals
     float res[RBM];
 #pragma unroll
     for (int r = 0; r < RBM; ++r) {
       res[r] = 0.f;
       if (r < a.RB) {
-        const float yv = a.y[row0 + r];
+        const float yv = __ldg(a.y + row0 + r);
         if (a.loss == GC_LSQ) {
           res[r] = z[r] - yv;
         } else {
-          const float sg = 1.f / (1.f + expf(-z[r]));
+          const float sg = 1.f / (1.f + __expf(-z[r]));
           res[r] = sg - 0.5f * (yv + 1.f);
         }
-        if (tid == 0 && rank == 0) {
-          const double zd = z[r], yd = yv;
+      }
+    }
+    // ---- the loss: lane r of warp 0 takes row r (fp32), one fp64 add per batch
+    if (a.want_loss && rank == 0 && warp == 0) {
+      float lr = 0.f;
+#pragma unroll
+      for (int r = 0; r < RBM; ++r) {
+        if (r < a.RB && lane == r) {
+          const float yv = __ldg(a.y + row0 + r);
           if (a.loss == GC_LSQ) {
-            loss_acc += 0.5 * (zd - yd) * (zd - yd);
+            const float e = z[r] - yv;
+            lr = 0.5f * e * e;
           } else {
-            const double t = -yd * zd;  // log(1 + e^t), stable
-            loss_acc += (t > 0.0 ? t : 0.0) + log1p(exp(-fabs(t)));
+            const float t = -yv * z[r];  // log(1 + e^t), stable
+            lr = fmaxf(t, 0.f) + log1pf(expf(-fabsf(t)));
           }
         }
       }
+#pragma unroll
+      for (int o = 2; o > 0; o >>= 1) lr += __shfl_xor_sync(0xffffffffu, lr, o);
+      if (lane == 0) loss_acc += (double)lr;
     }
     // ---- pass 2: acc += r * x
 #pragma unroll
@@ -505,6 +517,7 @@ int launch_chunkgrad(const void* X, int x_dtype, const float* y, const float* w,
   a.S = p.S;
   a.maxt = p.maxt;
   a.loss = loss;
+  a.want_loss = loss_out != nullptr;
   a.use_tma = p.use_tma;
   a.parts = ws.take<float>((size_t)p.nclusters * p.maxt * d);
   a.loss_parts = ws.take<double>(p.nclusters);

@@ -1,0 +1,511 @@
+// Batched decode-combine on the 5th-generation tensor cores (tcgen05).
+//
+//   Ghat (M x L) = C (M x K) . Gv (K x L),  M = npat*ell, K = N*ell, L = ceil(d/ell),
+//
+// where row (b, k) of C is the decode matrix R B_b restricted to block k
+// (Algorithm 1) and row (i, k') of Gv is block k' of g_{D_i} (zero past d).
+// This is the PS decode of Sec. II-B applied to the eq. (2) transmissions of
+// every straggler pattern at once (R B = [Pi_1 ... Pi_N]).
+//
+// Precision: the operands are fp32 (C from fp64 projectors, chunk gradients
+// in fp32); each is split into bf16 hi + lo parts (x ~= hi + lo with relative
+// error 2^-17) and the product is accumulated in fp32 as
+//   C_hi G_hi + C_hi G_lo + C_lo G_hi       (the C_lo G_lo term, ~2^-16
+// relative, is dropped), i.e. three kind::f16 MMAs per K step.
+//
+// Kernel structure (persistent, one CTA per SM, 192 threads):
+//   warp 0      TMA producer: per k-block one 3-D tensor load for A (hi and
+//               lo planes, 128 x 64) and one for B (hi and lo, 256 x 64),
+//               128-byte swizzle, into a 2-stage shared-memory ring.
+//   warp 1      allocates 512 TMEM columns (two 128 x 256 fp32 accumulators)
+//               and one lane issues the MMAs; tcgen05.commit frees smem
+//               stages and signals a finished accumulator.
+//   warps 2..5  epilogue: tcgen05.ld (32 lanes x 32 columns per load), store
+//               to Ghat and/or reduce the squared error to sum_i g_{D_i}
+//               per row; the accumulator is handed back as soon as it is
+//               read, so the epilogue of tile t overlaps the MMAs of t + 1.
+// Tiles are visited n-tile-major so that concurrently running CTAs share the
+// same B tile through L2.  Every mbarrier wait is bounded; on expiry the
+// kernel flags GC_ERR_TIMEOUT in the status word, drains its own copies and
+// MMAs (with bounded waits) and frees TMEM.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+
+#include <algorithm>
+
+#include "gc_internal.cuh"
+
+namespace gc {
+namespace tc {
+
+constexpr int BM = 128, BN = 256, BK = 64, STAGES = 2;
+constexpr int A_PLANE = BM * BK * 2;                 // bytes of one bf16 plane (16 KB)
+constexpr int B_PLANE = BN * BK * 2;                 // 32 KB
+constexpr int STAGE_BYTES = 2 * A_PLANE + 2 * B_PLANE;  // 96 KB
+constexpr int THREADS = 192;
+constexpr uint32_t TMEM_COLS = 512;
+constexpr long long kSpin = 1LL << 32;  // clock cycles per wait (~2 s)
+constexpr size_t SMEM_BYTES = (size_t)STAGES * STAGE_BYTES + 1024 + 256;
+
+struct Params {
+  int M, Kp, L, ell, d;
+  int num_m_tiles, num_n_tiles, nkb;
+  long long num_tiles;
+  int vec_ok;           // d % 4 == 0 && L % 4 == 0: 16-byte row segments
+  float* Ghat;          // npat x d or null
+  const float* gsum;    // d, or null when no MSE is wanted
+  float* msep;          // M x num_n_tiles partial squared errors, or null
+  uint32_t* status;
+};
+
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count) : "memory");
+}
+__device__ __forceinline__ void mbar_expect_tx(uint64_t* bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)),
+               "r"(bytes)
+               : "memory");
+}
+__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(smem_u32(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+// Bounded wait; gives up when the limit passes or another role aborted.
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag,
+                                          uint32_t* status, long long limit = kSpin) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const long long t0 = clock64();
+  while (!mbar_try_wait(bar, parity)) {
+    if (*abort_flag) return false;
+    if (clock64() - t0 > limit) {
+      atomicOr(status, ST_TIMEOUT);
+      *abort_flag = 1;
+      return false;
+    }
+  }
+  return true;
+}
+__device__ __forceinline__ void tma_load_3d(void* dst, const CUtensorMap* map, int x, int y, int z,
+                                            uint64_t* bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.shared::cluster.global.mbarrier::complete_tx::bytes "
+      "[%0], [%1, {%2, %3, %4}], [%5];" ::"r"(smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(z), "r"(smem_u32(bar))
+      : "memory");
+}
+// Shared-memory matrix descriptor: K-major, 128-byte swizzle, 8-row groups
+// 1024 bytes apart (stride byte offset), descriptor version 1.
+__device__ __forceinline__ uint64_t sdesc(uint32_t saddr) {
+  uint64_t d = 0;
+  d |= (uint64_t)((saddr >> 4) & 0x3FFFu);
+  d |= (uint64_t)1u << 16;             // leading byte offset (unused for swizzled K-major)
+  d |= (uint64_t)(1024u >> 4) << 32;   // stride byte offset
+  d |= (uint64_t)1u << 46;             // version
+  d |= (uint64_t)2u << 61;             // SWIZZLE_128B
+  return d;
+}
+// Instruction descriptor, kind::f16: D fp32, A and B bf16, both K-major.
+constexpr uint32_t kIdesc = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(BN >> 3) << 17) |
+                            ((uint32_t)(BM >> 4) << 24);
+
+__device__ __forceinline__ void mma_bf16(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t accum) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "l"(a), "l"(b), "r"(kIdesc), "r"(accum)
+      : "memory");
+}
+__device__ __forceinline__ void mma_commit(uint64_t* bar) {
+  asm volatile(
+      "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
+          smem_u32(bar))
+      : "memory");
+}
+__device__ __forceinline__ void fence_before() {
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void fence_after() {
+  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
+  uint32_t r[32];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
+      "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, "
+      "%16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31}, [%32];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
+        "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]),
+        "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]),
+        "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+      : "r"(taddr));
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+  for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(r[j]);
+}
+
+__global__ void __launch_bounds__(THREADS, 1)
+    k_combine_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                 Params p) {
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~static_cast<uintptr_t>(1023));
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + STAGES * STAGE_BYTES);
+  uint64_t* empty = full + STAGES;
+  uint64_t* tfull = empty + STAGES;   // [2]
+  uint64_t* tempty = tfull + 2;       // [2]
+  uint64_t* done = tempty + 2;        // MMA drain
+  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(done + 1);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_holder + 1);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < STAGES; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    for (int a = 0; a < 2; ++a) {
+      mbar_init(&tfull[a], 1);
+      mbar_init(&tempty[a], 4);
+    }
+    mbar_init(done, 1);
+    *abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == 1) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                     smem_u32(tmem_holder)),
+                 "r"(TMEM_COLS)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+  fence_before();
+  __syncthreads();
+  fence_after();
+  const uint32_t tmem_base = *tmem_holder;
+
+  if (warp == 0) {
+    // ------------------------------------------------------------- producer
+    if (lane == 0) {
+      uint32_t it = 0;
+      bool ok = true;
+      for (long long t = blockIdx.x; t < p.num_tiles && ok; t += gridDim.x) {
+        const int nt = (int)(t / p.num_m_tiles), mt = (int)(t % p.num_m_tiles);
+        for (int kb = 0; kb < p.nkb; ++kb, ++it) {
+          const int s = it % STAGES;
+          const uint32_t ph = (it / STAGES) & 1;
+          if (!mbar_wait(&empty[s], ph ^ 1, abort_flag, p.status)) {
+            ok = false;
+            break;
+          }
+          uint8_t* st = smem + s * STAGE_BYTES;
+          mbar_expect_tx(&full[s], STAGE_BYTES);
+          tma_load_3d(st, &tmA, kb * BK, mt * BM, 0, &full[s]);
+          tma_load_3d(st + 2 * A_PLANE, &tmB, kb * BK, nt * BN, 0, &full[s]);
+        }
+      }
+      // drain: every issued stage has landed before the CTA may exit
+      const uint32_t issued = it;
+      for (uint32_t k = (issued > (uint32_t)STAGES ? issued - STAGES : 0); k < issued; ++k) {
+        volatile int no_abort = 0;
+        mbar_wait(&full[k % STAGES], (k / STAGES) & 1, &no_abort, p.status, 1LL << 28);
+      }
+    }
+  } else if (warp == 1) {
+    // ------------------------------------------------------------- MMA issuer
+    if (lane == 0) {
+      uint32_t it = 0, tile_it = 0;
+      bool ok = true;
+      for (long long t = blockIdx.x; t < p.num_tiles && ok; t += gridDim.x, ++tile_it) {
+        const int ab = tile_it & 1;
+        if (!mbar_wait(&tempty[ab], ((tile_it >> 1) & 1) ^ 1, abort_flag, p.status)) break;
+        fence_after();
+        const uint32_t d_tmem = tmem_base + (uint32_t)(ab * BN);
+        for (int kb = 0; kb < p.nkb; ++kb, ++it) {
+          const int s = it % STAGES;
+          const uint32_t ph = (it / STAGES) & 1;
+          if (!mbar_wait(&full[s], ph, abort_flag, p.status)) {
+            ok = false;
+            break;
+          }
+          fence_after();
+          const uint32_t a_hi = smem_u32(smem + s * STAGE_BYTES);
+          const uint32_t a_lo = a_hi + A_PLANE;
+          const uint32_t b_hi = a_hi + 2 * A_PLANE;
+          const uint32_t b_lo = b_hi + B_PLANE;
+          const int rem = p.Kp - kb * BK;
+          const int nks = rem >= BK ? BK / 16 : (rem + 15) / 16;
+          for (int ks = 0; ks < nks; ++ks) {
+            const uint32_t off = ks * 32;  // 16 bf16 along K inside the swizzle atom
+            const uint32_t acc = (kb > 0 || ks > 0) ? 1u : 0u;
+            mma_bf16(d_tmem, sdesc(a_hi + off), sdesc(b_hi + off), acc);
+            mma_bf16(d_tmem, sdesc(a_hi + off), sdesc(b_lo + off), 1u);
+            mma_bf16(d_tmem, sdesc(a_lo + off), sdesc(b_hi + off), 1u);
+          }
+          mma_commit(&empty[s]);
+        }
+        if (!ok) break;
+        mma_commit(&tfull[ab]);
+      }
+      // drain: all issued MMAs have completed
+      mma_commit(done);
+      volatile int no_abort = 0;
+      mbar_wait(done, 0, &no_abort, p.status, 1LL << 28);
+    }
+  } else {
+    // ------------------------------------------------------------- epilogue
+    const int quarter = warp & 3;  // TMEM lanes 32*quarter .. +31
+    uint32_t tile_it = 0;
+    for (long long t = blockIdx.x; t < p.num_tiles; t += gridDim.x, ++tile_it) {
+      const int ab = tile_it & 1;
+      const int nt = (int)(t / p.num_m_tiles), mt = (int)(t % p.num_m_tiles);
+      if (!mbar_wait(&tfull[ab], (tile_it >> 1) & 1, abort_flag, p.status)) break;
+      fence_after();
+      const int row = mt * BM + quarter * 32 + lane;
+      const bool rv = row < p.M;
+      const int b = rv ? row / p.ell : 0;
+      const int k = rv ? row - b * p.ell : 0;
+      const int n0 = nt * BN;
+      float* out = p.Ghat ? p.Ghat + (size_t)b * p.d + (size_t)k * p.L : nullptr;
+      const float* gs = p.gsum ? p.gsum + (size_t)k * p.L : nullptr;
+      float sq = 0.f;
+      const uint32_t taddr = tmem_base + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(ab * BN);
+#pragma unroll 1
+      for (int cc = 0; cc < BN; cc += 32) {
+        float v[32];
+        __syncwarp();
+        tmem_ld32(taddr + cc, v);  // warp-collective: every lane, every chunk
+        const int c0 = n0 + cc;
+        const int lim = (rv && c0 < p.L) ? min(32, min(p.L - c0, p.d - k * p.L - c0)) : 0;
+        if (lim <= 0) {
+        } else if (lim == 32 && p.vec_ok) {
+          if (out) {
+            float4* o4 = reinterpret_cast<float4*>(out + c0);
+#pragma unroll
+            for (int j = 0; j < 8; ++j)
+              o4[j] = make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
+          }
+          if (gs) {
+            const float4* g4 = reinterpret_cast<const float4*>(gs + c0);
+#pragma unroll
+            for (int j = 0; j < 8; ++j) {
+              const float4 g = __ldg(g4 + j);
+              float df = v[4 * j] - g.x;
+              sq = fmaf(df, df, sq);
+              df = v[4 * j + 1] - g.y;
+              sq = fmaf(df, df, sq);
+              df = v[4 * j + 2] - g.z;
+              sq = fmaf(df, df, sq);
+              df = v[4 * j + 3] - g.w;
+              sq = fmaf(df, df, sq);
+            }
+          }
+        } else {
+#pragma unroll
+          for (int j = 0; j < 32; ++j) {
+            if (j < lim) {
+              if (out) out[c0 + j] = v[j];
+              if (gs) {
+                const float df = v[j] - __ldg(gs + c0 + j);
+                sq = fmaf(df, df, sq);
+              }
+            }
+          }
+        }
+      }
+      fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&tempty[ab]);
+      if (p.msep && rv) p.msep[(size_t)row * p.num_n_tiles + nt] = sq;
+    }
+  }
+  fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    fence_after();
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem_base),
+                 "r"(TMEM_COLS)
+                 : "memory");
+  }
+}
+
+// C (M x K fp32) -> planes [2][M][Kp] bf16: hi = bf16(c), lo = bf16(c - hi); zero pad.
+__global__ void k_split_c(const float* __restrict__ C, int M, int K, int Kp,
+                          __nv_bfloat16* __restrict__ out) {
+  const long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+  const long long tot = (long long)M * Kp;
+  if (idx >= tot) return;
+  const int row = (int)(idx / Kp), kk = (int)(idx - (long long)row * Kp);
+  const float v = kk < K ? __ldg(C + (size_t)row * K + kk) : 0.f;
+  const __nv_bfloat16 hi = __float2bfloat16_rn(v);
+  const __nv_bfloat16 lo = __float2bfloat16_rn(v - __bfloat162float(hi));
+  out[idx] = hi;
+  out[tot + idx] = lo;
+}
+
+// G (N x d fp32) -> planes [2][L][Kp] bf16 of Gv^T: element (c, i*ell + k') =
+// g_{D_i}[k'*L + c] (zero past d and for padding columns).  32 x 32 tiles
+// transposed through shared memory.
+__global__ void k_split_gt(const float* __restrict__ G, int N, int d, int ell, int L, int Kp,
+                           __nv_bfloat16* __restrict__ out) {
+  __shared__ float tile[32][33];
+  const int c0 = blockIdx.x * 32, k0 = blockIdx.y * 32;
+  const int tx = threadIdx.x, ty = threadIdx.y;  // 32 x 8
+  const int K = N * ell;
+  for (int r = ty; r < 32; r += 8) {
+    const int kk = k0 + r, c = c0 + tx;
+    float v = 0.f;
+    if (kk < K && c < L) {
+      const int i = kk / ell, kp = kk - i * ell;
+      const int col = kp * L + c;
+      if (col < d) v = __ldg(G + (size_t)i * d + col);
+    }
+    tile[r][tx] = v;
+  }
+  __syncthreads();
+  const size_t plane = (size_t)L * Kp;
+  for (int r = ty; r < 32; r += 8) {
+    const int c = c0 + r, kk = k0 + tx;
+    if (c < L && kk < Kp) {
+      const float v = tile[tx][r];
+      const __nv_bfloat16 hi = __float2bfloat16_rn(v);
+      const __nv_bfloat16 lo = __float2bfloat16_rn(v - __bfloat162float(hi));
+      out[(size_t)c * Kp + kk] = hi;
+      out[plane + (size_t)c * Kp + kk] = lo;
+    }
+  }
+}
+
+__global__ void k_mse_reduce_tiles(const float* __restrict__ msep, int npat, int ell,
+                                   int num_n_tiles, int d, double* __restrict__ grad_mse) {
+  const int b = blockIdx.x * blockDim.x + threadIdx.x;
+  if (b >= npat) return;
+  double s = 0.0;
+  for (int k = 0; k < ell; ++k) {
+    const float* r = msep + ((size_t)b * ell + k) * num_n_tiles;
+    for (int t = 0; t < num_n_tiles; ++t) s += (double)r[t];
+  }
+  grad_mse[b] = s / (double)d;
+}
+
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  if (!fn) {
+    void* ptr = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(ptr);
+  }
+  return fn;
+}
+
+// 3-D map over [2][rows][Kp] bf16 planes, box {64, box_rows, 2}, 128-byte swizzle.
+int make_map(CUtensorMap* map, const void* base, int rows, int Kp, int box_rows) {
+  auto fn = encode_fn();
+  if (!fn) return fail(GC_ERR_CUDA, "cuTensorMapEncodeTiled entry point unavailable");
+  cuuint64_t dims[3] = {(cuuint64_t)Kp, (cuuint64_t)rows, 2};
+  cuuint64_t strides[2] = {(cuuint64_t)Kp * 2, (cuuint64_t)rows * Kp * 2};
+  cuuint32_t box[3] = {(cuuint32_t)BK, (cuuint32_t)box_rows, 2};
+  cuuint32_t estr[3] = {1, 1, 1};
+  CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides,
+                  box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                  CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) return fail(GC_ERR_CUDA, "cuTensorMapEncodeTiled failed (%d)", (int)r);
+  return GC_OK;
+}
+
+}  // namespace tc
+
+size_t combine_tc_ws_bytes(int N, int ell, int npat, int d) {
+  const int L = (d + ell - 1) / ell;
+  const long long M = (long long)npat * ell;
+  const int K = N * ell;
+  const int Kp = (K + 7) / 8 * 8;
+  const int nnt = (L + tc::BN - 1) / tc::BN;
+  return align_up((size_t)2 * M * Kp * 2, 256) + align_up((size_t)2 * L * Kp * 2, 256) +
+         align_up((size_t)M * nnt * sizeof(float), 256);
+}
+
+int launch_combine_tc(const float* C, const float* G, const float* gsum, int N, int ell, int npat,
+                      int d, float* Ghat, double* grad_mse, Carve& ws, uint32_t* status,
+                      cudaStream_t s) {
+  using namespace tc;
+  const int L = (d + ell - 1) / ell;
+  const long long M = (long long)npat * ell;
+  const int K = N * ell;
+  const int Kp = (K + 7) / 8 * 8;
+  if (M > (1LL << 31) - 1) return fail(GC_ERR_UNSUPPORTED, "npat*ell too large");
+  const int nmt = (int)((M + BM - 1) / BM), nnt = (L + BN - 1) / BN;
+  __nv_bfloat16* Cs = ws.take<__nv_bfloat16>((size_t)2 * M * Kp);
+  __nv_bfloat16* Gs = ws.take<__nv_bfloat16>((size_t)2 * L * Kp);
+  float* msep = grad_mse ? ws.take<float>((size_t)M * nnt) : nullptr;
+
+  {
+    const long long tot = M * Kp;
+    k_split_c<<<(unsigned)((tot + 255) / 256), 256, 0, s>>>(C, (int)M, K, Kp, Cs);
+    count_launches(1);
+    dim3 grid((L + 31) / 32, (Kp + 31) / 32);
+    k_split_gt<<<grid, dim3(32, 8), 0, s>>>(G, N, d, ell, L, Kp, Gs);
+    count_launches(1);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return cuda_check(e, "split kernels");
+  }
+  CUtensorMap mA, mB;
+  int rc = make_map(&mA, Cs, (int)M, Kp, BM);
+  if (rc) return rc;
+  rc = make_map(&mB, Gs, L, Kp, BN);
+  if (rc) return rc;
+  Params p{};
+  p.M = (int)M;
+  p.Kp = Kp;
+  p.L = L;
+  p.ell = ell;
+  p.d = d;
+  p.num_m_tiles = nmt;
+  p.num_n_tiles = nnt;
+  p.nkb = (Kp + BK - 1) / BK;
+  p.num_tiles = (long long)nmt * nnt;
+  p.vec_ok = (d % 4 == 0) && (L % 4 == 0);
+  p.Ghat = Ghat;
+  p.gsum = grad_mse ? gsum : nullptr;
+  p.msep = msep;
+  p.status = status;
+  static bool attr_set = false;
+  if (!attr_set) {
+    cudaError_t e = cudaFuncSetAttribute(k_combine_tc, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)SMEM_BYTES);
+    if (e != cudaSuccess) return cuda_check(e, "cudaFuncSetAttribute(k_combine_tc)");
+    attr_set = true;
+  }
+  const int sms = device_sm_count();
+  const int grid = (int)std::min<long long>(p.num_tiles, sms);
+  k_combine_tc<<<grid, THREADS, SMEM_BYTES, s>>>(mA, mB, p);
+  count_launches(1);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return cuda_check(e, "k_combine_tc");
+  if (grad_mse) {
+    k_mse_reduce_tiles<<<(npat + 255) / 256, 256, 0, s>>>(msep, npat, ell, nnt, d, grad_mse);
+    count_launches(1);
+    e = cudaGetLastError();
+    if (e != cudaSuccess) return cuda_check(e, "k_mse_reduce_tiles");
+  }
+  return GC_OK;
+}
+
+}  // namespace gc
