@@ -161,6 +161,16 @@ int gc_encode(const double* R, int ell, const int32_t* order, int N, int m, int 
               const int32_t* psi, int npat, const float* G, int d, float* T, void* ws,
               size_t ws_bytes, void* stream);
 
+/* ---- worker encoding from given coefficients (eq. 2 alone) -----------
+ * T[b][j] = sum_{p < psi[b][j]} sum_k E[b][j][p][k] g_{D_order[j][p]}[k], with
+ * E the npat x m x delta x ell coefficients gc_find_encoding_coeff returns
+ * (Algorithm 1).  Lets a caller run Algorithm 1 while the chunk gradients
+ * are still being computed.  No workspace.
+ */
+int gc_encode_with_coeffs(const double* E, int ell, const int32_t* order, int N, int m, int delta,
+                          const int32_t* psi, int npat, const float* G, int d, float* T,
+                          void* stream);
+
 /* ---- PS decoding of received transmissions (Sec. II-B) ----------------
  * ghat[b][k*L + c] = sum_j R[k][j] T[b][j][c] for k*L + c < d.
  * T npat x m x L float32; ghat npat x d float32.  No workspace.

@@ -26,6 +26,7 @@ from .binding import (  # noqa: F401
     gc_kernel_launches,
     gc_decode_tx,
     gc_encode,
+    gc_encode_with_coeffs,
     gc_encode_workspace,
     gc_find_encoding_coeff,
     gc_last_error,

@@ -49,6 +49,7 @@ _sig("gc_find_encoding_coeff", _i, _p, _i, _p, _i, _i, _i, _p, _i, _p, _p, _p, _
      _sz, _p)
 _sig("gc_encode_workspace", _sz, _i, _i, _i, _i, _i, _i)
 _sig("gc_encode", _i, _p, _i, _p, _i, _i, _i, _p, _i, _p, _i, _p, _p, _sz, _p)
+_sig("gc_encode_with_coeffs", _i, _p, _i, _p, _i, _i, _i, _p, _i, _p, _i, _p, _p)
 _sig("gc_decode_tx", _i, _p, _i, _i, _p, _i, _i, _p, _p)
 _sig("gc_decode_batch_workspace", _sz, _i, _i, _i, _i, _i, _i)
 _sig("gc_decode_batch", _i, _p, _i, _p, _i, _i, _i, _p, _i, _p, _i, _p, _p, _p, _p, _p, _sz, _p)
@@ -227,6 +228,22 @@ def gc_encode(R, ell, order, N, m, delta, psi, G, T=None, ws: Workspace | None =
                          _dev(psi, torch.int32, "psi", (npat, m)), npat,
                          _dev(G, torch.float32, "G", (N, d)), d,
                          _dev(T, torch.float32, "T", (npat, m, L)), wp, wn, _stream()))
+    return T
+
+
+def gc_encode_with_coeffs(E, ell, order, N, m, delta, psi, G, T=None):
+    """Eq. (2) alone: transmissions from Algorithm 1's coefficients E
+    (npat x m x delta x ell float64, as gc_find_encoding_coeff returns)."""
+    npat = psi.shape[0]
+    d = G.shape[1]
+    L = block_length(d, ell)
+    if T is None:
+        T = torch.empty(npat, m, L, dtype=torch.float32, device=G.device)
+    _check(lib.gc_encode_with_coeffs(_dev(E, torch.float64, "E", (npat, m, delta, ell)), ell,
+                                     _dev(order, torch.int32, "order", (m, delta)), N, m, delta,
+                                     _dev(psi, torch.int32, "psi", (npat, m)), npat,
+                                     _dev(G, torch.float32, "G", (N, d)), d,
+                                     _dev(T, torch.float32, "T", (npat, m, L)), _stream()))
     return T
 
 

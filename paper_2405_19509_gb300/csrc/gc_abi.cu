@@ -258,6 +258,18 @@ int gc_encode(const double* R, int ell, const int32_t* order, int N, int m, int 
   return launch_encode(E, order, psi, N, m, delta, ell, npat, G, d, T, s);
 }
 
+int gc_encode_with_coeffs(const double* E, int ell, const int32_t* order, int N, int m, int delta,
+                          const int32_t* psi, int npat, const float* G, int d, float* T,
+                          void* stream) {
+  int rc = check_dims(N, m, delta, ell, npat);
+  if (rc) return rc;
+  if (d < 1) return fail(GC_ERR_SHAPE, "d=%d must be >= 1", d);
+  if (!E || !order || !G || !T || (!psi && npat > 0))
+    return fail(GC_ERR_ARG, "E, order, psi, G and T must be non-NULL");
+  if (npat == 0) return GC_OK;
+  return launch_encode(E, order, psi, N, m, delta, ell, npat, G, d, T, as_stream(stream));
+}
+
 int gc_decode_tx(const double* R, int ell, int m, const float* T, int npat, int d, float* ghat,
                  void* stream) {
   if (!R || !T || !ghat) return fail(GC_ERR_ARG, "R, T and ghat must be non-NULL");

@@ -24,6 +24,7 @@
 // Rows that are not 16-byte multiples, or unaligned X, take the same kernel
 // with plain cooperative loads instead of TMA (use_tma = 0).
 #include <math.h>
+#include <stdlib.h>
 
 #include <algorithm>
 #include <mutex>
@@ -116,6 +117,10 @@ struct Vec<__nv_bfloat16> {
 };
 
 constexpr int kMaxStages = 4;
+// DSMEM exchange slots: a peer can run at most ~1.5 batches ahead of this CTA
+// (it needs this CTA's sums of batch n + 1 before writing batch n + 4), so
+// four slots keep a slot from being rewritten before it is read.
+constexpr int kZSlots = 4;
 constexpr long long kSpinLimit = 1LL << 31;  // clock cycles (~1 s) per wait
 
 struct CGArgs {
@@ -139,17 +144,62 @@ struct CGArgs {
   uint32_t* status;
 };
 
+__device__ __forceinline__ void mbar_arrive_local(uint64_t* bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
+// Arrive on the mbarrier at the same offset in cluster peer `rank`, releasing
+// this thread's prior shared::cluster stores to it.
+__device__ __forceinline__ void mbar_arrive_remote(uint64_t* bar, uint32_t rank) {
+  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(
+                   mapa(smem_u32(bar), rank))
+               : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait_cluster(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(smem_u32(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+// Bounded wait; `cl` selects cluster-scope acquire (remote arrivals).
+__device__ __forceinline__ bool bounded_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag,
+                                             uint32_t* status, bool cl = false) {
+  auto tw = [&]() { return cl ? mbar_try_wait_cluster(bar, parity) : mbar_try_wait(bar, parity); };
+  if (tw()) return true;
+  const long long t0 = clock64();
+  while (!tw()) {
+    if (*abort_flag) return false;
+    if (clock64() - t0 > kSpinLimit) {
+      atomicOr(status, ST_TIMEOUT);
+      *abort_flag = 1;
+      return false;
+    }
+  }
+  return true;
+}
+__device__ __forceinline__ void consumer_sync(int nthreads) {
+  asm volatile("bar.sync 1, %0;" ::"r"(nthreads) : "memory");
+}
+
+// NT consumer threads (warps 0 .. NW-1) plus one producer warp (warp NW).
 template <typename T, int CL, int NT, int NVT, int RBM>
-__global__ void __launch_bounds__(NT, 1) k_chunkgrad(CGArgs a) {
+__global__ void __launch_bounds__(NT + 32, 1) k_chunkgrad(CGArgs a) {
   constexpr int V = Vec<T>::V;
   constexpr int NW = NT / 32;
   extern __shared__ __align__(128) unsigned char smem[];
   T* stages = reinterpret_cast<T*>(smem);
   const size_t stage_elems = (size_t)RBM * a.ld_s;
   float* red = reinterpret_cast<float*>(smem + a.S * stage_elems * sizeof(T));  // [2][NW][RBM]
-  float* zcl = red + 2 * NW * RBM;                                               // [2][CL][RBM]
-  uint64_t* full = reinterpret_cast<uint64_t*>(zcl + 2 * CL * RBM + 2);          // [S] (8B aligned)
-  volatile int& s_abort = *reinterpret_cast<int*>(full + kMaxStages);
+  float* zcl = red + 2 * NW * RBM;                                               // [kZSlots][CL][RBM]
+  uint64_t* bars = reinterpret_cast<uint64_t*>(zcl + kZSlots * CL * RBM + 2);    // 8-byte aligned
+  uint64_t* full = bars;                    // [kMaxStages] data landed
+  uint64_t* empty = bars + kMaxStages;      // [kMaxStages] consumers done with the stage
+  uint64_t* zfull = bars + 2 * kMaxStages;  // [kZSlots] every peer's partial dots arrived
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(bars + 2 * kMaxStages + kZSlots);
 
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int rank = CL > 1 ? (int)cluster_rank() : 0;
@@ -161,206 +211,232 @@ __global__ void __launch_bounds__(NT, 1) k_chunkgrad(CGArgs a) {
   const int nvs = a.Wc / V;  // vectors in this CTA's slice
   const T* X = static_cast<const T*>(a.X);
 
-  // w slice in registers (zeros past d)
-  float wv[NVT][V];
-#pragma unroll
-  for (int u = 0; u < NVT; ++u) {
-    const int v = tid + u * NT;
-#pragma unroll
-    for (int e = 0; e < V; ++e) {
-      const int col = c0 + v * V + e;
-      wv[u][e] = (v < nvs && col < a.d) ? a.w[col] : 0.f;
-    }
-  }
-  float acc[NVT][V];
-#pragma unroll
-  for (int u = 0; u < NVT; ++u)
-#pragma unroll
-    for (int e = 0; e < V; ++e) acc[u][e] = 0.f;
-
   if (tid == 0) {
-    s_abort = 0;
-    for (int s = 0; s < a.S; ++s) mbar_init(&full[s], 1);
+    *abort_flag = 0;
+    for (int s = 0; s < a.S; ++s) {
+      mbar_init(&full[s], a.use_tma ? 1 : 32);
+      mbar_init(&empty[s], NW);
+    }
+    for (int z = 0; z < kZSlots; ++z) mbar_init(&zfull[z], CL);
     fence_mbar_init();
   }
   __syncthreads();
-  if (CL > 1) cluster_sync_all();  // every peer has started before any DSMEM store
+  if (CL > 1) cluster_sync_all();  // every peer has started and initialised its barriers
 
-  const uint32_t row_bytes = (uint32_t)(a.Wc * sizeof(T));
-  auto issue = [&](int n) {  // TMA loads of batch n into stage n % S (thread 0 only)
-    const int s = n % a.S;
-    mbar_expect_tx(&full[s], row_bytes * a.RB);
-    const long long row = r0 + (long long)n * a.RB;
-    for (int r = 0; r < a.RB; ++r)
-      bulk_g2s(stages + s * stage_elems + (size_t)r * a.ld_s, X + (row + r) * a.d + c0, row_bytes,
-               &full[s]);
-  };
-  if (a.use_tma && tid == 0)
-    for (int n = 0; n < min(a.S, nb); ++n) issue(n);
-
-  const long long first_chunk = r0 / a.n_c;
-  long long cur = -1;
-  double loss_acc = 0.0;
-
-  auto flush = [&](long long chunk) {
-    float* dst = a.parts + ((size_t)q * a.maxt + (size_t)(chunk - first_chunk)) * a.d;
+  if (warp == NW) {
+    // ------------------------------------------------------------ producer warp
+    const uint32_t row_bytes = (uint32_t)(a.Wc * sizeof(T));
+    for (int n = 0; n < nb; ++n) {
+      const int s = n % a.S;
+      const uint32_t ph = (uint32_t)((n / a.S) & 1);
+      if (!bounded_wait(&empty[s], ph ^ 1, abort_flag, a.status)) break;
+      T* st = stages + s * stage_elems;
+      const long long row = r0 + (long long)n * a.RB;
+      if (a.use_tma) {
+        if (lane == 0) {
+          mbar_expect_tx(&full[s], row_bytes * a.RB);
+          for (int r = 0; r < a.RB; ++r)
+            bulk_g2s(st + (size_t)r * a.ld_s, X + (row + r) * a.d + c0, row_bytes, &full[s]);
+        }
+      } else {
+        // plain loads with bounds (zero fill past d), then every lane arrives
+        for (int r = 0; r < a.RB; ++r) {
+          const T* src = X + (row + r) * a.d;
+          for (int c = lane; c < a.ld_s; c += 32) {
+            const int col = c0 + c;
+            st[(size_t)r * a.ld_s + c] = (c < a.Wc && col < a.d) ? src[col] : T(0.f);
+          }
+        }
+        mbar_arrive_local(&full[s]);
+      }
+    }
+    // drain: the CTA must not exit with copies in flight
+    if (a.use_tma && lane == 0) {
+      volatile int no_abort = 0;
+      for (int n = max(0, nb - a.S); n < nb; ++n)
+        bounded_wait(&full[n % a.S], (uint32_t)((n / a.S) & 1), &no_abort, a.status);
+    }
+  } else {
+    // ------------------------------------------------------------ consumer warps
+    float wv[NVT][V];
 #pragma unroll
     for (int u = 0; u < NVT; ++u) {
       const int v = tid + u * NT;
-      if (v < nvs) {
 #pragma unroll
-        for (int e = 0; e < V; ++e) {
-          const int col = c0 + v * V + e;
-          if (col < a.d) dst[col] = acc[u][e];
-        }
+      for (int e = 0; e < V; ++e) {
+        const int col = c0 + v * V + e;
+        wv[u][e] = (v < nvs && col < a.d) ? a.w[col] : 0.f;
       }
     }
-  };
+    float acc[NVT][V];
+#pragma unroll
+    for (int u = 0; u < NVT; ++u)
+#pragma unroll
+      for (int e = 0; e < V; ++e) acc[u][e] = 0.f;
+    const long long first_chunk = r0 / a.n_c;
+    long long cur = -1;
+    double loss_acc = 0.0;
+    auto flush = [&](long long chunk) {
+      float* dst = a.parts + ((size_t)q * a.maxt + (size_t)(chunk - first_chunk)) * a.d;
+#pragma unroll
+      for (int u = 0; u < NVT; ++u) {
+        const int v = tid + u * NT;
+        if (v < nvs) {
+#pragma unroll
+          for (int e = 0; e < V; ++e) {
+            const int col = c0 + v * V + e;
+            if (col < a.d) dst[col] = acc[u][e];
+          }
+        }
+      }
+    };
 
-  for (int n = 0; n < nb; ++n) {
-    const int s = n % a.S;
-    const long long row0 = r0 + (long long)n * a.RB;
-    const long long chunk = row0 / a.n_c;
-    if (chunk != cur) {
-      if (cur >= 0) flush(cur);
+    // Pass 1 of batch n: partial dot products, CTA reduction and (clusters)
+    // the send to every peer.  Returns the CTA sums in every lane.
+    auto pass1 = [&](int n, float (&z)[RBM]) {
+      const int s = n % a.S;
+      bounded_wait(&full[s], (uint32_t)((n / a.S) & 1), abort_flag, a.status);
+      const T* st = stages + s * stage_elems;
+      float pd[RBM];
 #pragma unroll
-      for (int u = 0; u < NVT; ++u)
+      for (int r = 0; r < RBM; ++r) {
+        pd[r] = 0.f;
+        if (r < a.RB) {
 #pragma unroll
-        for (int e = 0; e < V; ++e) acc[u][e] = 0.f;
-      cur = chunk;
-    }
-    T* st = stages + s * stage_elems;
-    if (a.use_tma) {
-      if (!s_abort) {
-        const uint32_t parity = (uint32_t)((n / a.S) & 1);
-        if (!mbar_try_wait(&full[s], parity)) {
-          const long long t0 = clock64();
-          while (!mbar_try_wait(&full[s], parity)) {
-            if (clock64() - t0 > kSpinLimit) {
-              atomicOr(a.status, ST_TIMEOUT);
-              s_abort = 1;
-              break;
+          for (int u = 0; u < NVT; ++u) {
+            const int v = tid + u * NT;
+            if (v < nvs) {
+              float x[V];
+              Vec<T>::load(st + (size_t)r * a.ld_s + v * V, x);
+#pragma unroll
+              for (int e = 0; e < V; ++e) pd[r] = fmaf(x[e], wv[u][e], pd[r]);
             }
           }
         }
       }
-    } else {
-      // cooperative load with bounds (zero fill past d)
-      for (int r = 0; r < a.RB; ++r) {
-        const T* src = X + (row0 + r) * a.d;
-        for (int c = tid; c < a.ld_s; c += NT) {
-          const int col = c0 + c;
-          st[(size_t)r * a.ld_s + c] = (c < a.Wc && col < a.d) ? src[col] : T(0.f);
-        }
-      }
-      __syncthreads();
-    }
-    // ---- pass 1: partial dot products
-    float pd[RBM];
 #pragma unroll
-    for (int r = 0; r < RBM; ++r) {
-      pd[r] = 0.f;
-      if (r < a.RB) {
+      for (int r = 0; r < RBM; ++r)
 #pragma unroll
-        for (int u = 0; u < NVT; ++u) {
-          const int v = tid + u * NT;
-          if (v < nvs) {
-            float x[V];
-            Vec<T>::load(st + (size_t)r * a.ld_s + v * V, x);
+        for (int o = 16; o > 0; o >>= 1) pd[r] += __shfl_xor_sync(0xffffffffu, pd[r], o);
+      float* redn = red + (n & 1) * NW * RBM;
+      if (lane == 0)
 #pragma unroll
-            for (int e = 0; e < V; ++e) pd[r] = fmaf(x[e], wv[u][e], pd[r]);
-          }
-        }
-      }
-    }
-#pragma unroll
-    for (int r = 0; r < RBM; ++r)
-#pragma unroll
-      for (int o = 16; o > 0; o >>= 1) pd[r] += __shfl_xor_sync(0xffffffffu, pd[r], o);
-    float* redn = red + (n & 1) * NW * RBM;
-    if (lane == 0)
-#pragma unroll
-      for (int r = 0; r < RBM; ++r) redn[warp * RBM + r] = pd[r];
-    __syncthreads();
-    // the previous stage is free now: refill it with batch n - 1 + S
-    if (a.use_tma && tid == 0 && n >= 1 && n - 1 + a.S < nb && !s_abort) issue(n - 1 + a.S);
-    float z[RBM];
-#pragma unroll
-    for (int r = 0; r < RBM; ++r) {
-      float t = 0.f;
-      for (int w = 0; w < NW; ++w) t += redn[w * RBM + r];
-      z[r] = t;
-    }
-    if (CL > 1) {
-      float* zc = zcl + (n & 1) * CL * RBM;
-      if (tid < CL * RBM) {
-        const int peer = tid / RBM, r = tid % RBM;
-        st_cluster_f32(mapa(smem_u32(zc + rank * RBM + r), peer), z[r]);
-      }
-      cluster_sync_all();
+        for (int r = 0; r < RBM; ++r) redn[warp * RBM + r] = pd[r];
+      consumer_sync(NT);
+      // every warp reduces the NW partials redundantly (lane w holds warp w's,
+      // zeros past NW), then a full xor tree: identical sums in every lane
 #pragma unroll
       for (int r = 0; r < RBM; ++r) {
-        float t = 0.f;
-        for (int p = 0; p < CL; ++p) t += zc[p * RBM + r];
+        float t = lane < NW ? redn[lane * RBM + r] : 0.f;
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) t += __shfl_xor_sync(0xffffffffu, t, o);
         z[r] = t;
       }
-    }
-    // ---- residuals
-    float res[RBM];
+      if (CL > 1 && tid < CL) {
+        // thread p writes the CTA sums into peer p's slot and arrives there (release)
+        float* zc = zcl + (n % kZSlots) * CL * RBM;
+        const uint32_t peer = (uint32_t)tid;
 #pragma unroll
-    for (int r = 0; r < RBM; ++r) {
-      res[r] = 0.f;
-      if (r < a.RB) {
-        const float yv = __ldg(a.y + row0 + r);
-        if (a.loss == GC_LSQ) {
-          res[r] = z[r] - yv;
-        } else {
-          const float sg = 1.f / (1.f + __expf(-z[r]));
-          res[r] = sg - 0.5f * (yv + 1.f);
+        for (int r = 0; r < RBM; ++r)
+          st_cluster_f32(mapa(smem_u32(zc + rank * RBM + r), peer), z[r]);
+        mbar_arrive_remote(&zfull[n % kZSlots], peer);
+      }
+    };
+
+    float znext[RBM];
+    if (nb > 0) pass1(0, znext);
+    for (int n = 0; n < nb; ++n) {
+      const int s = n % a.S;
+      const long long row0 = r0 + (long long)n * a.RB;
+      const long long chunk = row0 / a.n_c;
+      float z[RBM];
+#pragma unroll
+      for (int r = 0; r < RBM; ++r) z[r] = znext[r];
+      // software pipelining: batch n + 1's pass 1 (and its send) before the
+      // wait for batch n's cluster sums
+      if (n + 1 < nb) pass1(n + 1, znext);
+      if (CL > 1) {
+        bounded_wait(&zfull[n % kZSlots], (uint32_t)((n / kZSlots) & 1), abort_flag, a.status,
+                     true);
+        const float* zc = zcl + (n % kZSlots) * CL * RBM;
+#pragma unroll
+        for (int r = 0; r < RBM; ++r) {
+          float t = 0.f;
+          for (int p = 0; p < CL; ++p) t += zc[p * RBM + r];
+          z[r] = t;
         }
       }
-    }
-    // ---- the loss: lane r of warp 0 takes row r (fp32), one fp64 add per batch
-    if (a.want_loss && rank == 0 && warp == 0) {
-      float lr = 0.f;
+      if (chunk != cur) {
+        if (cur >= 0) flush(cur);
+#pragma unroll
+        for (int u = 0; u < NVT; ++u)
+#pragma unroll
+          for (int e = 0; e < V; ++e) acc[u][e] = 0.f;
+        cur = chunk;
+      }
+      const T* st = stages + s * stage_elems;
+      // ---- residuals: lane r takes row r, then broadcast
+      float res[RBM];
+      {
+        float mine = 0.f;
+#pragma unroll
+        for (int r = 0; r < RBM; ++r) {
+          if (lane == r && r < a.RB) {
+            const float yv = __ldg(a.y + row0 + r);
+            if (a.loss == GC_LSQ) {
+              mine = z[r] - yv;
+            } else {
+              const float sg = 1.f / (1.f + __expf(-z[r]));
+              mine = sg - 0.5f * (yv + 1.f);
+            }
+          }
+        }
+#pragma unroll
+        for (int r = 0; r < RBM; ++r) res[r] = __shfl_sync(0xffffffffu, mine, r);
+      }
+      // ---- the loss: lane r of warp 0 takes row r (fp32), one fp64 add per batch
+      if (a.want_loss && rank == 0 && warp == 0) {
+        float lr = 0.f;
+#pragma unroll
+        for (int r = 0; r < RBM; ++r) {
+          if (r < a.RB && lane == r) {
+            const float yv = __ldg(a.y + row0 + r);
+            if (a.loss == GC_LSQ) {
+              const float e = z[r] - yv;
+              lr = 0.5f * e * e;
+            } else {
+              const float t = -yv * z[r];  // log(1 + e^t), stable
+              lr = fmaxf(t, 0.f) + log1pf(expf(-fabsf(t)));
+            }
+          }
+        }
+#pragma unroll
+        for (int o = 2; o > 0; o >>= 1) lr += __shfl_xor_sync(0xffffffffu, lr, o);
+        if (lane == 0) loss_acc += (double)lr;
+      }
+      // ---- pass 2: acc += r * x, then hand the stage back to the producer
 #pragma unroll
       for (int r = 0; r < RBM; ++r) {
-        if (r < a.RB && lane == r) {
-          const float yv = __ldg(a.y + row0 + r);
-          if (a.loss == GC_LSQ) {
-            const float e = z[r] - yv;
-            lr = 0.5f * e * e;
-          } else {
-            const float t = -yv * z[r];  // log(1 + e^t), stable
-            lr = fmaxf(t, 0.f) + log1pf(expf(-fabsf(t)));
+        if (r < a.RB) {
+#pragma unroll
+          for (int u = 0; u < NVT; ++u) {
+            const int v = tid + u * NT;
+            if (v < nvs) {
+              float x[V];
+              Vec<T>::load(st + (size_t)r * a.ld_s + v * V, x);
+#pragma unroll
+              for (int e = 0; e < V; ++e) acc[u][e] = fmaf(res[r], x[e], acc[u][e]);
+            }
           }
         }
       }
-#pragma unroll
-      for (int o = 2; o > 0; o >>= 1) lr += __shfl_xor_sync(0xffffffffu, lr, o);
-      if (lane == 0) loss_acc += (double)lr;
+      __syncwarp();
+      if (lane == 0) mbar_arrive_local(&empty[s]);
     }
-    // ---- pass 2: acc += r * x
-#pragma unroll
-    for (int r = 0; r < RBM; ++r) {
-      if (r < a.RB) {
-#pragma unroll
-        for (int u = 0; u < NVT; ++u) {
-          const int v = tid + u * NT;
-          if (v < nvs) {
-            float x[V];
-            Vec<T>::load(st + (size_t)r * a.ld_s + v * V, x);
-#pragma unroll
-            for (int e = 0; e < V; ++e) acc[u][e] = fmaf(res[r], x[e], acc[u][e]);
-          }
-        }
-      }
-    }
-    if (!a.use_tma) __syncthreads();
+    if (cur >= 0) flush(cur);
+    if (tid == 0 && rank == 0) a.loss_parts[q] = loss_acc;
   }
-  if (cur >= 0) flush(cur);
-  if (tid == 0 && rank == 0) a.loss_parts[q] = loss_acc;
-  if (CL > 1) cluster_sync_all();  // keep shared memory alive until peers are done
+  if (CL > 1) cluster_sync_all();  // no CTA leaves while a peer may still address it
 }
 
 // G[i][col] = sum of the partials of chunk i, clusters in increasing order.
@@ -381,10 +457,13 @@ __global__ void k_chunkgrad_reduce(const float* __restrict__ parts,
     }
     G[idx] = s;
   }
-  if (loss_out && idx == 0) {
+  if (loss_out && blockIdx.x == 0 && threadIdx.x < 32) {
+    // lane l adds clusters l, l + 32, ...; then a fixed xor tree
     double t = 0.0;
-    for (int q = 0; q < nclusters; ++q) t += loss_parts[q];
-    *loss_out = t / (double)Ntil;
+    for (int q = threadIdx.x; q < nclusters; q += 32) t += loss_parts[q];
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) t += __shfl_xor_sync(0xffffffffu, t, o);
+    if (threadIdx.x == 0) *loss_out = t / (double)Ntil;
   }
 }
 
@@ -393,39 +472,53 @@ __global__ void k_chunkgrad_reduce(const float* __restrict__ parts,
 // ---------------------------------------------------------------------------
 struct Plan {
   int CL, NT, NVT, RBM, RB, S, Wc, ld_s, V, use_tma;
+  bool valid;
   long long rpc;
   int nclusters, maxt;
   size_t smem;
 };
 
+int max_active_clusters(const Plan& p, int x_dtype);
+
 Plan make_plan(int N, int n_c, int d, int x_dtype, bool tma_ok) {
   Plan p{};
+  // Two CTAs per SM (two independent TMA rings) when each one still streams
+  // many rows; one when the rows per SM are few (ramp-up dominates) or a
+  // cluster is needed.  Chosen from measurements on GB300.
+  const long long rows_per_sm = (long long)N * n_c / std::max(1, device_sm_count());
+  const long long row_bytes0 = (long long)d * (x_dtype == GC_BF16 ? 2 : 4);
+  const int cps = (rows_per_sm >= 512 && row_bytes0 <= 16384) ? 2 : 1;
   const int esz = x_dtype == GC_BF16 ? 2 : 4;
   p.V = 16 / esz;
   // cluster size: row slice per CTA at most 32 KB
   const long long row_bytes = (long long)d * esz;
+  // per-CTA row slice at most 32 KB (fp32) / 16 KB (bf16: unpacking needs
+  // registers), so every thread holds at most 16 (fp32) or 16 (bf16) columns
+  const long long max_slice = x_dtype == GC_BF16 ? 16384 : 32768;
   p.CL = 1;
-  while (p.CL < 8 && row_bytes / p.CL > 32768) p.CL *= 2;
+  while (p.CL < 8 && row_bytes / p.CL > max_slice) p.CL *= 2;
   p.use_tma = tma_ok && (row_bytes % 16 == 0) && (d % (p.CL * p.V) == 0);
   p.Wc = p.use_tma ? d / p.CL : (int)align_up((size_t)((d + p.CL - 1) / p.CL), (size_t)p.V);
   p.ld_s = p.Wc;  // stage row stride (elements)
-  const int nv = p.Wc / p.V;
+  const int nv = p.Wc / p.V;  // 16-byte vectors per row slice (<= 2048 by the slice caps)
   p.NT = nv >= 1024 ? 512 : (nv >= 256 ? 256 : 128);
-  p.NVT = (nv + p.NT - 1) / p.NT;
-  if (p.NVT > 4) p.NVT = 4;  // nv <= 4 * 512 because Wc * esz <= 32 KB
-  p.NVT = p.NVT <= 1 ? 1 : (p.NVT <= 2 ? 2 : 4);
+  if (cps == 2 && p.NT == 512) p.NT = 256;  // only when nv <= 1024 (16 KB slices)
+  const int need = (nv + p.NT - 1) / p.NT;
+  p.NVT = need <= 1 ? 1 : (need <= 2 ? 2 : 4);
+  p.valid = (long long)p.NVT * p.NT >= nv;  // every vector of the slice has a thread
   p.RBM = p.NVT >= 4 ? 2 : 4;
   p.RB = p.RBM;
   while (p.RB > 1 && n_c % p.RB != 0) p.RB /= 2;
   const size_t stage_bytes = (size_t)p.RBM * p.ld_s * esz;
-  p.S = (int)std::min<size_t>(kMaxStages, std::max<size_t>(2, (192 * 1024) / stage_bytes));
+  p.S = (int)std::min<size_t>(kMaxStages, std::max<size_t>(2, (192 * 1024 / cps) / stage_bytes));
   const int NW = p.NT / 32;
-  p.smem = p.S * stage_bytes + (2 * NW * p.RBM + 2 * p.CL * p.RBM + 2) * sizeof(float) +
-           kMaxStages * sizeof(uint64_t) + 16;
+  p.smem = p.S * stage_bytes + (2 * NW * p.RBM + kZSlots * p.CL * p.RBM + 2) * sizeof(float) +
+           (2 * kMaxStages + kZSlots) * sizeof(uint64_t) + 16;
   // flat row partition over one wave of clusters
   const int sms = device_sm_count();
   const long long Ntil = (long long)N * n_c;
-  long long waves_cl = std::max(1, sms / p.CL);
+  long long waves_cl = std::max(1, sms * cps / p.CL);
+  if (p.CL > 1) waves_cl = std::max(1, std::min<int>((int)waves_cl, max_active_clusters(p, x_dtype)));
   long long rpc = (Ntil + waves_cl - 1) / waves_cl;
   rpc = ((rpc + p.RB - 1) / p.RB) * p.RB;
   if (rpc < p.RB) rpc = p.RB;
@@ -447,7 +540,7 @@ int launch_one(const Plan& p, const CGArgs& a, cudaStream_t s) {
   }
   cudaLaunchConfig_t cfg{};
   cfg.gridDim = dim3(p.nclusters * CL);
-  cfg.blockDim = dim3(NT);
+  cfg.blockDim = dim3(NT + 32);  // consumers + the producer warp
   cfg.dynamicSmemBytes = p.smem;
   cfg.stream = s;
   cudaLaunchAttribute attr[1];
@@ -487,6 +580,62 @@ int dispatch_cl(const Plan& p, const CGArgs& a, cudaStream_t s) {
   }
 }
 
+template <typename T, int CL, int NT, int NVT, int RBM>
+int occ_one(const Plan& p) {
+  auto kern = k_chunkgrad<T, CL, NT, NVT, RBM>;
+  if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)p.smem) !=
+      cudaSuccess)
+    return 1;
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = dim3(CL * 64);
+  cfg.blockDim = dim3(NT + 32);
+  cfg.dynamicSmemBytes = p.smem;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = CL;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  int n = 0;
+  if (cudaOccupancyMaxActiveClusters(&n, kern, &cfg) != cudaSuccess || n < 1) {
+    cudaGetLastError();
+    return 1;
+  }
+  return n;
+}
+template <typename T, int CL>
+int occ_nt(const Plan& p) {
+  if (p.NT == 512) {
+    if (p.NVT == 4) return occ_one<T, CL, 512, 4, 2>(p);
+    if (p.NVT == 2) return occ_one<T, CL, 512, 2, 4>(p);
+    return occ_one<T, CL, 512, 1, 4>(p);
+  }
+  if (p.NT == 256) {
+    if (p.NVT == 4) return occ_one<T, CL, 256, 4, 2>(p);
+    return occ_one<T, CL, 256, 1, 4>(p);
+  }
+  return occ_one<T, CL, 128, 1, 4>(p);
+}
+template <typename T>
+int occ_cl(const Plan& p) {
+  switch (p.CL) {
+    case 2: return occ_nt<T, 2>(p);
+    case 4: return occ_nt<T, 4>(p);
+    default: return occ_nt<T, 8>(p);
+  }
+}
+// Clusters of this plan that can be resident at once (cached per shape).
+int max_active_clusters(const Plan& p, int x_dtype) {
+  static int cache[2][4][3][3] = {};
+  const int ci = p.CL == 2 ? 1 : (p.CL == 4 ? 2 : 3);
+  const int ni = p.NT == 512 ? 0 : (p.NT == 256 ? 1 : 2);
+  const int vi = p.NVT == 4 ? 0 : (p.NVT == 2 ? 1 : 2);
+  int& c = cache[x_dtype == GC_BF16][ci][ni][vi];
+  if (c == 0) c = x_dtype == GC_BF16 ? occ_cl<__nv_bfloat16>(p) : occ_cl<float>(p);
+  return c;
+}
+
 }  // namespace
 
 size_t chunkgrad_ws_bytes(int N, int n_c, int d, int x_dtype) {
@@ -503,6 +652,7 @@ int launch_chunkgrad(const void* X, int x_dtype, const float* y, const float* w,
                      cudaStream_t s) {
   const bool aligned = (reinterpret_cast<uintptr_t>(X) % 16) == 0;
   const Plan p = make_plan(N, n_c, d, x_dtype, aligned);
+  if (!p.valid) return fail(GC_ERR_UNSUPPORTED, "chunk-gradient plan does not cover d=%d", d);
   CGArgs a{};
   a.X = X;
   a.y = y;

@@ -31,6 +31,8 @@
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
+#include <string.h>
+
 #include <algorithm>
 
 #include "gc_internal.cuh"
@@ -38,23 +40,34 @@
 namespace gc {
 namespace tc {
 
-constexpr int BM = 128, BN = 256, BK = 64, STAGES = 2;
+constexpr int BM = 128, BN = 256, BK = 64;
 constexpr int A_PLANE = BM * BK * 2;                 // bytes of one bf16 plane (16 KB)
 constexpr int B_PLANE = BN * BK * 2;                 // 32 KB
 constexpr int STAGE_BYTES = 2 * A_PLANE + 2 * B_PLANE;  // 96 KB
-constexpr int THREADS = 192;
 constexpr uint32_t TMEM_COLS = 512;
 constexpr long long kSpin = 1LL << 32;  // clock cycles per wait (~2 s)
-constexpr size_t SMEM_BYTES = (size_t)STAGES * STAGE_BYTES + 1024 + 256;
+constexpr int OUT_BUF = 32 * 32 * 4;                 // one 32 x 32 fp32 store box (4 KB)
+// Two shapes: STAGES = 2 smem stages with 4 epilogue warps when K spans
+// several 64-wide blocks (MMA-bound), STAGES = 1 with 8 epilogue warps (two
+// per TMEM lane quarter, half the columns each) when one block holds all of
+// K and the output write bounds the kernel.
+template <int STAGES, int EPI>
+struct Shape {
+  static constexpr int THREADS = 64 + 32 * EPI;
+  static constexpr int OUT_BYTES = EPI * 2 * OUT_BUF;  // 2 staging boxes per epilogue warp
+  static constexpr size_t SMEM = (size_t)STAGES * STAGE_BYTES + OUT_BYTES + 1024 + 256;
+};
 
 struct Params {
-  int M, Kp, L, ell, d;
+  int M, K, Kp, L, ell, d;
   int num_m_tiles, num_n_tiles, nkb;
   long long num_tiles;
   int vec_ok;           // d % 4 == 0 && L % 4 == 0: 16-byte row segments
+  int tma_store;        // Ghat written by TMA tensor stores (needs d == ell * L, L % 4 == 0)
   float* Ghat;          // npat x d or null
   const float* gsum;    // d, or null when no MSE is wanted
-  float* msep;          // M x num_n_tiles partial squared errors, or null
+  float* msep;          // M x parts_per_row partial squared errors, or null
+  int parts_per_row;    // num_n_tiles * (epilogue warps per TMEM lane quarter)
   uint32_t* status;
 };
 
@@ -105,6 +118,22 @@ __device__ __forceinline__ void tma_load_3d(void* dst, const CUtensorMap* map, i
       "[%0], [%1, {%2, %3, %4}], [%5];" ::"r"(smem_u32(dst)),
       "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(z), "r"(smem_u32(bar))
       : "memory");
+}
+__device__ __forceinline__ void tma_store_2d(const CUtensorMap* map, const void* src, int x, int y) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.global.shared::cta.bulk_group [%0, {%1, %2}], [%3];" ::"l"(
+          reinterpret_cast<uint64_t>(map)),
+      "r"(x), "r"(y), "r"(smem_u32(src))
+      : "memory");
+}
+__device__ __forceinline__ void bulk_commit() {
+  asm volatile("cp.async.bulk.commit_group;" ::: "memory");
+}
+__device__ __forceinline__ void bulk_wait_read1() {
+  asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory");
+}
+__device__ __forceinline__ void bulk_wait_all() {
+  asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
 }
 // Shared-memory matrix descriptor: K-major, 128-byte swizzle, 8-row groups
 // 1024 bytes apart (stride byte offset), descriptor version 1.
@@ -158,13 +187,16 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
   for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(r[j]);
 }
 
-__global__ void __launch_bounds__(THREADS, 1)
+template <int STAGES, int EPI>
+__global__ void __launch_bounds__(64 + 32 * EPI, 1)
     k_combine_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
-                 Params p) {
+                 const __grid_constant__ CUtensorMap tmC, Params p) {
+  constexpr int OUT_BYTES = Shape<STAGES, EPI>::OUT_BYTES;
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
-  uint64_t* full = reinterpret_cast<uint64_t*>(smem + STAGES * STAGE_BYTES);
+  float* outbuf = reinterpret_cast<float*>(smem + STAGES * STAGE_BYTES);  // 1024-aligned
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + STAGES * STAGE_BYTES + OUT_BYTES);
   uint64_t* empty = full + STAGES;
   uint64_t* tfull = empty + STAGES;   // [2]
   uint64_t* tempty = tfull + 2;       // [2]
@@ -180,7 +212,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init(&tfull[a], 1);
-      mbar_init(&tempty[a], 4);
+      mbar_init(&tempty[a], EPI);
     }
     mbar_init(done, 1);
     *abort_flag = 0;
@@ -247,7 +279,7 @@ __global__ void __launch_bounds__(THREADS, 1)
           const uint32_t a_lo = a_hi + A_PLANE;
           const uint32_t b_hi = a_hi + 2 * A_PLANE;
           const uint32_t b_lo = b_hi + B_PLANE;
-          const int rem = p.Kp - kb * BK;
+          const int rem = p.K - kb * BK;
           const int nks = rem >= BK ? BK / 16 : (rem + 15) / 16;
           for (int ks = 0; ks < nks; ++ks) {
             const uint32_t off = ks * 32;  // 16 bf16 along K inside the swizzle atom
@@ -269,7 +301,11 @@ __global__ void __launch_bounds__(THREADS, 1)
   } else {
     // ------------------------------------------------------------- epilogue
     const int quarter = warp & 3;  // TMEM lanes 32*quarter .. +31
-    uint32_t tile_it = 0;
+    const int e = warp - 2;        // epilogue warp index
+    constexpr int SPAN = BN / (EPI / 4);  // columns per epilogue warp
+    const int cbeg = (e / 4) * SPAN;
+    float* wbuf = outbuf + e * 2 * (OUT_BUF / 4);
+    uint32_t tile_it = 0, chunk_it = 0;
     for (long long t = blockIdx.x; t < p.num_tiles; t += gridDim.x, ++tile_it) {
       const int ab = tile_it & 1;
       const int nt = (int)(t / p.num_m_tiles), mt = (int)(t % p.num_m_tiles);
@@ -284,26 +320,59 @@ __global__ void __launch_bounds__(THREADS, 1)
       const float* gs = p.gsum ? p.gsum + (size_t)k * p.L : nullptr;
       float sq = 0.f;
       const uint32_t taddr = tmem_base + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(ab * BN);
+      // the fast path's reference values are loaded one chunk ahead
+      const bool fast_gs = gs && p.vec_ok && rv;
+      float4 gnext[8];
+      if (fast_gs && n0 + cbeg + 32 <= p.L) {
+#pragma unroll
+        for (int j = 0; j < 8; ++j)
+          gnext[j] = __ldg(reinterpret_cast<const float4*>(gs + n0 + cbeg) + j);
+      }
 #pragma unroll 1
-      for (int cc = 0; cc < BN; cc += 32) {
+      for (int cc = cbeg; cc < cbeg + SPAN; cc += 32) {
         float v[32];
+        float4 gcur[8];
+#pragma unroll
+        for (int j = 0; j < 8; ++j) gcur[j] = gnext[j];
+        if (fast_gs && cc + 32 < cbeg + SPAN && n0 + cc + 64 <= p.L) {
+#pragma unroll
+          for (int j = 0; j < 8; ++j)
+            gnext[j] = __ldg(reinterpret_cast<const float4*>(gs + n0 + cc + 32) + j);
+        }
         __syncwarp();
         tmem_ld32(taddr + cc, v);  // warp-collective: every lane, every chunk
         const int c0 = n0 + cc;
+        if (p.tma_store && c0 < p.L) {
+          // stage the 32 x 32 box (row = lane) with the 128-byte swizzle, then one TMA store
+          float* buf = wbuf + (chunk_it & 1) * (OUT_BUF / 4);
+          if (lane == 0) bulk_wait_read1();  // the store that used this buffer has read it
+          __syncwarp();
+          char* rowp = reinterpret_cast<char*>(buf) + lane * 128;
+#pragma unroll
+          for (int j = 0; j < 8; ++j)
+            *reinterpret_cast<float4*>(rowp + ((j ^ (lane & 7)) << 4)) =
+                make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
+          asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+          __syncwarp();
+          if (lane == 0) {
+            tma_store_2d(&tmC, buf, c0, mt * BM + quarter * 32);
+            bulk_commit();
+          }
+          ++chunk_it;
+        }
         const int lim = (rv && c0 < p.L) ? min(32, min(p.L - c0, p.d - k * p.L - c0)) : 0;
         if (lim <= 0) {
         } else if (lim == 32 && p.vec_ok) {
-          if (out) {
+          if (out && !p.tma_store) {
             float4* o4 = reinterpret_cast<float4*>(out + c0);
 #pragma unroll
             for (int j = 0; j < 8; ++j)
               o4[j] = make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
           }
           if (gs) {
-            const float4* g4 = reinterpret_cast<const float4*>(gs + c0);
 #pragma unroll
             for (int j = 0; j < 8; ++j) {
-              const float4 g = __ldg(g4 + j);
+              const float4 g = gcur[j];
               float df = v[4 * j] - g.x;
               sq = fmaf(df, df, sq);
               df = v[4 * j + 1] - g.y;
@@ -318,7 +387,7 @@ __global__ void __launch_bounds__(THREADS, 1)
 #pragma unroll
           for (int j = 0; j < 32; ++j) {
             if (j < lim) {
-              if (out) out[c0 + j] = v[j];
+              if (out && !p.tma_store) out[c0 + j] = v[j];
               if (gs) {
                 const float df = v[j] - __ldg(gs + c0 + j);
                 sq = fmaf(df, df, sq);
@@ -330,8 +399,9 @@ __global__ void __launch_bounds__(THREADS, 1)
       fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&tempty[ab]);
-      if (p.msep && rv) p.msep[(size_t)row * p.num_n_tiles + nt] = sq;
+      if (p.msep && rv) p.msep[(size_t)row * p.parts_per_row + nt * (EPI / 4) + e / 4] = sq;
     }
+    if (lane == 0) bulk_wait_all();  // every store of this warp has completed
   }
   fence_before();
   __syncthreads();
@@ -391,13 +461,13 @@ __global__ void k_split_gt(const float* __restrict__ G, int N, int d, int ell, i
 }
 
 __global__ void k_mse_reduce_tiles(const float* __restrict__ msep, int npat, int ell,
-                                   int num_n_tiles, int d, double* __restrict__ grad_mse) {
+                                   int parts, int d, double* __restrict__ grad_mse) {
   const int b = blockIdx.x * blockDim.x + threadIdx.x;
   if (b >= npat) return;
   double s = 0.0;
   for (int k = 0; k < ell; ++k) {
-    const float* r = msep + ((size_t)b * ell + k) * num_n_tiles;
-    for (int t = 0; t < num_n_tiles; ++t) s += (double)r[t];
+    const float* r = msep + ((size_t)b * ell + k) * parts;
+    for (int t = 0; t < parts; ++t) s += (double)r[t];
   }
   grad_mse[b] = s / (double)d;
 }
@@ -413,6 +483,22 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
       fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(ptr);
   }
   return fn;
+}
+
+// 2-D fp32 map over Ghat viewed as (npat*ell) rows of L (requires d == ell*L),
+// box 32 x 32, 128-byte swizzle (matches the epilogue's staging layout).
+int make_out_map(CUtensorMap* map, float* base, long long rows, int L) {
+  auto fn = encode_fn();
+  if (!fn) return fail(GC_ERR_CUDA, "cuTensorMapEncodeTiled entry point unavailable");
+  cuuint64_t dims[2] = {(cuuint64_t)L, (cuuint64_t)rows};
+  cuuint64_t strides[1] = {(cuuint64_t)L * 4};
+  cuuint32_t box[2] = {32, 32};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, base, dims, strides, box, estr,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                  CU_TENSOR_MAP_L2_PROMOTION_NONE, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) return fail(GC_ERR_CUDA, "cuTensorMapEncodeTiled(out) failed (%d)", (int)r);
+  return GC_OK;
 }
 
 // 3-D map over [2][rows][Kp] bf16 planes, box {64, box_rows, 2}, 128-byte swizzle.
@@ -432,14 +518,30 @@ int make_map(CUtensorMap* map, const void* base, int rows, int Kp, int box_rows)
 
 }  // namespace tc
 
+template <int STAGES, int EPI>
+int launch_tc(int grid, const CUtensorMap& mA, const CUtensorMap& mB, const CUtensorMap& mC,
+              const tc::Params& p, cudaStream_t s) {
+  using Sh = tc::Shape<STAGES, EPI>;
+  static bool attr_set = false;
+  if (!attr_set) {
+    cudaError_t e = cudaFuncSetAttribute(tc::k_combine_tc<STAGES, EPI>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)Sh::SMEM);
+    if (e != cudaSuccess) return cuda_check(e, "cudaFuncSetAttribute(k_combine_tc)");
+    attr_set = true;
+  }
+  tc::k_combine_tc<STAGES, EPI><<<grid, Sh::THREADS, Sh::SMEM, s>>>(mA, mB, mC, p);
+  count_launches(1);
+  return cuda_check(cudaGetLastError(), "k_combine_tc");
+}
+
 size_t combine_tc_ws_bytes(int N, int ell, int npat, int d) {
   const int L = (d + ell - 1) / ell;
   const long long M = (long long)npat * ell;
   const int K = N * ell;
-  const int Kp = (K + 7) / 8 * 8;
+  const int Kp = (K + tc::BK - 1) / tc::BK * tc::BK;
   const int nnt = (L + tc::BN - 1) / tc::BN;
   return align_up((size_t)2 * M * Kp * 2, 256) + align_up((size_t)2 * L * Kp * 2, 256) +
-         align_up((size_t)M * nnt * sizeof(float), 256);
+         align_up((size_t)M * nnt * 2 * sizeof(float), 256);
 }
 
 int launch_combine_tc(const float* C, const float* G, const float* gsum, int N, int ell, int npat,
@@ -449,12 +551,13 @@ int launch_combine_tc(const float* C, const float* G, const float* gsum, int N, 
   const int L = (d + ell - 1) / ell;
   const long long M = (long long)npat * ell;
   const int K = N * ell;
-  const int Kp = (K + 7) / 8 * 8;
+  // K padded to whole 64-element blocks: every TMA row is one aligned 128-byte line
+  const int Kp = (K + BK - 1) / BK * BK;
   if (M > (1LL << 31) - 1) return fail(GC_ERR_UNSUPPORTED, "npat*ell too large");
   const int nmt = (int)((M + BM - 1) / BM), nnt = (L + BN - 1) / BN;
   __nv_bfloat16* Cs = ws.take<__nv_bfloat16>((size_t)2 * M * Kp);
   __nv_bfloat16* Gs = ws.take<__nv_bfloat16>((size_t)2 * L * Kp);
-  float* msep = grad_mse ? ws.take<float>((size_t)M * nnt) : nullptr;
+  float* msep = grad_mse ? ws.take<float>((size_t)M * nnt * 2) : nullptr;
 
   {
     const long long tot = M * Kp;
@@ -466,13 +569,21 @@ int launch_combine_tc(const float* C, const float* G, const float* gsum, int N, 
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return cuda_check(e, "split kernels");
   }
-  CUtensorMap mA, mB;
+  CUtensorMap mA, mB, mC;
   int rc = make_map(&mA, Cs, (int)M, Kp, BM);
   if (rc) return rc;
   rc = make_map(&mB, Gs, L, Kp, BN);
   if (rc) return rc;
+  const bool tma_store = Ghat && (long long)ell * L == d && L % 4 == 0 &&
+                         reinterpret_cast<uintptr_t>(Ghat) % 16 == 0;
+  memset(&mC, 0, sizeof(mC));
+  if (tma_store) {
+    rc = make_out_map(&mC, Ghat, M, L);
+    if (rc) return rc;
+  }
   Params p{};
   p.M = (int)M;
+  p.K = K;
   p.Kp = Kp;
   p.L = L;
   p.ell = ell;
@@ -482,25 +593,21 @@ int launch_combine_tc(const float* C, const float* G, const float* gsum, int N, 
   p.nkb = (Kp + BK - 1) / BK;
   p.num_tiles = (long long)nmt * nnt;
   p.vec_ok = (d % 4 == 0) && (L % 4 == 0);
+  p.tma_store = tma_store ? 1 : 0;
   p.Ghat = Ghat;
   p.gsum = grad_mse ? gsum : nullptr;
   p.msep = msep;
   p.status = status;
-  static bool attr_set = false;
-  if (!attr_set) {
-    cudaError_t e = cudaFuncSetAttribute(k_combine_tc, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         (int)SMEM_BYTES);
-    if (e != cudaSuccess) return cuda_check(e, "cudaFuncSetAttribute(k_combine_tc)");
-    attr_set = true;
-  }
+  const bool one_block = p.nkb == 1;
+  p.parts_per_row = nnt * (one_block ? 2 : 1);
   const int sms = device_sm_count();
   const int grid = (int)std::min<long long>(p.num_tiles, sms);
-  k_combine_tc<<<grid, THREADS, SMEM_BYTES, s>>>(mA, mB, p);
-  count_launches(1);
-  cudaError_t e = cudaGetLastError();
-  if (e != cudaSuccess) return cuda_check(e, "k_combine_tc");
+  int rc2 = one_block ? launch_tc<1, 8>(grid, mA, mB, mC, p, s) : launch_tc<2, 4>(grid, mA, mB, mC, p, s);
+  if (rc2) return rc2;
+  cudaError_t e;
   if (grad_mse) {
-    k_mse_reduce_tiles<<<(npat + 255) / 256, 256, 0, s>>>(msep, npat, ell, nnt, d, grad_mse);
+    k_mse_reduce_tiles<<<(npat + 255) / 256, 256, 0, s>>>(msep, npat, ell, p.parts_per_row, d,
+                                                         grad_mse);
     count_launches(1);
     e = cudaGetLastError();
     if (e != cudaSuccess) return cuda_check(e, "k_mse_reduce_tiles");

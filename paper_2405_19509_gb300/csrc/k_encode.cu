@@ -8,51 +8,61 @@
 namespace gc {
 
 // T[b][j][c] = sum_{p < psi[b][j]} sum_k E[b][j][p][k] * g_{order[j][p]}[k*L + c]
-// (g zero past d).  One thread per (b, j, c).
+// (g zero past d).  Block = (column tile, worker j, pattern b); worker j's
+// coefficients and chunk list are staged in shared memory (fp32) once per
+// block.
 __global__ void k_encode(const double* __restrict__ E, const int32_t* __restrict__ order,
                          const int32_t* __restrict__ psi, int N, int m, int delta, int ell,
                          int npat, const float* __restrict__ G, int d, int L,
                          float* __restrict__ T) {
-  const long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;
-  const long long tot = (long long)npat * m * L;
-  if (idx >= tot) return;
-  const int c = (int)(idx % L);
-  const long long bj = idx / L;
-  const int j = (int)(bj % m);
-  const int b = (int)(bj / m);
+  __shared__ float s_e[GC_MAX_DELTA * GC_MAX_ELL];
+  __shared__ int s_chunk[GC_MAX_DELTA];
+  const int j = blockIdx.y, b = blockIdx.z;
   int np = psi[(size_t)b * m + j];
   np = np < 0 ? 0 : (np > delta ? delta : np);  // bad values are flagged by the solve
   const double* Ej = E + ((size_t)b * m + j) * delta * ell;
+  for (int t = threadIdx.x; t < np * ell; t += blockDim.x) s_e[t] = (float)Ej[t];
+  for (int t = threadIdx.x; t < np; t += blockDim.x) s_chunk[t] = order[(size_t)j * delta + t];
+  __syncthreads();
+  const int c = blockIdx.x * blockDim.x + threadIdx.x;
+  if (c >= L) return;
   float acc = 0.f;
+#pragma unroll 4
   for (int p = 0; p < np; ++p) {
-    const int i = order[(size_t)j * delta + p];
+    const int i = s_chunk[p];
     if (i < 0 || i >= N) continue;
     const float* gi = G + (size_t)i * d;
     for (int k = 0; k < ell; ++k) {
       const int col = k * L + c;
-      if (col < d) acc = fmaf((float)Ej[p * ell + k], __ldg(gi + col), acc);
+      if (col < d) acc = fmaf(s_e[p * ell + k], __ldg(gi + col), acc);
     }
   }
-  T[idx] = acc;
+  T[((size_t)b * m + j) * L + c] = acc;
 }
 
 int launch_encode(const double* E, const int32_t* order, const int32_t* psi, int N, int m,
                   int delta, int ell, int npat, const float* G, int d, float* T, cudaStream_t s) {
   const int L = (d + ell - 1) / ell;
-  const long long tot = (long long)npat * m * L;
-  if (tot == 0) return GC_OK;
+  if ((long long)npat * m * L == 0) return GC_OK;
+  if (npat > 65535 || m > 65535) return fail(GC_ERR_UNSUPPORTED, "encode grid: npat and m <= 65535");
   const int threads = 256;
-  k_encode<<<(unsigned)((tot + threads - 1) / threads), threads, 0, s>>>(E, order, psi, N, m,
-                                                                         delta, ell, npat, G, d, L,
-                                                                         T);
+  dim3 grid((L + threads - 1) / threads, m, npat);
+  k_encode<<<grid, threads, 0, s>>>(E, order, psi, N, m, delta, ell, npat, G, d, L, T);
   count_launches(1);
   return cuda_check(cudaGetLastError(), "k_encode");
 }
 
-// ghat[b][k*L + c] = sum_j R[k][j] * T[b][j][c].  One thread per (b, c).
+// ghat[b][k*L + c] = sum_j R[k][j] * T[b][j][c].  One thread per (b, c); R is
+// staged in shared memory as fp32 (m <= kDecodeSmemM) or read as fp64.
+constexpr int kDecodeSmemM = 1024;
 template <int ELL>
 __global__ void k_decode_tx(const double* __restrict__ R, int m, const float* __restrict__ T,
                             int npat, int d, int L, float* __restrict__ ghat) {
+  __shared__ float s_r[ELL * kDecodeSmemM];
+  const bool staged = m <= kDecodeSmemM;
+  if (staged)
+    for (int t = threadIdx.x; t < ELL * m; t += blockDim.x) s_r[t] = (float)R[t];
+  __syncthreads();
   const long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;
   if (idx >= (long long)npat * L) return;
   const int c = (int)(idx % L);
@@ -61,10 +71,14 @@ __global__ void k_decode_tx(const double* __restrict__ R, int m, const float* __
 #pragma unroll
   for (int k = 0; k < ELL; ++k) acc[k] = 0.f;
   const float* Tb = T + (size_t)b * m * L + c;
+#pragma unroll 8
   for (int j = 0; j < m; ++j) {
     const float t = __ldg(Tb + (size_t)j * L);
 #pragma unroll
-    for (int k = 0; k < ELL; ++k) acc[k] = fmaf((float)__ldg(R + (size_t)k * m + j), t, acc[k]);
+    for (int k = 0; k < ELL; ++k) {
+      const float r = staged ? s_r[k * m + j] : (float)__ldg(R + (size_t)k * m + j);
+      acc[k] = fmaf(r, t, acc[k]);
+    }
   }
 #pragma unroll
   for (int k = 0; k < ELL; ++k) {

@@ -27,6 +27,8 @@
 // inputs.
 #include <math.h>
 
+#include <algorithm>
+
 #include "gc_internal.cuh"
 
 namespace gc {
@@ -126,25 +128,30 @@ __device__ __forceinline__ int solve_block(const double* __restrict__ R, int m, 
 #pragma unroll
         for (int c = 0; c <= a; ++c) Lc[a][c] = fma(x[a], x[c], Lc[a][c]);
     }
+    // The diagonal is kept as reciprocals (one rsqrt per pivot): GB300's
+    // fp64 divisions and square roots are long instruction sequences.
     bool bad = false;
+    double rdiag[ELL];
 #pragma unroll
     for (int a = 0; a < ELL; ++a) {
       double s = Lc[a][a];
 #pragma unroll
       for (int c = 0; c < a; ++c) s -= Lc[a][c] * Lc[a][c];
       const double ref = Lc[a][a];
-      if (!(s > 1e-26 * ref) || !isfinite(s)) {
+      // pivot^2 / M_aa below 1e-14 (kappa(X) of order 1e7 or more): numerically
+      // rank deficient in fp64; flagged, and clamped so the result stays finite
+      if (!(s > 1e-14 * ref) || !isfinite(s)) {
         bad = true;
-        s = ref > 0.0 ? 1e-26 * ref : 1e-300;
+        s = ref > 0.0 ? 1e-14 * ref : 1e-300;
       }
-      const double piv = sqrt(s);
-      Lc[a][a] = piv;
+      const double rp = rsqrt(s);
+      rdiag[a] = rp;
 #pragma unroll
       for (int r = a + 1; r < ELL; ++r) {
         double t = Lc[r][a];
 #pragma unroll
         for (int c = 0; c < a; ++c) t -= Lc[r][c] * Lc[a][c];
-        Lc[r][a] = t / piv;
+        Lc[r][a] = t * rp;
       }
     }
     if (bad) atomicOr(status, ST_SINGULAR);
@@ -158,14 +165,14 @@ __device__ __forceinline__ int solve_block(const double* __restrict__ R, int m, 
           double t = Bm[a][k];
 #pragma unroll
           for (int c = 0; c < a; ++c) t -= Lc[a][c] * yv[c];
-          yv[a] = t / Lc[a][a];
+          yv[a] = t * rdiag[a];
         }
 #pragma unroll
         for (int a = ELL - 1; a >= 0; --a) {
           double t = yv[a];
 #pragma unroll
           for (int c = a + 1; c < ELL; ++c) t -= Lc[c][a] * Bm[c][k];
-          Bm[a][k] = t / Lc[a][a];
+          Bm[a][k] = t * rdiag[a];
         }
       }
     };
@@ -235,7 +242,7 @@ __device__ __forceinline__ int solve_block(const double* __restrict__ R, int m, 
         ++q;
       }
     }
-    double Xc[MQ][ELL], Q[MQ][ELL], Rr[MQ][MQ], Xp[MQ][ELL];
+    double Xc[MQ][ELL], Q[MQ][ELL], Rr[MQ][MQ], Xp[MQ][ELL], rr[MQ];
 #pragma unroll
     for (int qq = 0; qq < MQ; ++qq) {
 #pragma unroll
@@ -275,14 +282,15 @@ __device__ __forceinline__ int solve_block(const double* __restrict__ R, int m, 
         double nn = 0.0;
 #pragma unroll
         for (int a = 0; a < ELL; ++a) nn = fma(v[a], v[a], nn);
-        if (!(nn > 1e-26 * n0) || !isfinite(nn)) {
+        if (!(nn > 1e-14 * n0) || !isfinite(nn)) {  // same criterion as the Cholesky pivot
           bad = true;
-          nn = n0 > 0.0 ? 1e-26 * n0 : 1e-300;
+          nn = n0 > 0.0 ? 1e-14 * n0 : 1e-300;
         }
-        const double nrm = sqrt(nn);
-        Rr[qq][qq] = nrm;
+        const double rn = rsqrt(nn);
+        Rr[qq][qq] = nn * rn;
+        rr[qq] = rn;
 #pragma unroll
-        for (int a = 0; a < ELL; ++a) Q[qq][a] = v[a] / nrm;
+        for (int a = 0; a < ELL; ++a) Q[qq][a] = v[a] * rn;
       }
     }
     if (bad) atomicOr(status, ST_SINGULAR);
@@ -296,7 +304,7 @@ __device__ __forceinline__ int solve_block(const double* __restrict__ R, int m, 
 #pragma unroll
           for (int r = qq + 1; r < MQ; ++r)
             if (r < D) t -= Rr[qq][r] * Xp[r][k];
-          Xp[qq][k] = t / Rr[qq][qq];
+          Xp[qq][k] = t * rr[qq];
         }
       }
     }
@@ -347,13 +355,13 @@ __device__ __forceinline__ int solve_block(const double* __restrict__ R, int m, 
 struct Table {
   int bits;     // masks per chunk = 1 << bits
   double* xp;   // [N][1<<bits][bits][ell]
-  double* pi;   // [N][1<<bits][ell][ell]
+  float* pi;    // [N][1<<bits][ell][ell] (fp32: the decode matrix is emitted in fp32)
   double* err;  // [N][1<<bits]
 };
 
 template <int ELL>
-__global__ void __launch_bounds__(128) k_table(const double* __restrict__ R, Holders hd, int N,
-                                              int m, Table tb, uint32_t* status) {
+__global__ void __launch_bounds__(32) k_table(const double* __restrict__ R, Holders hd, int N,
+                                              int m, Table tb, int need_xp, uint32_t* status) {
   const long long e = (long long)blockIdx.x * blockDim.x + threadIdx.x;
   const long long nent = (long long)N << tb.bits;
   if (e >= nent) return;
@@ -362,16 +370,27 @@ __global__ void __launch_bounds__(128) k_table(const double* __restrict__ R, Hol
   const int cnt = hd.cnt[i];
   if (cnt > tb.bits) return;  // such chunks are solved directly per pattern
   if (mask >> cnt) return;    // masks beyond this chunk's holders never occur
+  if (!need_xp && __popc(mask) >= ELL) {
+    // full row rank: R_S X^+ = I exactly (Sec. II-A); nothing to solve when the
+    // caller does not want the coefficients themselves
+    float* pi = tb.pi + (size_t)e * ELL * ELL;
+#pragma unroll
+    for (int a = 0; a < ELL; ++a)
+#pragma unroll
+      for (int k = 0; k < ELL; ++k) pi[a * ELL + k] = a == k ? 1.f : 0.f;
+    tb.err[e] = 0.0;
+    return;
+  }
   double Pi[ELL][ELL];
   double err;
   double* xp = tb.xp + (size_t)e * tb.bits * ELL;
   solve_block<ELL>(R, m, cnt, hd.w + (size_t)i * GC_MAX_REPL, mask, Pi, err, status,
                    [&](int h, int k, double v) { xp[h * ELL + k] = v; });
-  double* pi = tb.pi + (size_t)e * ELL * ELL;
+  float* pi = tb.pi + (size_t)e * ELL * ELL;
 #pragma unroll
   for (int a = 0; a < ELL; ++a)
 #pragma unroll
-    for (int k = 0; k < ELL; ++k) pi[a * ELL + k] = Pi[a][k];
+    for (int k = 0; k < ELL; ++k) pi[a * ELL + k] = (float)Pi[a][k];
   tb.err[e] = err;
 }
 
@@ -379,17 +398,21 @@ __global__ void __launch_bounds__(128) k_table(const double* __restrict__ R, Hol
 // Per (pattern, chunk): completion mask, Delta, then table lookup or direct
 // solve; per-pattern error sums reduced in a fixed order.
 // ---------------------------------------------------------------------------
+// 128-thread blocks (64 registers each) so that the solve fits beside the
+// chunk-gradient kernel's register file when both run concurrently.
+constexpr int kPatThreads = 128;
+
 template <int ELL, bool TABLE>
-__global__ void __launch_bounds__(256) k_patterns(const double* __restrict__ R,
+__global__ void __launch_bounds__(kPatThreads) k_patterns(const double* __restrict__ R,
                                                  const int32_t* __restrict__ psi, Holders hd,
                                                  int N, int m, int delta, int npat, int ppb,
                                                  Table tb, SolveOut out, uint32_t* status) {
-  __shared__ double s_err[256];
-  __shared__ int s_def[256];
+  __shared__ double s_err[kPatThreads];
+  __shared__ int s_def[kPatThreads];
   const int tid = threadIdx.x;
   int b, i, istep;
   bool active;
-  if (ppb > 0) {  // N <= 256: ppb patterns per block, one chunk per thread
+  if (ppb > 0) {  // N <= kPatThreads: ppb patterns per block, one chunk per thread
     const int lp = tid / N;
     b = blockIdx.x * ppb + lp;
     i = tid - lp * N;
@@ -398,7 +421,7 @@ __global__ void __launch_bounds__(256) k_patterns(const double* __restrict__ R,
   } else {  // one pattern per block, threads stride over chunks
     b = blockIdx.x;
     i = tid;
-    istep = 256;
+    istep = kPatThreads;
     active = b < npat;
   }
   double my_err = 0.0;
@@ -418,7 +441,7 @@ __global__ void __launch_bounds__(256) k_patterns(const double* __restrict__ R,
         }
         if (hp[h] < v) mask |= 1u << h;
       }
-      double Pi[ELL][ELL];
+      float Pf[ELL][ELL];
       double err;
       int D;
       double* E = out.E;
@@ -427,11 +450,11 @@ __global__ void __launch_bounds__(256) k_patterns(const double* __restrict__ R,
       };
       if (TABLE && cnt <= tb.bits) {
         const size_t e = ((size_t)i << tb.bits) | mask;
-        const double* pi = tb.pi + e * ELL * ELL;
+        const float* pi = tb.pi + e * ELL * ELL;
 #pragma unroll
         for (int a = 0; a < ELL; ++a)
 #pragma unroll
-          for (int k = 0; k < ELL; ++k) Pi[a][k] = pi[a * ELL + k];
+          for (int k = 0; k < ELL; ++k) Pf[a][k] = pi[a * ELL + k];
         err = tb.err[e];
         D = __popc(mask);
         if (E) {
@@ -440,15 +463,28 @@ __global__ void __launch_bounds__(256) k_patterns(const double* __restrict__ R,
 #pragma unroll
             for (int k = 0; k < ELL; ++k) emit(h, k, xp[h * ELL + k]);
         }
+      } else if (!E && __popc(mask) >= ELL) {
+        // full row rank: the decode block is I exactly (Sec. II-A)
+        D = __popc(mask);
+#pragma unroll
+        for (int a = 0; a < ELL; ++a)
+#pragma unroll
+          for (int k = 0; k < ELL; ++k) Pf[a][k] = a == k ? 1.f : 0.f;
+        err = 0.0;
       } else {
+        double Pi[ELL][ELL];
         D = solve_block<ELL>(R, m, cnt, hw, mask, Pi, err, status, emit);
+#pragma unroll
+        for (int a = 0; a < ELL; ++a)
+#pragma unroll
+          for (int k = 0; k < ELL; ++k) Pf[a][k] = (float)Pi[a][k];
       }
       if (out.C) {
         float* Cb = out.C + (size_t)b * ELL * N * ELL + (size_t)i * ELL;
 #pragma unroll
         for (int a = 0; a < ELL; ++a)
 #pragma unroll
-          for (int k = 0; k < ELL; ++k) Cb[(size_t)a * N * ELL + k] = (float)Pi[a][k];
+          for (int k = 0; k < ELL; ++k) Cb[(size_t)a * N * ELL + k] = Pf[a][k];
       }
       if (out.delta_out) out.delta_out[(size_t)b * N + i] = (uint8_t)D;
       if (out.support) {
@@ -465,27 +501,30 @@ __global__ void __launch_bounds__(256) k_patterns(const double* __restrict__ R,
   s_def[tid] = my_def;
   __syncthreads();
   if (!(out.coef_err || out.est)) return;
-  if (ppb > 0) {
-    const int lp = tid / N;
-    if (active && tid - lp * N == 0) {
-      double se = 0.0;
-      int sd = 0;
-      for (int t = 0; t < N; ++t) {
-        se += s_err[tid + t];
-        sd += s_def[tid + t];
-      }
-      if (out.coef_err) out.coef_err[b] = se;
-      if (out.est) out.est[b] = (double)sd;
-    }
-  } else if (tid == 0 && active) {
+  // per pattern: lane l adds entries l, l + 32, ... of the pattern's run of
+  // threads, then a fixed xor tree (deterministic); warp w takes patterns
+  // w, w + 8, ...
+  const int lane = tid & 31, warp = tid >> 5;
+  const int npb = ppb > 0 ? ppb : 1;       // patterns in this block
+  const int run = ppb > 0 ? N : kPatThreads;  // threads holding one pattern's sums
+  for (int q = warp; q < npb; q += kPatThreads / 32) {
+    const int bq = ppb > 0 ? blockIdx.x * ppb + q : blockIdx.x;
+    if (bq >= npat) break;
     double se = 0.0;
     int sd = 0;
-    for (int t = 0; t < 256; ++t) {
-      se += s_err[t];
-      sd += s_def[t];
+    for (int t = lane; t < run; t += 32) {
+      se += s_err[q * run + t];
+      sd += s_def[q * run + t];
     }
-    if (out.coef_err) out.coef_err[b] = se;
-    if (out.est) out.est[b] = (double)sd;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      se += __shfl_xor_sync(0xffffffffu, se, o);
+      sd += __shfl_xor_sync(0xffffffffu, sd, o);
+    }
+    if (lane == 0) {
+      if (out.coef_err) out.coef_err[bq] = se;
+      if (out.est) out.est[bq] = (double)sd;
+    }
   }
 }
 
@@ -506,7 +545,90 @@ size_t solve_table_bytes(int N, int ell, int bits) {
   if (bits < 0) return 0;
   const size_t ent = (size_t)N << bits;
   return align_up(ent * bits * ell * sizeof(double), 256) +
-         align_up(ent * ell * ell * sizeof(double), 256) + align_up(ent * sizeof(double), 256);
+         align_up(ent * ell * ell * sizeof(float), 256) + align_up(ent * sizeof(double), 256);
+}
+
+// Lean variant for N <= 32 without coefficient output: one warp per pattern
+// (lane i = chunk i), grid-stride over patterns, sums by warp shuffles; no
+// shared memory or block barriers, so it runs well beside other kernels.
+template <int ELL, bool TABLE>
+__global__ void __launch_bounds__(128) k_patterns_warp(const double* __restrict__ R,
+                                                       const int32_t* __restrict__ psi,
+                                                       Holders hd, int N, int m, int delta,
+                                                       int npat, Table tb, SolveOut out,
+                                                       uint32_t* status) {
+  const int lane = threadIdx.x & 31;
+  const int gw = (int)((blockIdx.x * blockDim.x + threadIdx.x) >> 5);
+  const int nw = (int)((gridDim.x * blockDim.x) >> 5);
+  const int i = lane;
+  const bool on = i < N;
+  const int cnt = on ? hd.cnt[i] : 0;
+  const int16_t* hw = hd.w + (size_t)(on ? i : 0) * GC_MAX_REPL;
+  const int8_t* hp = hd.p + (size_t)(on ? i : 0) * GC_MAX_REPL;
+  for (int b = gw; b < npat; b += nw) {
+    double err = 0.0;
+    int def = 0;
+    if (on) {
+      const int32_t* ps = psi + (size_t)b * m;
+      uint32_t mask = 0;
+      for (int h = 0; h < cnt; ++h) {
+        int v = __ldg(ps + hw[h]);
+        if (v < 0 || v > delta) {
+          atomicOr(status, ST_BAD_PSI);
+          v = 0;
+        }
+        if (hp[h] < v) mask |= 1u << h;
+      }
+      const int D = __popc(mask);
+      float Pf[ELL][ELL];
+      if (D >= ELL) {  // full row rank: the decode block is I exactly (Sec. II-A)
+#pragma unroll
+        for (int a = 0; a < ELL; ++a)
+#pragma unroll
+          for (int k = 0; k < ELL; ++k) Pf[a][k] = a == k ? 1.f : 0.f;
+      } else if (TABLE && cnt <= tb.bits) {
+        const size_t e = ((size_t)i << tb.bits) | mask;
+        const float* pi = tb.pi + e * ELL * ELL;
+#pragma unroll
+        for (int a = 0; a < ELL; ++a)
+#pragma unroll
+          for (int k = 0; k < ELL; ++k) Pf[a][k] = pi[a * ELL + k];
+        err = tb.err[e];
+      } else {
+        double Pi[ELL][ELL];
+        solve_block<ELL>(R, m, cnt, hw, mask, Pi, err, status, [](int, int, double) {});
+#pragma unroll
+        for (int a = 0; a < ELL; ++a)
+#pragma unroll
+          for (int k = 0; k < ELL; ++k) Pf[a][k] = (float)Pi[a][k];
+      }
+      if (out.C) {
+        float* Cb = out.C + (size_t)b * ELL * N * ELL + (size_t)i * ELL;
+#pragma unroll
+        for (int a = 0; a < ELL; ++a)
+#pragma unroll
+          for (int k = 0; k < ELL; ++k) Cb[(size_t)a * N * ELL + k] = Pf[a][k];
+      }
+      if (out.delta_out) out.delta_out[(size_t)b * N + i] = (uint8_t)D;
+      if (out.support) {
+        uint8_t* row = out.support + ((size_t)b * N + i) * m;
+        for (int j = 0; j < m; ++j) row[j] = 0;
+        for (int h = 0; h < cnt; ++h)
+          if ((mask >> h) & 1u) row[hw[h]] = 1;
+      }
+      def = D < ELL ? ELL - D : 0;
+    }
+    // fixed xor tree over the 32 lanes (deterministic)
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      err += __shfl_xor_sync(0xffffffffu, err, o);
+      def += __shfl_xor_sync(0xffffffffu, def, o);
+    }
+    if (lane == 0) {
+      if (out.coef_err) out.coef_err[b] = err;
+      if (out.est) out.est[b] = (double)def;
+    }
+  }
 }
 
 template <int ELL>
@@ -514,18 +636,33 @@ static void run_solve(const double* R, const int32_t* psi, Holders h, int N, int
                       int npat, SolveOut out, Table tb, bool use_table, uint32_t* status,
                       cudaStream_t s) {
   if (use_table) {
+    // one warp per block: the fp64 pipe is narrow, so spread the solves over SMs
     const long long nent = (long long)N << tb.bits;
-    const int blocks = (int)((nent + 127) / 128);
-    k_table<ELL><<<blocks, 128, 0, s>>>(R, h, N, m, tb, status);
+    const int blocks = (int)((nent + 31) / 32);
+    k_table<ELL><<<blocks, 32, 0, s>>>(R, h, N, m, tb, out.E != nullptr, status);
     count_launches(1);
   }
-  int ppb = N <= 256 ? 256 / N : 0;
+  if (!out.E && N <= 32) {
+    const int warps = 4;  // per 128-thread block
+    const int blocks = std::max(1, std::min((npat + warps - 1) / warps, 8 * device_sm_count()));
+    count_launches(1);
+    if (use_table)
+      k_patterns_warp<ELL, true><<<blocks, 128, 0, s>>>(R, psi, h, N, m, delta, npat, tb, out,
+                                                        status);
+    else
+      k_patterns_warp<ELL, false><<<blocks, 128, 0, s>>>(R, psi, h, N, m, delta, npat, tb, out,
+                                                         status);
+    return;
+  }
+  int ppb = N <= kPatThreads ? kPatThreads / N : 0;
   const int grid = ppb > 0 ? (npat + ppb - 1) / ppb : npat;
   count_launches(1);
   if (use_table)
-    k_patterns<ELL, true><<<grid, 256, 0, s>>>(R, psi, h, N, m, delta, npat, ppb, tb, out, status);
+    k_patterns<ELL, true><<<grid, kPatThreads, 0, s>>>(R, psi, h, N, m, delta, npat, ppb, tb, out,
+                                                      status);
   else
-    k_patterns<ELL, false><<<grid, 256, 0, s>>>(R, psi, h, N, m, delta, npat, ppb, tb, out, status);
+    k_patterns<ELL, false><<<grid, kPatThreads, 0, s>>>(R, psi, h, N, m, delta, npat, ppb, tb, out,
+                                                       status);
 }
 
 // The table region is carved by the caller right after the holders.
@@ -539,8 +676,8 @@ int launch_solve_impl(const double* R, int ell, const int32_t* psi, Holders h, i
     char* p = static_cast<char*>(table_mem);
     tb.xp = reinterpret_cast<double*>(p);
     p += align_up(ent * bits * ell * sizeof(double), 256);
-    tb.pi = reinterpret_cast<double*>(p);
-    p += align_up(ent * ell * ell * sizeof(double), 256);
+    tb.pi = reinterpret_cast<float*>(p);
+    p += align_up(ent * ell * ell * sizeof(float), 256);
     tb.err = reinterpret_cast<double*>(p);
   }
   if (out.E) {

@@ -270,3 +270,24 @@ def test_singular_R_flagged(gc):
     with pytest.raises(gc.GCError) as ei:
         gc.gc_status(ws)
     assert ei.value.code == -7 and "rank" in str(ei.value)
+
+
+def test_encode_with_coeffs_matches_encode(gc):
+    """Algorithm 1 then eq. (2) in two calls gives the same transmissions as
+    gc_encode, and the oracle's."""
+    cfg = get("tiny")
+    N, m, delta, d, ell = cfg.N, cfg.m, cfg.delta, cfg.d, 3
+    order = O.cyclic_order(N, m, delta)
+    R = make_R(cfg, ell)
+    psi = make_patterns(cfg, npat=40)
+    G = np.random.default_rng(12).standard_normal((N, d)).astype(np.float32)
+    Rd, od, pd = dev_tensors(R, order, psi)
+    Gd = torch.from_numpy(G).cuda()
+    E = gc.gc_find_encoding_coeff(Rd, ell, od, N, m, delta, pd, C=False)["E"]
+    T2 = gc.gc_encode_with_coeffs(E, ell, od, N, m, delta, pd, Gd)
+    T1 = gc.gc_encode(Rd, ell, od, N, m, delta, pd, Gd)
+    assert torch.equal(T1, T2)
+    for b in range(psi.shape[0]):
+        r = O.run_pattern(R, order, psi[b], N, G.astype(np.float64))
+        if np.max(np.abs(r.T)) > 0:
+            assert rel_inf(to_np(T2[b]), r.T) <= 1e-4
