@@ -3,7 +3,6 @@
 // returns a GC_* status; the text of the last error is thread-local.
 #include <stdarg.h>
 #include <stdio.h>
-#include <stdlib.h>
 #include <string.h>
 
 #include <algorithm>
@@ -82,18 +81,6 @@ SolveWs carve_solve(Carve& c, int N, int m, int delta, int ell, int npat) {
 
 uint32_t* status_of(void* ws) { return static_cast<uint32_t*>(ws); }
 
-size_t combine_any_ws(int N, int ell, int npat, int d) {
-  return std::max(combine_ws_bytes(N, ell, npat, d), combine_tc_ws_bytes(N, ell, npat, d));
-}
-
-// Decode-combine on the tensor cores; GC_COMBINE_SIMT=1 selects the SIMT
-// kernel for A/B comparisons.
-int run_combine(const float* C, const float* G, const float* gsum, int N, int ell, int npat, int d,
-                float* Ghat, double* grad_mse, Carve& c, uint32_t* status, cudaStream_t s) {
-  static const bool simt = getenv("GC_COMBINE_SIMT") && getenv("GC_COMBINE_SIMT")[0] == '1';
-  if (simt) return launch_combine(C, G, gsum, N, ell, npat, d, Ghat, grad_mse, c, status, s);
-  return launch_combine_tc(C, G, gsum, N, ell, npat, d, Ghat, grad_mse, c, status, s);
-}
 
 }  // namespace
 }  // namespace gc
@@ -286,7 +273,7 @@ size_t gc_decode_batch_workspace(int N, int m, int delta, int ell, int npat, int
   carve_solve(c, N, m, delta, ell, npat);
   c.take<float>((size_t)npat * ell * N * ell);  // C
   c.take<float>((size_t)d);                      // sum of chunk gradients
-  c.take<char>(combine_any_ws(N, ell, npat, d));
+  c.take<char>(combine_tc_ws_bytes(N, ell, npat, d));
   return c.bytes();
 }
 
@@ -318,14 +305,14 @@ int gc_decode_batch(const double* R, int ell, const int32_t* order, int N, int m
     rc = launch_colsum(G, N, d, gsum, s);
     if (rc) return rc;
   }
-  return run_combine(C, G, gsum, N, ell, npat, d, Ghat, grad_mse, c, status_of(ws), s);
+  return launch_combine_tc(C, G, gsum, N, ell, npat, d, Ghat, grad_mse, c, status_of(ws), s);
 }
 
 size_t gc_decode_combine_workspace(int N, int ell, int npat, int d) {
   if (N < 1 || ell < 1 || ell > GC_MAX_ELL || npat < 0 || d < 1) return 0;
   Carve c(nullptr);
   c.take<float>((size_t)d);
-  c.take<char>(combine_any_ws(N, ell, npat, d));
+  c.take<char>(combine_tc_ws_bytes(N, ell, npat, d));
   return c.bytes();
 }
 
@@ -347,7 +334,7 @@ int gc_decode_combine(const float* C, int ell, int N, int npat, const float* G, 
     rc = launch_colsum(G, N, d, gsum, s);
     if (rc) return rc;
   }
-  return run_combine(C, G, gsum, N, ell, npat, d, Ghat, grad_mse, c, status_of(ws), s);
+  return launch_combine_tc(C, G, gsum, N, ell, npat, d, Ghat, grad_mse, c, status_of(ws), s);
 }
 
 size_t gc_mse_workspace(int N, int m, int delta, int ell, int npat, int d) {

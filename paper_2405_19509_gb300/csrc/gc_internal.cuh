@@ -95,14 +95,10 @@ int launch_decode_tx(const double* R, int ell, int m, const float* T, int npat, 
 int launch_sgd(float* w, const float* ghat, int d, float lr, int64_t Ntil, cudaStream_t s);
 int launch_colsum(const float* G, int N, int d, float* gsum, cudaStream_t s);
 
-// ---- batched decode-combine (k_combine.cu SIMT, k_combine_tc.cu tcgen05) --
+// ---- batched decode-combine on the tensor cores (k_combine_tc.cu) --------
 size_t combine_tc_ws_bytes(int N, int ell, int npat, int d);
 int launch_combine_tc(const float* C, const float* G, const float* gsum, int N, int ell, int npat,
                       int d, float* Ghat, double* grad_mse, Carve& ws, uint32_t* status,
                       cudaStream_t s);
-size_t combine_ws_bytes(int N, int ell, int npat, int d);
-int launch_combine(const float* C, const float* G, const float* gsum, int N, int ell, int npat,
-                   int d, float* Ghat, double* grad_mse, Carve& ws, uint32_t* status,
-                   cudaStream_t s);
 
 }  // namespace gc
