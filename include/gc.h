@@ -150,6 +150,33 @@ int gc_find_encoding_coeff(const double* R, int ell, const int32_t* order, int N
                            uint8_t* support, double* coef_err, double* est, void* ws,
                            size_t ws_bytes, void* stream);
 
+/* ---- Algorithm 1 without any allocation -------------------------------
+ * The paper has no counterpart: this is a service for callers that cannot
+ * allocate device memory at all (a runtime that reserves its memory once at
+ * start-up and forbids later cudaMalloc, an embedding without a CUDA
+ * allocator, a thread that must not take the allocator's locks), so cannot
+ * pass the workspace gc_find_encoding_coeff needs.
+ * Same arguments and outputs as gc_find_encoding_coeff, minus (ws, ws_bytes):
+ * the scratch is a file-scope __device__ array of GC_NOALLOC_SCRATCH_BYTES
+ * inside libgc.so, held by every GPU that loads the library until the process
+ * exits.  Nothing is allocated or freed.
+ *  - Sizes whose scratch (holder table, plus the memo table when it fits)
+ *    exceeds GC_NOALLOC_SCRATCH_BYTES are rejected with GC_ERR_WORKSPACE.
+ *  - The first call on each device looks up the array's device address
+ *    (cudaGetSymbolAddress) with that device current; make that first call
+ *    before any stream capture.
+ *  - All calls share the array: two calls whose executions overlap on the
+ *    GPU (other streams, other host threads) race and give wrong results.
+ *  - Device-detected data errors (psi out of range, a singular R_S) are
+ *    handled as in gc_find_encoding_coeff but are not reported; run the
+ *    workspace variant with gc_status to check inputs.
+ */
+#define GC_NOALLOC_SCRATCH_BYTES (8u << 20)
+int gc_find_encoding_coeff_noalloc(const double* R, int ell, const int32_t* order, int N, int m,
+                                   int delta, const int32_t* psi, int npat, double* E, float* C,
+                                   uint8_t* delta_out, uint8_t* support, double* coef_err,
+                                   double* est, void* stream);
+
 /* ---- worker encoding (eq. 2) ------------------------------------------
  * Runs Algorithm 1 for every pattern, then each worker's transmission
  *   T[b][j] = sum_{p < psi[b][j]} sum_k E[b][j][p][k] g_{D_order[j][p]}[k],

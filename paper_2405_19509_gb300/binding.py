@@ -47,6 +47,8 @@ _sig("gc_chunk_grads", _i, _p, _i, _p, _p, _i, _i, _i, _i, _p, _p, _p, _sz, _p)
 _sig("gc_coeff_workspace", _sz, _i, _i, _i, _i, _i)
 _sig("gc_find_encoding_coeff", _i, _p, _i, _p, _i, _i, _i, _p, _i, _p, _p, _p, _p, _p, _p, _p,
      _sz, _p)
+_sig("gc_find_encoding_coeff_noalloc", _i, _p, _i, _p, _i, _i, _i, _p, _i, _p, _p, _p, _p, _p, _p,
+     _p)
 _sig("gc_encode_workspace", _sz, _i, _i, _i, _i, _i, _i)
 _sig("gc_encode", _i, _p, _i, _p, _i, _i, _i, _p, _i, _p, _i, _p, _p, _sz, _p)
 _sig("gc_encode_with_coeffs", _i, _p, _i, _p, _i, _i, _i, _p, _i, _p, _i, _p, _p)
