@@ -14,10 +14,11 @@ One step (every row of the hot path once):
      gradients written) with the fused gradient MSE       (gc_decode_combine)
   4. the live realization: worker encoding (eq. 2), PS
      decode of the transmissions, and the SGD update      (gc_encode, gc_decode_tx, gc_sgd_step)
-Each stage is captured once in a CUDA graph.  Stages that depend only on the
-step's inputs run concurrently on two streams (chunk gradients beside
-Algorithm 1; the batched combine beside the live realization); CUDA events
-around every graph replay time each stage live inside the timed region.
+Each stage is captured once in a CUDA graph.  Stages that do not depend on
+each other run concurrently on two streams (Algorithm 1 beside the chunk
+gradients; the live encode / decode / update beside the batched combine);
+CUDA events around every graph replay time each stage live inside the timed
+region.
 
 Metric: decoded gradients per second (whole job).  `e2e` repeats the timed
 loop through the same C-ABI calls with the step's inputs (the pattern batch
@@ -288,15 +289,14 @@ def gpu_arm(args, rank, world, local_rank):
     stream = torch.cuda.current_stream(dev)
     aux = torch.cuda.Stream(dev)
     gA, gB, gC, gD1, gD2 = graphs
-    ev_in, ev_B, ev_D1 = (torch.cuda.Event() for _ in range(3))
+    ev_in, ev_A, ev_B, ev_D2 = (torch.cuda.Event() for _ in range(4))
 
     def run_step(t, evs=None, host=None):
-        """One step on two streams.  The coefficient solves depend only on the
-        step's inputs, so they run beside the chunk gradients: main = chunk
-        gradients (A), live encode/decode/update (D2, needs A and D1), batched
-        decode-combine (C, needs A and B); aux = Algorithm 1 for the batch (B)
-        and for the live realization (D1).  evs[2s], evs[2s+1] bracket stage s
-        (A, B, C, D1, D2) on its own stream."""
+        """One step on two streams.  main: chunk gradients (A), then the
+        batched decode-combine (C, needs A and B).  aux: Algorithm 1 for the
+        live realization (D1) and for the batch (B) while A runs, then the
+        live encode / decode / update (D2, needs A and D1) beside C.
+        evs[2s], evs[2s+1] bracket stage s (A, B, C, D1, D2) on its stream."""
         def rec(i, st):
             if evs is not None:
                 evs[i].record(st)
@@ -308,26 +308,28 @@ def gpu_arm(args, rank, world, local_rank):
             live_s.copy_(host[1][t], non_blocking=True)
         ev_in.record(stream)
         aux.wait_event(ev_in)
+        rec(0, stream)
+        gA.replay()
+        rec(1, stream)
+        ev_A.record(stream)
         with torch.cuda.stream(aux):
             rec(6, aux)
             gD1.replay()
             rec(7, aux)
-            ev_D1.record(aux)
             rec(2, aux)
             gB.replay()
             rec(3, aux)
             ev_B.record(aux)
-        rec(0, stream)
-        gA.replay()
-        rec(1, stream)
-        stream.wait_event(ev_D1)
-        rec(8, stream)
-        gD2.replay()
-        rec(9, stream)
+            aux.wait_event(ev_A)
+            rec(8, aux)
+            gD2.replay()
+            rec(9, aux)
+            ev_D2.record(aux)
         stream.wait_event(ev_B)
         rec(4, stream)
         gC.replay()
         rec(5, stream)
+        stream.wait_event(ev_D2)
 
     import torch.distributed as tdist
 
@@ -428,7 +430,7 @@ def gpu_arm(args, rank, world, local_rank):
                 "unit": "GB/s", "frac": achieved / hbm, "peak_source": f"{pk_src} hbm_gbs",
                 "traffic": _traffic(names[dom], srcs[dom]),
                 "timing": "CUDA events around the stage's graph (kernel plus its small helpers), "
-                          "averaged over the timed steps; stages B and D1 run concurrently with A",
+                          "averaged over the timed steps; B and D1 run beside A, D2 beside C",
                 "stage_ms": {n: float(v) for n, v in zip(names, stage_ms)},
                 "stage_frac_of_hbm": {n: float(b / (t / 1e3) / 1e9 / hbm) for n, b, t in
                                       zip(names, alg_bytes, stage_ms)}}

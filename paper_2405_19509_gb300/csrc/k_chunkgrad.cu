@@ -440,24 +440,40 @@ __global__ void __launch_bounds__(NT + 32, 1) k_chunkgrad(CGArgs a) {
 }
 
 // G[i][col] = sum of the partials of chunk i, clusters in increasing order.
-__global__ void k_chunkgrad_reduce(const float* __restrict__ parts,
-                                   const double* __restrict__ loss_parts, float* __restrict__ G,
-                                   double* loss_out, int N, int n_c, int d, long long rpc,
-                                   int maxt, int nclusters, long long Ntil) {
-  const long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;
-  if (idx < (long long)N * d) {
-    const int i = (int)(idx / d);
-    const int col = (int)(idx - (long long)i * d);
+// Block (x, i): chunk i, columns [x*1024, (x+1)*1024); the contributing
+// clusters and their slot offsets are computed once per block.
+constexpr int kRedMaxParts = 256;
+__global__ void __launch_bounds__(256) k_chunkgrad_reduce(const float* __restrict__ parts,
+                                                          const double* __restrict__ loss_parts,
+                                                          float* __restrict__ G, double* loss_out,
+                                                          int N, int n_c, int d, long long rpc,
+                                                          int maxt, int nclusters, long long Ntil) {
+  __shared__ long long s_off[kRedMaxParts];
+  __shared__ int s_np;
+  const int i = blockIdx.y;
+  if (threadIdx.x == 0) {
     const long long qlo = ((long long)i * n_c) / rpc;
     const long long qhi = ((long long)(i + 1) * n_c - 1) / rpc;
-    float s = 0.f;
-    for (long long q = qlo; q <= qhi; ++q) {
+    int np = 0;
+    for (long long q = qlo; q <= qhi && np < kRedMaxParts; ++q, ++np) {
       const long long first = (q * rpc) / n_c;
-      s += parts[((size_t)q * maxt + (size_t)(i - first)) * d + col];
+      s_off[np] = ((long long)q * maxt + (i - first)) * (long long)d;
     }
-    G[idx] = s;
+    s_np = np;
   }
-  if (loss_out && blockIdx.x == 0 && threadIdx.x < 32) {
+  __syncthreads();
+  const int np = s_np;
+  const int c0 = blockIdx.x * 1024;
+#pragma unroll
+  for (int k = 0; k < 4; ++k) {
+    const int col = c0 + k * 256 + threadIdx.x;
+    if (col < d) {
+      float acc = 0.f;
+      for (int t = 0; t < np; ++t) acc += __ldg(parts + s_off[t] + col);
+      G[(size_t)i * d + col] = acc;
+    }
+  }
+  if (loss_out && blockIdx.x == 0 && blockIdx.y == 0 && threadIdx.x < 32) {
     // lane l adds clusters l, l + 32, ...; then a fixed xor tree
     double t = 0.0;
     for (int q = threadIdx.x; q < nclusters; q += 32) t += loss_parts[q];
@@ -674,12 +690,12 @@ int launch_chunkgrad(const void* X, int x_dtype, const float* y, const float* w,
   a.status = status;
   int rc = x_dtype == GC_BF16 ? dispatch_cl<__nv_bfloat16>(p, a, s) : dispatch_cl<float>(p, a, s);
   if (rc != GC_OK) return rc;
-  const long long tot = (long long)N * d;
-  const int threads = 256;
-  const long long blocks = std::max<long long>(1, (tot + threads - 1) / threads);
-  k_chunkgrad_reduce<<<(unsigned)blocks, threads, 0, s>>>(a.parts, a.loss_parts, G, loss_out, N,
-                                                          n_c, d, p.rpc, p.maxt, p.nclusters,
-                                                          a.Ntil);
+  if (p.rpc < 1 || (long long)n_c / p.rpc + 2 > kRedMaxParts)
+    return fail(GC_ERR_UNSUPPORTED, "chunk of %d rows spans too many row blocks", n_c);
+  if (N > 65535) return fail(GC_ERR_UNSUPPORTED, "N=%d exceeds 65535 chunks", N);
+  dim3 grid((d + 1023) / 1024, N);
+  k_chunkgrad_reduce<<<grid, 256, 0, s>>>(a.parts, a.loss_parts, G, loss_out, N, n_c, d, p.rpc,
+                                          p.maxt, p.nclusters, a.Ntil);
   count_launches(1);
   return cuda_check(cudaGetLastError(), "k_chunkgrad_reduce");
 }
