@@ -8,10 +8,10 @@ communication factor l = 2.
 
 One step (every row of the hot path once):
   1. chunk gradients g_{D_i} at the current w            (gc_chunk_grads)
-  2. Algorithm 1 for all 10^4 patterns -> decode matrix C,
-     coefficient error and estimate                       (gc_find_encoding_coeff)
+  2. Algorithm 1 for all 10^4 patterns -> decode plan,
+     coefficient error and estimate                       (gc_decode_plan)
   3. batched decode-combine Ghat = C . G (10^4 decoded
-     gradients written) with the fused gradient MSE       (gc_decode_combine)
+     gradients written) with the fused gradient MSE       (gc_decode_apply)
   4. the live realization: worker encoding (eq. 2), PS
      decode of the transmissions, and the SGD update      (gc_encode, gc_decode_tx, gc_sgd_step)
 Each stage is captured once in a CUDA graph.  Stages that do not depend on
@@ -236,7 +236,7 @@ def gpu_arm(args, rank, world, local_rank):
     live_s = torch.empty(1, m, dtype=torch.int32, device=dev)
     G_s = torch.empty(N, d, dtype=torch.float32, device=dev)
     loss_s = torch.zeros(1, dtype=torch.float64, device=dev)
-    C_s = torch.empty(npat, ell, N * ell, dtype=torch.float32, device=dev)
+    plan_s = torch.empty(int(gc.lib.gc_decode_plan_bytes(N, ell, npat)), dtype=torch.uint8, device=dev)
     ce_s = torch.empty(npat, dtype=torch.float64, device=dev)
     est_s = torch.empty(npat, dtype=torch.float64, device=dev)
     Gh_s = torch.empty(npat, d, dtype=torch.float32, device=dev)
@@ -249,12 +249,12 @@ def gpu_arm(args, rank, world, local_rank):
     def stage_a():
         gc.gc_chunk_grads(X, y, w, N, n_c, gc.GC_LOGISTIC, G=G_s, loss_out=loss_s, ws=wsA)
 
-    def stage_b():
-        gc.gc_find_encoding_coeff(Rd, ell, od, N, m, delta, psi_s, E=False, C=C_s, delta_out=False,
-                                  support=False, coef_err=ce_s, est=est_s, ws=wsB)
+    def stage_b():  # Algorithm 1 for the batch -> decode plan (psi side, no G needed)
+        gc.gc_decode_plan(Rd, ell, od, N, m, delta, psi_s, plan=plan_s, coef_err=ce_s, est=est_s,
+                          ws=wsB)
 
-    def stage_c():
-        gc.gc_decode_combine(C_s, ell, N, G_s, Ghat=Gh_s, grad_mse=mse_s, ws=wsC)
+    def stage_c():  # batched decode-combine from the plan and G
+        gc.gc_decode_apply(plan_s, ell, N, npat, G_s, Ghat=Gh_s, grad_mse=mse_s, ws=wsC)
 
     def stage_d1():  # Algorithm 1 for the live realization (independent of G)
         gc.gc_find_encoding_coeff(Rd, ell, od, N, m, delta, live_s, E=E_s, C=False, delta_out=False,
@@ -415,8 +415,8 @@ def gpu_arm(args, rank, world, local_rank):
              "encode+decode_tx+sgd"]
     alg_bytes = [
         cfg.Ntil * d * 4 + cfg.Ntil * 4 + N * d * 4,                          # X, y read; G written
-        npat * m * 4 + npat * ell * N * ell * 4 + 2 * npat * 8,               # psi read; C, errors written
-        npat * d * 4 + npat * ell * N * ell * 4 + N * d * 4 + npat * 8,       # Ghat written; C, G read
+        npat * m * 4 + npat * ell * N * ell * 4 + 2 * npat * 8,               # psi read; C (hi+lo), errors written
+        npat * d * 4 + npat * ell * N * ell * 4 + N * d * 4 + npat * 8,       # Ghat written; C (hi+lo), G read
         m * 4 + m * delta * ell * 8,                                          # psi read; E written
         N * d * 4 + m * L * 4 * 2 + d * 4 * 3,                                # G read; T; ghat; w
     ]

@@ -223,6 +223,26 @@ int gc_decode_batch(const double* R, int ell, const int32_t* order, int N, int m
                     double* coef_err, double* est, double* grad_mse, void* ws, size_t ws_bytes,
                     void* stream);
 
+/* ---- decoding in two halves: coefficients, then data --------------------
+ * The decode coefficients depend only on psi and R, not on the gradients,
+ * so a PS can solve them while the chunk gradients are still being computed.
+ * gc_decode_plan runs Algorithm 1 for every pattern (as gc_find_encoding_coeff)
+ * and writes the decode matrix R B into `plan`, an opaque caller-owned device
+ * buffer of gc_decode_plan_bytes(N, ell, npat) bytes (256-byte aligned) laid
+ * out for the tensor-core combine; coef_err and est as in
+ * gc_find_encoding_coeff (each may be NULL).  gc_decode_apply then computes
+ * Ghat and/or grad_mse from the plan and G exactly as gc_decode_batch does;
+ * it must be given the same (N, ell, npat) as the plan.
+ */
+size_t gc_decode_plan_bytes(int N, int ell, int npat);
+size_t gc_decode_plan_workspace(int N, int m, int delta, int ell, int npat);
+int gc_decode_plan(const double* R, int ell, const int32_t* order, int N, int m, int delta,
+                   const int32_t* psi, int npat, void* plan, size_t plan_bytes, double* coef_err,
+                   double* est, void* ws, size_t ws_bytes, void* stream);
+size_t gc_decode_apply_workspace(int N, int ell, int npat, int d);
+int gc_decode_apply(const void* plan, int ell, int N, int npat, const float* G, int d,
+                    float* Ghat, double* grad_mse, void* ws, size_t ws_bytes, void* stream);
+
 /* ---- decode-combine alone ----------------------------------------------
  * The GEMM step of gc_decode_batch for a decode matrix the caller already
  * has (e.g. from gc_find_encoding_coeff):

@@ -21,7 +21,9 @@ from .binding import (  # noqa: F401
     gc_coeff_workspace,
     gc_decode_batch,
     gc_decode_batch_workspace,
+    gc_decode_apply,
     gc_decode_combine,
+    gc_decode_plan,
     gc_decode_combine_workspace,
     gc_kernel_launches,
     gc_decode_tx,

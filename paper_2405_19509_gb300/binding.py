@@ -55,6 +55,11 @@ _sig("gc_encode_with_coeffs", _i, _p, _i, _p, _i, _i, _i, _p, _i, _p, _i, _p, _p
 _sig("gc_decode_tx", _i, _p, _i, _i, _p, _i, _i, _p, _p)
 _sig("gc_decode_batch_workspace", _sz, _i, _i, _i, _i, _i, _i)
 _sig("gc_decode_batch", _i, _p, _i, _p, _i, _i, _i, _p, _i, _p, _i, _p, _p, _p, _p, _p, _sz, _p)
+_sig("gc_decode_plan_bytes", _sz, _i, _i, _i)
+_sig("gc_decode_plan_workspace", _sz, _i, _i, _i, _i, _i)
+_sig("gc_decode_plan", _i, _p, _i, _p, _i, _i, _i, _p, _i, _p, _sz, _p, _p, _p, _sz, _p)
+_sig("gc_decode_apply_workspace", _sz, _i, _i, _i, _i)
+_sig("gc_decode_apply", _i, _p, _i, _i, _i, _p, _i, _p, _p, _p, _sz, _p)
 _sig("gc_decode_combine_workspace", _sz, _i, _i, _i, _i)
 _sig("gc_decode_combine", _i, _p, _i, _i, _i, _p, _i, _p, _p, _p, _sz, _p)
 _sig("gc_mse_workspace", _sz, _i, _i, _i, _i, _i, _i)
@@ -292,6 +297,45 @@ def gc_decode_batch(R, ell, order, N, m, delta, psi, G, Ghat=True, coef_err=True
         _dev(res["coef_err"], torch.float64, "coef_err"), _dev(res["est"], torch.float64, "est"),
         _dev(res["grad_mse"], torch.float64, "grad_mse"), wp, wn, _stream()))
     return res
+
+
+def gc_decode_plan(R, ell, order, N, m, delta, psi, plan=None, coef_err=True, est=True,
+                   ws: Workspace | None = None):
+    """Algorithm 1 for every pattern into an opaque plan (uint8 device tensor)
+    for gc_decode_apply.  Returns dict with plan, coef_err, est."""
+    npat = psi.shape[0]
+    dev = psi.device
+    nb = lib.gc_decode_plan_bytes(N, ell, npat)
+    if plan is None:
+        plan = torch.empty(max(int(nb), 256), dtype=torch.uint8, device=dev)
+    ce = coef_err if isinstance(coef_err, torch.Tensor) else (
+        torch.empty(npat, dtype=torch.float64, device=dev) if coef_err else None)
+    es = est if isinstance(est, torch.Tensor) else (
+        torch.empty(npat, dtype=torch.float64, device=dev) if est else None)
+    ws, (wp, wn) = _ws(ws, lib.gc_decode_plan_workspace(N, m, delta, ell, npat), dev)
+    _check(lib.gc_decode_plan(_dev(R, torch.float64, "R", (ell, m)), ell,
+                              _dev(order, torch.int32, "order", (m, delta)), N, m, delta,
+                              _dev(psi, torch.int32, "psi", (npat, m)), npat,
+                              _dev(plan, torch.uint8, "plan"), plan.numel(),
+                              _dev(ce, torch.float64, "coef_err"), _dev(es, torch.float64, "est"),
+                              wp, wn, _stream()))
+    return {"plan": plan, "coef_err": ce, "est": es}
+
+
+def gc_decode_apply(plan, ell, N, npat, G, Ghat=True, grad_mse=True, ws: Workspace | None = None):
+    """Ghat (npat x d) and/or grad_mse (npat) from a gc_decode_plan plan and G."""
+    d = G.shape[1]
+    dev = G.device
+    if not isinstance(Ghat, torch.Tensor):
+        Ghat = torch.empty(npat, d, dtype=torch.float32, device=dev) if Ghat else None
+    if not isinstance(grad_mse, torch.Tensor):
+        grad_mse = torch.empty(npat, dtype=torch.float64, device=dev) if grad_mse else None
+    ws, (wp, wn) = _ws(ws, lib.gc_decode_apply_workspace(N, ell, npat, d), dev)
+    _check(lib.gc_decode_apply(_dev(plan, torch.uint8, "plan"), ell, N, npat,
+                               _dev(G, torch.float32, "G", (N, d)), d,
+                               _dev(Ghat, torch.float32, "Ghat", (npat, d)),
+                               _dev(grad_mse, torch.float64, "grad_mse"), wp, wn, _stream()))
+    return {"Ghat": Ghat, "grad_mse": grad_mse}
 
 
 def gc_kernel_launches() -> int:

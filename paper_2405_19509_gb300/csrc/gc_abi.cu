@@ -266,14 +266,76 @@ int gc_decode_tx(const double* R, int ell, int m, const float* T, int npat, int 
   return launch_decode_tx(R, ell, m, T, npat, d, ghat, as_stream(stream));
 }
 
-// ---------------------------------------------------------------- decode batch / mse
+// ---------------------------------------------------------------- decode plan / apply / batch
+size_t gc_decode_plan_bytes(int N, int ell, int npat) {
+  if (N < 1 || ell < 1 || ell > GC_MAX_ELL || npat < 0) return 0;
+  return plan_bytes(N, ell, npat);
+}
+
+size_t gc_decode_plan_workspace(int N, int m, int delta, int ell, int npat) {
+  return gc_coeff_workspace(N, m, delta, ell, npat);
+}
+
+int gc_decode_plan(const double* R, int ell, const int32_t* order, int N, int m, int delta,
+                   const int32_t* psi, int npat, void* plan, size_t plan_bytes_, double* coef_err,
+                   double* est, void* ws, size_t ws_bytes, void* stream) {
+  int rc = check_dims(N, m, delta, ell, npat);
+  if (rc) return rc;
+  if (!R || !order || (!psi && npat > 0)) return fail(GC_ERR_ARG, "R, order and psi must be non-NULL");
+  if (npat == 0) return GC_OK;
+  if (!plan) return fail(GC_ERR_ARG, "plan is NULL");
+  if (plan_bytes_ < plan_bytes(N, ell, npat))
+    return fail(GC_ERR_WORKSPACE, "plan buffer too small: %zu < %zu bytes", plan_bytes_,
+                plan_bytes(N, ell, npat));
+  if (reinterpret_cast<uintptr_t>(plan) % 256 != 0)
+    return fail(GC_ERR_WORKSPACE, "plan buffer must be 256-byte aligned");
+  rc = check_ws(ws, ws_bytes, gc_decode_plan_workspace(N, m, delta, ell, npat));
+  if (rc) return rc;
+  cudaStream_t s = as_stream(stream);
+  Carve c(ws);
+  SolveWs sw = carve_solve(c, N, m, delta, ell, npat);
+  launch_holders(order, N, m, delta, sw.h, status_of(ws), s);
+  SolveOut out{nullptr, nullptr, nullptr, nullptr, coef_err, est,
+               static_cast<__nv_bfloat16*>(plan), combine_kp(N, ell)};
+  return launch_solve_impl(R, ell, psi, sw.h, N, m, delta, npat, out, sw.table, sw.bits,
+                           status_of(ws), s);
+}
+
+size_t gc_decode_apply_workspace(int N, int ell, int npat, int d) {
+  if (N < 1 || ell < 1 || ell > GC_MAX_ELL || npat < 0 || d < 1) return 0;
+  return kHeaderBytes + apply_ws_bytes(N, ell, npat, d);
+}
+
+static int check_apply(int N, int ell, int npat, int d, const void* G, const float* Ghat,
+                       const double* grad_mse) {
+  if (N < 1 || npat < 0 || d < 1) return fail(GC_ERR_SHAPE, "N, d >= 1 and npat >= 0 required");
+  if (ell < 1) return fail(GC_ERR_SHAPE, "ell=%d must be >= 1", ell);
+  if (ell > GC_MAX_ELL) return fail(GC_ERR_UNSUPPORTED, "ell=%d exceeds %d", ell, GC_MAX_ELL);
+  if ((long long)N * ell > (1LL << 30)) return fail(GC_ERR_UNSUPPORTED, "N*ell too large");
+  if (!G) return fail(GC_ERR_ARG, "G must be non-NULL");
+  if (npat > 0 && !Ghat && !grad_mse) return fail(GC_ERR_ARG, "Ghat and grad_mse are both NULL");
+  return GC_OK;
+}
+
+int gc_decode_apply(const void* plan, int ell, int N, int npat, const float* G, int d, float* Ghat,
+                    double* grad_mse, void* ws, size_t ws_bytes, void* stream) {
+  int rc = check_apply(N, ell, npat, d, G, Ghat, grad_mse);
+  if (rc) return rc;
+  if (npat == 0) return GC_OK;
+  if (!plan) return fail(GC_ERR_ARG, "plan is NULL");
+  rc = check_ws(ws, ws_bytes, gc_decode_apply_workspace(N, ell, npat, d));
+  if (rc) return rc;
+  Carve c(ws);
+  return launch_apply(static_cast<const __nv_bfloat16*>(plan), G, N, ell, npat, d, Ghat, grad_mse,
+                      c, status_of(ws), as_stream(stream));
+}
+
 size_t gc_decode_batch_workspace(int N, int m, int delta, int ell, int npat, int d) {
   if (check_dims(N, m, delta, ell, npat) || d < 1) return 0;
   Carve c(nullptr);
   carve_solve(c, N, m, delta, ell, npat);
-  c.take<float>((size_t)npat * ell * N * ell);  // C
-  c.take<float>((size_t)d);                      // sum of chunk gradients
-  c.take<char>(combine_tc_ws_bytes(N, ell, npat, d));
+  c.take<char>(plan_bytes(N, ell, npat));
+  c.take<char>(apply_ws_bytes(N, ell, npat, d));
   return c.bytes();
 }
 
@@ -290,51 +352,40 @@ int gc_decode_batch(const double* R, int ell, const int32_t* order, int N, int m
   if (!Ghat && !grad_mse) return fail(GC_ERR_ARG, "Ghat and grad_mse are both NULL");
   rc = check_ws(ws, ws_bytes, gc_decode_batch_workspace(N, m, delta, ell, npat, d));
   if (rc) return rc;
-  if (npat == 0) return GC_OK;
   cudaStream_t s = as_stream(stream);
   Carve c(ws);
   SolveWs sw = carve_solve(c, N, m, delta, ell, npat);
-  float* C = c.take<float>((size_t)npat * ell * N * ell);
-  float* gsum = c.take<float>((size_t)d);
+  __nv_bfloat16* Cs = c.take<__nv_bfloat16>(plan_bytes(N, ell, npat) / sizeof(__nv_bfloat16));
   launch_holders(order, N, m, delta, sw.h, status_of(ws), s);
-  SolveOut out{nullptr, C, nullptr, nullptr, coef_err, est};
+  SolveOut out{nullptr, nullptr, nullptr, nullptr, coef_err, est, Cs, combine_kp(N, ell)};
   rc = launch_solve_impl(R, ell, psi, sw.h, N, m, delta, npat, out, sw.table, sw.bits,
                          status_of(ws), s);
   if (rc) return rc;
-  if (grad_mse) {
-    rc = launch_colsum(G, N, d, gsum, s);
-    if (rc) return rc;
-  }
-  return launch_combine_tc(C, G, gsum, N, ell, npat, d, Ghat, grad_mse, c, status_of(ws), s);
+  return launch_apply(Cs, G, N, ell, npat, d, Ghat, grad_mse, c, status_of(ws), s);
 }
 
 size_t gc_decode_combine_workspace(int N, int ell, int npat, int d) {
   if (N < 1 || ell < 1 || ell > GC_MAX_ELL || npat < 0 || d < 1) return 0;
   Carve c(nullptr);
-  c.take<float>((size_t)d);
-  c.take<char>(combine_tc_ws_bytes(N, ell, npat, d));
+  c.take<char>(plan_bytes(N, ell, npat));
+  c.take<char>(apply_ws_bytes(N, ell, npat, d));
   return c.bytes();
 }
 
 int gc_decode_combine(const float* C, int ell, int N, int npat, const float* G, int d,
                       float* Ghat, double* grad_mse, void* ws, size_t ws_bytes, void* stream) {
-  if (N < 1 || npat < 0 || d < 1) return fail(GC_ERR_SHAPE, "N, d >= 1 and npat >= 0 required");
-  if (ell < 1) return fail(GC_ERR_SHAPE, "ell=%d must be >= 1", ell);
-  if (ell > GC_MAX_ELL) return fail(GC_ERR_UNSUPPORTED, "ell=%d exceeds %d", ell, GC_MAX_ELL);
-  if ((long long)N * ell > (1LL << 30)) return fail(GC_ERR_UNSUPPORTED, "N*ell too large");
-  if (!C || !G) return fail(GC_ERR_ARG, "C and G must be non-NULL");
+  int rc = check_apply(N, ell, npat, d, G, Ghat, grad_mse);
+  if (rc) return rc;
+  if (!C) return fail(GC_ERR_ARG, "C must be non-NULL");
   if (npat == 0) return GC_OK;
-  if (!Ghat && !grad_mse) return fail(GC_ERR_ARG, "Ghat and grad_mse are both NULL");
-  int rc = check_ws(ws, ws_bytes, gc_decode_combine_workspace(N, ell, npat, d));
+  rc = check_ws(ws, ws_bytes, gc_decode_combine_workspace(N, ell, npat, d));
   if (rc) return rc;
   cudaStream_t s = as_stream(stream);
   Carve c(ws);
-  float* gsum = c.take<float>((size_t)d);
-  if (grad_mse) {
-    rc = launch_colsum(G, N, d, gsum, s);
-    if (rc) return rc;
-  }
-  return launch_combine_tc(C, G, gsum, N, ell, npat, d, Ghat, grad_mse, c, status_of(ws), s);
+  __nv_bfloat16* Cs = c.take<__nv_bfloat16>(plan_bytes(N, ell, npat) / sizeof(__nv_bfloat16));
+  rc = launch_split_c(C, N, ell, npat, Cs, s);
+  if (rc) return rc;
+  return launch_apply(Cs, G, N, ell, npat, d, Ghat, grad_mse, c, status_of(ws), s);
 }
 
 size_t gc_mse_workspace(int N, int m, int delta, int ell, int npat, int d) {

@@ -73,6 +73,8 @@ struct SolveOut {
   uint8_t* support;   // npat x N x m (nullable)
   double* coef_err;   // npat (nullable)
   double* est;        // npat (nullable)
+  __nv_bfloat16* Cs;  // decode matrix as bf16 hi/lo planes [2][npat*ell][Kp] (nullable)
+  int Kp;             // row stride of Cs: N*ell rounded up to whole 64-element blocks
 };
 // Memo table of every holder subset (bits = masks per chunk in log2, -1 = none).
 int solve_table_bits(int N, int m, int delta, int npat);
@@ -93,12 +95,19 @@ int launch_encode(const double* E, const int32_t* order, const int32_t* psi, int
 int launch_decode_tx(const double* R, int ell, int m, const float* T, int npat, int d, float* ghat,
                      cudaStream_t s);
 int launch_sgd(float* w, const float* ghat, int d, float lr, int64_t Ntil, cudaStream_t s);
-int launch_colsum(const float* G, int N, int d, float* gsum, cudaStream_t s);
 
 // ---- batched decode-combine on the tensor cores (k_combine_tc.cu) --------
-size_t combine_tc_ws_bytes(int N, int ell, int npat, int d);
-int launch_combine_tc(const float* C, const float* G, const float* gsum, int N, int ell, int npat,
-                      int d, float* Ghat, double* grad_mse, Carve& ws, uint32_t* status,
-                      cudaStream_t s);
+// K = N*ell padded to whole 64-element blocks (the GEMM's K extent).
+inline int combine_kp(int N, int ell) { return (N * ell + 63) / 64 * 64; }
+// bytes of the bf16 hi/lo planes of the decode matrix ("decode plan")
+inline size_t plan_bytes(int N, int ell, int npat) {
+  return align_up((size_t)2 * npat * ell * combine_kp(N, ell) * 2, 256);
+}
+// scratch of the GEMM side given the planes (G planes, sum of G, MSE partials)
+size_t apply_ws_bytes(int N, int ell, int npat, int d);
+int launch_apply(const __nv_bfloat16* Cs, const float* G, int N, int ell, int npat, int d,
+                 float* Ghat, double* grad_mse, Carve& ws, uint32_t* status, cudaStream_t s);
+// fp32 C (npat x ell x N*ell) -> planes
+int launch_split_c(const float* C, int N, int ell, int npat, __nv_bfloat16* Cs, cudaStream_t s);
 
 }  // namespace gc

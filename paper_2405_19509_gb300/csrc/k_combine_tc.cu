@@ -428,14 +428,25 @@ __global__ void k_split_c(const float* __restrict__ C, int M, int K, int Kp,
 }
 
 // G (N x d fp32) -> planes [2][L][Kp] bf16 of Gv^T: element (c, i*ell + k') =
-// g_{D_i}[k'*L + c] (zero past d and for padding columns).  32 x 32 tiles
-// transposed through shared memory.
+// g_{D_i}[k'*L + c] (zero past d and for padding columns), 32 x 32 tiles
+// transposed through shared memory; blocks with blockIdx.y == 0 also write
+// gsum[k'*L + c] = sum_i g_{D_i}[k'*L + c] (chunks in order) when gsum != 0.
 __global__ void k_split_gt(const float* __restrict__ G, int N, int d, int ell, int L, int Kp,
-                           __nv_bfloat16* __restrict__ out) {
+                           __nv_bfloat16* __restrict__ out, float* __restrict__ gsum) {
   __shared__ float tile[32][33];
   const int c0 = blockIdx.x * 32, k0 = blockIdx.y * 32;
   const int tx = threadIdx.x, ty = threadIdx.y;  // 32 x 8
   const int K = N * ell;
+  if (gsum && blockIdx.y == 0) {
+    for (int kp = ty; kp < ell; kp += 8) {
+      const int col = kp * L + c0 + tx;
+      if (c0 + tx < L && col < d) {
+        float acc = 0.f;
+        for (int i = 0; i < N; ++i) acc += __ldg(G + (size_t)i * d + col);
+        gsum[col] = acc;
+      }
+    }
+  }
   for (int r = ty; r < 32; r += 8) {
     const int kk = k0 + r, c = c0 + tx;
     float v = 0.f;
@@ -534,40 +545,43 @@ int launch_tc(int grid, const CUtensorMap& mA, const CUtensorMap& mB, const CUte
   return cuda_check(cudaGetLastError(), "k_combine_tc");
 }
 
-size_t combine_tc_ws_bytes(int N, int ell, int npat, int d) {
+size_t apply_ws_bytes(int N, int ell, int npat, int d) {
   const int L = (d + ell - 1) / ell;
   const long long M = (long long)npat * ell;
-  const int K = N * ell;
-  const int Kp = (K + tc::BK - 1) / tc::BK * tc::BK;
+  const int Kp = combine_kp(N, ell);
   const int nnt = (L + tc::BN - 1) / tc::BN;
-  return align_up((size_t)2 * M * Kp * 2, 256) + align_up((size_t)2 * L * Kp * 2, 256) +
+  return align_up((size_t)2 * L * Kp * 2, 256) + align_up((size_t)d * sizeof(float), 256) +
          align_up((size_t)M * nnt * 2 * sizeof(float), 256);
 }
 
-int launch_combine_tc(const float* C, const float* G, const float* gsum, int N, int ell, int npat,
-                      int d, float* Ghat, double* grad_mse, Carve& ws, uint32_t* status,
-                      cudaStream_t s) {
+int launch_split_c(const float* C, int N, int ell, int npat, __nv_bfloat16* Cs, cudaStream_t s) {
+  const long long M = (long long)npat * ell;
+  const int K = N * ell, Kp = combine_kp(N, ell);
+  const long long tot = M * Kp;
+  if (tot == 0) return GC_OK;
+  tc::k_split_c<<<(unsigned)((tot + 255) / 256), 256, 0, s>>>(C, (int)M, K, Kp, Cs);
+  count_launches(1);
+  return cuda_check(cudaGetLastError(), "k_split_c");
+}
+
+int launch_apply(const __nv_bfloat16* Cs, const float* G, int N, int ell, int npat, int d,
+                 float* Ghat, double* grad_mse, Carve& ws, uint32_t* status, cudaStream_t s) {
   using namespace tc;
   const int L = (d + ell - 1) / ell;
   const long long M = (long long)npat * ell;
   const int K = N * ell;
-  // K padded to whole 64-element blocks: every TMA row is one aligned 128-byte line
-  const int Kp = (K + BK - 1) / BK * BK;
+  const int Kp = combine_kp(N, ell);  // every TMA row is one aligned 128-byte line
   if (M > (1LL << 31) - 1) return fail(GC_ERR_UNSUPPORTED, "npat*ell too large");
   const int nmt = (int)((M + BM - 1) / BM), nnt = (L + BN - 1) / BN;
-  __nv_bfloat16* Cs = ws.take<__nv_bfloat16>((size_t)2 * M * Kp);
   __nv_bfloat16* Gs = ws.take<__nv_bfloat16>((size_t)2 * L * Kp);
+  float* gsum = ws.take<float>((size_t)d);
   float* msep = grad_mse ? ws.take<float>((size_t)M * nnt * 2) : nullptr;
-
   {
-    const long long tot = M * Kp;
-    k_split_c<<<(unsigned)((tot + 255) / 256), 256, 0, s>>>(C, (int)M, K, Kp, Cs);
-    count_launches(1);
     dim3 grid((L + 31) / 32, (Kp + 31) / 32);
-    k_split_gt<<<grid, dim3(32, 8), 0, s>>>(G, N, d, ell, L, Kp, Gs);
+    k_split_gt<<<grid, dim3(32, 8), 0, s>>>(G, N, d, ell, L, Kp, Gs, grad_mse ? gsum : nullptr);
     count_launches(1);
     cudaError_t e = cudaGetLastError();
-    if (e != cudaSuccess) return cuda_check(e, "split kernels");
+    if (e != cudaSuccess) return cuda_check(e, "k_split_gt");
   }
   CUtensorMap mA, mB, mC;
   int rc = make_map(&mA, Cs, (int)M, Kp, BM);
@@ -602,14 +616,13 @@ int launch_combine_tc(const float* C, const float* G, const float* gsum, int N, 
   p.parts_per_row = nnt * (one_block ? 2 : 1);
   const int sms = device_sm_count();
   const int grid = (int)std::min<long long>(p.num_tiles, sms);
-  int rc2 = one_block ? launch_tc<1, 8>(grid, mA, mB, mC, p, s) : launch_tc<2, 4>(grid, mA, mB, mC, p, s);
-  if (rc2) return rc2;
-  cudaError_t e;
+  rc = one_block ? launch_tc<1, 8>(grid, mA, mB, mC, p, s) : launch_tc<2, 4>(grid, mA, mB, mC, p, s);
+  if (rc) return rc;
   if (grad_mse) {
     k_mse_reduce_tiles<<<(npat + 255) / 256, 256, 0, s>>>(msep, npat, ell, p.parts_per_row, d,
                                                          grad_mse);
     count_launches(1);
-    e = cudaGetLastError();
+    cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return cuda_check(e, "k_mse_reduce_tiles");
   }
   return GC_OK;

@@ -1,7 +1,7 @@
-// Worker encoding (eq. 2), PS decoding of transmissions (Sec. II-B), the
-// parameter update (Sec. I) and the sum of chunk gradients.
+// Worker encoding (eq. 2), PS decoding of transmissions (Sec. II-B) and the
+// parameter update (Sec. I).
 //
-// All four are HBM-bound streaming kernels with coalesced accesses along the
+// All three are HBM-bound streaming kernels with coalesced accesses along the
 // block coordinate c (consecutive threads, consecutive columns).
 #include "gc_internal.cuh"
 
@@ -120,21 +120,6 @@ int launch_sgd(float* w, const float* ghat, int d, float lr, int64_t Ntil, cudaS
   k_sgd<<<(d + 255) / 256, 256, 0, s>>>(w, ghat, d, scale);
   count_launches(1);
   return cuda_check(cudaGetLastError(), "k_sgd");
-}
-
-// gsum[c] = sum_i G[i][c], chunks in increasing order.
-__global__ void k_colsum(const float* __restrict__ G, int N, int d, float* __restrict__ gsum) {
-  const int c = blockIdx.x * blockDim.x + threadIdx.x;
-  if (c >= d) return;
-  float s = 0.f;
-  for (int i = 0; i < N; ++i) s += __ldg(G + (size_t)i * d + c);
-  gsum[c] = s;
-}
-
-int launch_colsum(const float* G, int N, int d, float* gsum, cudaStream_t s) {
-  k_colsum<<<(d + 255) / 256, 256, 0, s>>>(G, N, d, gsum);
-  count_launches(1);
-  return cuda_check(cudaGetLastError(), "k_colsum");
 }
 
 }  // namespace gc

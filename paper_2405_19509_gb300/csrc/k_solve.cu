@@ -398,6 +398,40 @@ __global__ void __launch_bounds__(32) k_table(const double* __restrict__ R, Hold
 // Per (pattern, chunk): completion mask, Delta, then table lookup or direct
 // solve; per-pattern error sums reduced in a fixed order.
 // ---------------------------------------------------------------------------
+// Decode matrix block (pattern b, chunk i) as bf16 hi/lo planes, the layout
+// the tensor-core combine reads: plane h, row b*ell + a, column i*ell + k.
+template <int ELL>
+__device__ __forceinline__ void write_planes(__nv_bfloat16* Cs, int Kp, int npat, int b, int i,
+                                             const float (&Pf)[ELL][ELL]) {
+  const size_t plane = (size_t)npat * ELL * Kp;
+#pragma unroll
+  for (int a = 0; a < ELL; ++a)
+#pragma unroll
+    for (int k = 0; k < ELL; ++k) {
+      const float v = Pf[a][k];
+      const __nv_bfloat16 hi = __float2bfloat16_rn(v);
+      const __nv_bfloat16 lo = __float2bfloat16_rn(v - __bfloat162float(hi));
+      const size_t idx = ((size_t)b * ELL + a) * Kp + (size_t)i * ELL + k;
+      Cs[idx] = hi;
+      Cs[plane + idx] = lo;
+    }
+}
+// Zero the padding columns [N*ell, Kp) of pattern b's rows (both planes);
+// thread t of the `run` threads owning the pattern takes entries t, t+run, ...
+template <int ELL>
+__device__ __forceinline__ void zero_pad(__nv_bfloat16* Cs, int Kp, int N, int npat, int b, int t,
+                                         int run) {
+  const int K = N * ELL, pad = Kp - K;
+  if (pad <= 0) return;
+  const size_t plane = (size_t)npat * ELL * Kp;
+  const __nv_bfloat16 z = __float2bfloat16_rn(0.f);
+  for (int e = t; e < ELL * pad; e += run) {
+    const size_t idx = ((size_t)b * ELL + e / pad) * Kp + K + e % pad;
+    Cs[idx] = z;
+    Cs[plane + idx] = z;
+  }
+}
+
 // 128-thread blocks (64 registers each) so that the solve fits beside the
 // chunk-gradient kernel's register file when both run concurrently.
 constexpr int kPatThreads = 128;
@@ -486,6 +520,7 @@ __global__ void __launch_bounds__(kPatThreads) k_patterns(const double* __restri
 #pragma unroll
           for (int k = 0; k < ELL; ++k) Cb[(size_t)a * N * ELL + k] = Pf[a][k];
       }
+      if (out.Cs) write_planes<ELL>(out.Cs, out.Kp, npat, b, i, Pf);
       if (out.delta_out) out.delta_out[(size_t)b * N + i] = (uint8_t)D;
       if (out.support) {
         uint8_t* row = out.support + ((size_t)b * N + i) * m;
@@ -495,6 +530,10 @@ __global__ void __launch_bounds__(kPatThreads) k_patterns(const double* __restri
       }
       my_err += err;
       my_def += D < ELL ? ELL - D : 0;
+    }
+    if (out.Cs) {
+      const int t0 = ppb > 0 ? tid - (tid / N) * N : tid;
+      zero_pad<ELL>(out.Cs, out.Kp, N, npat, b, t0, ppb > 0 ? N : kPatThreads);
     }
   }
   s_err[tid] = my_err;
@@ -609,6 +648,7 @@ __global__ void __launch_bounds__(128) k_patterns_warp(const double* __restrict_
 #pragma unroll
           for (int k = 0; k < ELL; ++k) Cb[(size_t)a * N * ELL + k] = Pf[a][k];
       }
+      if (out.Cs) write_planes<ELL>(out.Cs, out.Kp, npat, b, i, Pf);
       if (out.delta_out) out.delta_out[(size_t)b * N + i] = (uint8_t)D;
       if (out.support) {
         uint8_t* row = out.support + ((size_t)b * N + i) * m;
@@ -618,6 +658,7 @@ __global__ void __launch_bounds__(128) k_patterns_warp(const double* __restrict_
       }
       def = D < ELL ? ELL - D : 0;
     }
+    if (out.Cs) zero_pad<ELL>(out.Cs, out.Kp, N, npat, b, lane, 32);
     // fixed xor tree over the 32 lanes (deterministic)
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) {

@@ -291,3 +291,30 @@ def test_encode_with_coeffs_matches_encode(gc):
         r = O.run_pattern(R, order, psi[b], N, G.astype(np.float64))
         if np.max(np.abs(r.T)) > 0:
             assert rel_inf(to_np(T2[b]), r.T) <= 1e-4
+
+
+@pytest.mark.parametrize("ell", [1, 3])
+def test_decode_plan_then_apply(gc, ell):
+    """gc_decode_plan (psi side) then gc_decode_apply (data side) equals
+    gc_decode_batch bit for bit and the oracle within tolerance; l = 3 has
+    padding columns (N*l = 18 of 64) that the plan must zero."""
+    cfg = get("tiny")
+    N, m, delta, d = cfg.N, cfg.m, cfg.delta, cfg.d
+    order = O.cyclic_order(N, m, delta)
+    R = make_R(cfg, ell)
+    psi = make_patterns(cfg, npat=300, stream=77)
+    G = np.random.default_rng(21).standard_normal((N, d)).astype(np.float32)
+    Rd, od, pd = dev_tensors(R, order, psi)
+    Gd = torch.from_numpy(G).cuda()
+    # dirty plan buffer: every byte the apply reads must be written by the plan
+    nb = gc.lib.gc_decode_plan_bytes(N, ell, psi.shape[0])
+    plan = torch.full((nb,), 0x7f, dtype=torch.uint8, device="cuda")
+    pl = gc.gc_decode_plan(Rd, ell, od, N, m, delta, pd, plan=plan)
+    ap = gc.gc_decode_apply(pl["plan"], ell, N, psi.shape[0], Gd)
+    ref = gc.gc_decode_batch(Rd, ell, od, N, m, delta, pd, Gd)
+    assert torch.equal(ap["Ghat"], ref["Ghat"])
+    assert torch.equal(ap["grad_mse"], ref["grad_mse"])
+    assert torch.equal(pl["coef_err"], ref["coef_err"]) and torch.equal(pl["est"], ref["est"])
+    for b in range(0, psi.shape[0], 7):
+        r = O.run_pattern(R, order, psi[b], N, G.astype(np.float64), want_transmit=False)
+        assert_grad_close(to_np(ap["Ghat"][b]), r.ghat, f"plan/apply b={b}")
