@@ -125,6 +125,23 @@ class Clocks:
                 "power_w_max": max(power) if power else None, "reasons": sorted(reasons)}
 
 
+# ------------------------------------------------------------------ multi-rank bookkeeping
+def max_over_ranks(values, world, device="cpu"):
+    """Element-wise max of per-rank timings (the slowest rank decides)."""
+    import torch
+
+    t = torch.tensor([float(v) for v in values], dtype=torch.float64, device=device)
+    if world > 1:
+        import torch.distributed as tdist
+        tdist.all_reduce(t, op=tdist.ReduceOp.MAX)
+    return t.tolist()
+
+
+def job_rate(units_per_rank, world, ms):
+    """Whole-job throughput: units all ranks processed / slowest rank's time."""
+    return world * units_per_rank / (ms / 1e3)
+
+
 # ------------------------------------------------------------------ oracle timing
 def oracle_step_rate(cfg, data_cpu, ell, n_sample, seed_stream):
     """Time the fp64 oracle on this host: one full chunk-gradient pass plus
@@ -401,12 +418,9 @@ def gpu_arm(args, rank, world, local_rank):
     assert np.all(np.isfinite(out_mse.numpy())) and np.all(out_est.numpy() >= 0)
 
     # ---- max over ranks
-    times = torch.tensor([total_ms, e2e_ms], dtype=torch.float64, device=dev)
-    if world > 1:
-        tdist.all_reduce(times, op=tdist.ReduceOp.MAX)
-    total_ms, e2e_ms = times.tolist()
-    value = world * npat * K / (total_ms / 1e3)
-    e2e_value = world * npat * K / (e2e_ms / 1e3)
+    total_ms, e2e_ms = max_over_ranks([total_ms, e2e_ms], world, dev)
+    value = job_rate(npat * K, world, total_ms)
+    e2e_value = job_rate(npat * K, world, e2e_ms)
 
     # ---- roofline of the dominant stage
     pk, pk_src = peaks()

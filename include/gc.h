@@ -80,6 +80,26 @@ int gc_version(void);
  * (launches recorded into a CUDA graph count once, at capture). */
 uint64_t gc_kernel_launches(void);
 
+/* Testing aid for the failure path: device waits (TMA and MMA mbarriers,
+ * cluster exchanges) give up after `cycles` SM clock cycles in kernels
+ * launched after this call (0 restores the defaults, about 1-2 s); a kernel
+ * that gives up records GC_ERR_TIMEOUT in its workspace status, drains its
+ * own copies and tensor-core work with separate fixed limits, and returns,
+ * leaving the CUDA context usable.  Process-wide. */
+int gc_set_wait_limit(int64_t cycles);
+
+/* Testing aid for the failure path, together with gc_set_wait_limit: arms a
+ * withheld copy in the NEXT launch of each kernel selected by `kernels` (an OR
+ * of the bits below; 0 disarms).  That launch's loader issues no copy and
+ * arrives on nothing, so its consumers wait on a barrier that nothing
+ * completes; the wait expires after the wait limit, the kernel records
+ * GC_ERR_TIMEOUT and returns, and the results of that call are undefined.  The
+ * bit is consumed by the launch it affects.  Do not arm it while capturing a
+ * CUDA graph (the capture would keep the withheld copy).  Process-wide. */
+#define GC_STALL_CHUNK_GRADS 1 /* the chunk-gradient kernel (gc_chunk_grads)  */
+#define GC_STALL_COMBINE 2     /* the tensor-core combine (decode apply, MSE) */
+int gc_inject_stall(int kernels);
+
 /* Zero the status header of a workspace (asynchronous on `stream`). */
 int gc_workspace_init(void* ws, size_t ws_bytes, void* stream);
 

@@ -35,6 +35,10 @@ from .binding import (  # noqa: F401
     gc_make_assignment,
     gc_mse,
     gc_mse_workspace,
+    gc_set_wait_limit,
+    gc_inject_stall,
+    GC_STALL_CHUNK_GRADS,
+    GC_STALL_COMBINE,
     gc_sgd_step,
     gc_status,
     gc_version,

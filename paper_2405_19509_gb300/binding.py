@@ -39,6 +39,8 @@ def _sig(name, res, *args):
 _sig("gc_last_error", ctypes.c_char_p)
 _sig("gc_version", _i)
 _sig("gc_kernel_launches", ctypes.c_uint64)
+_sig("gc_set_wait_limit", _i, _i64)
+_sig("gc_inject_stall", _i, _i)
 _sig("gc_workspace_init", _i, _p, _sz, _p)
 _sig("gc_status", _i, _p, _p)
 _sig("gc_make_assignment", _i, _i, _i, _i, _i, _p, _p, _p, _p)
@@ -336,6 +338,20 @@ def gc_decode_apply(plan, ell, N, npat, G, Ghat=True, grad_mse=True, ws: Workspa
                                _dev(Ghat, torch.float32, "Ghat", (npat, d)),
                                _dev(grad_mse, torch.float64, "grad_mse"), wp, wn, _stream()))
     return {"Ghat": Ghat, "grad_mse": grad_mse}
+
+
+def gc_set_wait_limit(cycles: int) -> None:
+    """Testing aid: device waits give up after `cycles` clock cycles (0 = default)."""
+    _check(lib.gc_set_wait_limit(int(cycles)))
+
+
+GC_STALL_CHUNK_GRADS = 1
+GC_STALL_COMBINE = 2
+
+
+def gc_inject_stall(kernels: int) -> None:
+    """Testing aid: the next launch of each selected kernel withholds its copies."""
+    _check(lib.gc_inject_stall(int(kernels)))
 
 
 def gc_kernel_launches() -> int:

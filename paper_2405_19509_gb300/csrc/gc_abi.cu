@@ -31,6 +31,14 @@ int cuda_check(cudaError_t e, const char* what) {
 static std::atomic<uint64_t> g_launches{0};
 void count_launches(int n) { g_launches.fetch_add((uint64_t)n, std::memory_order_relaxed); }
 
+static std::atomic<long long> g_wait_limit{0};
+long long wait_limit(long long dflt) {
+  const long long v = g_wait_limit.load(std::memory_order_relaxed);
+  return v > 0 ? v : dflt;
+}
+static std::atomic<int> g_stall{0};
+bool take_stall(int bit) { return (g_stall.fetch_and(~bit) & bit) != 0; }
+
 int device_sm_count() {
   int dev = 0, n = 0;
   if (cudaGetDevice(&dev) != cudaSuccess) return 152;
@@ -94,6 +102,19 @@ const char* gc_last_error(void) { return g_err; }
 int gc_version(void) { return 100; }
 
 uint64_t gc_kernel_launches(void) { return g_launches.load(); }
+
+int gc_inject_stall(int kernels) {
+  if (kernels & ~(GC_STALL_CHUNK_GRADS | GC_STALL_COMBINE))
+    return fail(GC_ERR_ARG, "kernels=0x%x has unknown bits", kernels);
+  g_stall.store(kernels);
+  return GC_OK;
+}
+
+int gc_set_wait_limit(int64_t cycles) {
+  if (cycles < 0) return fail(GC_ERR_ARG, "cycles=%lld must be >= 0", (long long)cycles);
+  g_wait_limit.store(cycles, std::memory_order_relaxed);
+  return GC_OK;
+}
 
 int gc_workspace_init(void* ws, size_t ws_bytes, void* stream) {
   if (!ws || ws_bytes < kHeaderBytes) return fail(GC_ERR_WORKSPACE, "workspace missing or < 256 bytes");

@@ -52,6 +52,11 @@ int device_sm_count();
 
 // Launch accounting for gc_kernel_launches().
 void count_launches(int n);
+// Limit (clock cycles) of the bounded device waits of kernels launched now:
+// `dflt` unless gc_set_wait_limit set one.
+long long wait_limit(long long dflt);
+// True (once) when gc_inject_stall armed `bit` for the next launch.
+bool take_stall(int bit);
 
 // ---- holder table: copies of every chunk, sorted by worker --------------
 // hold_w[i*GC_MAX_REPL + h], hold_p[...]: worker and slot of the h-th holder of

@@ -139,6 +139,8 @@ struct CGArgs {
   int loss;
   int want_loss;
   int use_tma;
+  long long spin_limit;  // clock cycles a wait may take before the kernel gives up
+  int stall;             // failure-path test: the loader issues nothing
   float* parts;        // [clusters][maxt][d]
   double* loss_parts;  // [clusters]
   uint32_t* status;
@@ -167,13 +169,13 @@ __device__ __forceinline__ bool mbar_try_wait_cluster(uint64_t* bar, uint32_t pa
 }
 // Bounded wait; `cl` selects cluster-scope acquire (remote arrivals).
 __device__ __forceinline__ bool bounded_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag,
-                                             uint32_t* status, bool cl = false) {
+                                             uint32_t* status, long long limit, bool cl = false) {
   auto tw = [&]() { return cl ? mbar_try_wait_cluster(bar, parity) : mbar_try_wait(bar, parity); };
   if (tw()) return true;
   const long long t0 = clock64();
   while (!tw()) {
     if (*abort_flag) return false;
-    if (clock64() - t0 > kSpinLimit) {
+    if (clock64() - t0 > limit) {
       atomicOr(status, ST_TIMEOUT);
       *abort_flag = 1;
       return false;
@@ -225,11 +227,17 @@ __global__ void __launch_bounds__(NT + 32, 1) k_chunkgrad(CGArgs a) {
 
   if (warp == NW) {
     // ------------------------------------------------------------ producer warp
+    // A batch is issued only while no wait has failed: then every earlier
+    // batch of the stage has landed (its consumers' waits succeeded), so each
+    // stage holds at most one copy in flight and the phases stay in order.
+    // The decision is warp-uniform.
     const uint32_t row_bytes = (uint32_t)(a.Wc * sizeof(T));
-    for (int n = 0; n < nb; ++n) {
+    int issued = 0;
+    for (int n = 0; n < (a.stall ? 0 : nb); ++n) {
       const int s = n % a.S;
       const uint32_t ph = (uint32_t)((n / a.S) & 1);
-      if (!bounded_wait(&empty[s], ph ^ 1, abort_flag, a.status)) break;
+      const bool ok = bounded_wait(&empty[s], ph ^ 1, abort_flag, a.status, a.spin_limit);
+      if (!__all_sync(0xffffffffu, ok && !*abort_flag)) break;
       T* st = stages + s * stage_elems;
       const long long row = r0 + (long long)n * a.RB;
       if (a.use_tma) {
@@ -249,12 +257,13 @@ __global__ void __launch_bounds__(NT + 32, 1) k_chunkgrad(CGArgs a) {
         }
         mbar_arrive_local(&full[s]);
       }
+      issued = n + 1;
     }
     // drain: the CTA must not exit with copies in flight
     if (a.use_tma && lane == 0) {
       volatile int no_abort = 0;
-      for (int n = max(0, nb - a.S); n < nb; ++n)
-        bounded_wait(&full[n % a.S], (uint32_t)((n / a.S) & 1), &no_abort, a.status);
+      for (int n = max(0, issued - a.S); n < issued; ++n)
+        bounded_wait(&full[n % a.S], (uint32_t)((n / a.S) & 1), &no_abort, a.status, kSpinLimit);
     }
   } else {
     // ------------------------------------------------------------ consumer warps
@@ -295,7 +304,7 @@ __global__ void __launch_bounds__(NT + 32, 1) k_chunkgrad(CGArgs a) {
     // the send to every peer.  Returns the CTA sums in every lane.
     auto pass1 = [&](int n, float (&z)[RBM]) {
       const int s = n % a.S;
-      bounded_wait(&full[s], (uint32_t)((n / a.S) & 1), abort_flag, a.status);
+      bounded_wait(&full[s], (uint32_t)((n / a.S) & 1), abort_flag, a.status, a.spin_limit);
       const T* st = stages + s * stage_elems;
       float pd[RBM];
 #pragma unroll
@@ -332,8 +341,10 @@ __global__ void __launch_bounds__(NT + 32, 1) k_chunkgrad(CGArgs a) {
         for (int o = 16; o > 0; o >>= 1) t += __shfl_xor_sync(0xffffffffu, t, o);
         z[r] = t;
       }
-      if (CL > 1 && tid < CL) {
-        // thread p writes the CTA sums into peer p's slot and arrives there (release)
+      if (CL > 1 && tid < CL && !*abort_flag) {
+        // thread p writes the CTA sums into peer p's slot and arrives there
+        // (release).  After a failed wait the CTA sends no more: a peer then
+        // never receives more arrivals in one phase than it expects.
         float* zc = zcl + (n % kZSlots) * CL * RBM;
         const uint32_t peer = (uint32_t)tid;
 #pragma unroll
@@ -357,7 +368,7 @@ __global__ void __launch_bounds__(NT + 32, 1) k_chunkgrad(CGArgs a) {
       if (n + 1 < nb) pass1(n + 1, znext);
       if (CL > 1) {
         bounded_wait(&zfull[n % kZSlots], (uint32_t)((n / kZSlots) & 1), abort_flag, a.status,
-                     true);
+                     a.spin_limit, true);
         const float* zc = zcl + (n % kZSlots) * CL * RBM;
 #pragma unroll
         for (int r = 0; r < RBM; ++r) {
@@ -685,6 +696,8 @@ int launch_chunkgrad(const void* X, int x_dtype, const float* y, const float* w,
   a.loss = loss;
   a.want_loss = loss_out != nullptr;
   a.use_tma = p.use_tma;
+  a.spin_limit = wait_limit(kSpinLimit);
+  a.stall = take_stall(GC_STALL_CHUNK_GRADS) ? 1 : 0;
   a.parts = ws.take<float>((size_t)p.nclusters * p.maxt * d);
   a.loss_parts = ws.take<double>(p.nclusters);
   a.status = status;

@@ -68,6 +68,8 @@ struct Params {
   const float* gsum;    // d, or null when no MSE is wanted
   float* msep;          // M x parts_per_row partial squared errors, or null
   int parts_per_row;    // num_n_tiles * (epilogue warps per TMEM lane quarter)
+  long long spin_limit; // clock cycles a wait may take before the kernel gives up
+  int stall;            // failure-path test: the TMA producer issues nothing
   uint32_t* status;
 };
 
@@ -98,7 +100,7 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
 }
 // Bounded wait; gives up when the limit passes or another role aborted.
 __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag,
-                                          uint32_t* status, long long limit = kSpin) {
+                                          uint32_t* status, long long limit) {
   if (mbar_try_wait(bar, parity)) return true;
   const long long t0 = clock64();
   while (!mbar_try_wait(bar, parity)) {
@@ -234,13 +236,13 @@ __global__ void __launch_bounds__(64 + 32 * EPI, 1)
     // ------------------------------------------------------------- producer
     if (lane == 0) {
       uint32_t it = 0;
-      bool ok = true;
+      bool ok = !p.stall;
       for (long long t = blockIdx.x; t < p.num_tiles && ok; t += gridDim.x) {
         const int nt = (int)(t / p.num_m_tiles), mt = (int)(t % p.num_m_tiles);
         for (int kb = 0; kb < p.nkb; ++kb, ++it) {
           const int s = it % STAGES;
           const uint32_t ph = (it / STAGES) & 1;
-          if (!mbar_wait(&empty[s], ph ^ 1, abort_flag, p.status)) {
+          if (!mbar_wait(&empty[s], ph ^ 1, abort_flag, p.status, p.spin_limit)) {
             ok = false;
             break;
           }
@@ -264,13 +266,14 @@ __global__ void __launch_bounds__(64 + 32 * EPI, 1)
       bool ok = true;
       for (long long t = blockIdx.x; t < p.num_tiles && ok; t += gridDim.x, ++tile_it) {
         const int ab = tile_it & 1;
-        if (!mbar_wait(&tempty[ab], ((tile_it >> 1) & 1) ^ 1, abort_flag, p.status)) break;
+        if (!mbar_wait(&tempty[ab], ((tile_it >> 1) & 1) ^ 1, abort_flag, p.status, p.spin_limit))
+          break;
         fence_after();
         const uint32_t d_tmem = tmem_base + (uint32_t)(ab * BN);
         for (int kb = 0; kb < p.nkb; ++kb, ++it) {
           const int s = it % STAGES;
           const uint32_t ph = (it / STAGES) & 1;
-          if (!mbar_wait(&full[s], ph, abort_flag, p.status)) {
+          if (!mbar_wait(&full[s], ph, abort_flag, p.status, p.spin_limit)) {
             ok = false;
             break;
           }
@@ -309,7 +312,9 @@ __global__ void __launch_bounds__(64 + 32 * EPI, 1)
     for (long long t = blockIdx.x; t < p.num_tiles; t += gridDim.x, ++tile_it) {
       const int ab = tile_it & 1;
       const int nt = (int)(t / p.num_m_tiles), mt = (int)(t % p.num_m_tiles);
-      if (!mbar_wait(&tfull[ab], (tile_it >> 1) & 1, abort_flag, p.status)) break;
+      // warp-uniform: the TMEM loads below are warp-collective
+      const bool ready = mbar_wait(&tfull[ab], (tile_it >> 1) & 1, abort_flag, p.status, p.spin_limit);
+      if (!__all_sync(0xffffffffu, ready)) break;
       fence_after();
       const int row = mt * BM + quarter * 32 + lane;
       const bool rv = row < p.M;
@@ -612,6 +617,8 @@ int launch_apply(const __nv_bfloat16* Cs, const float* G, int N, int ell, int np
   p.gsum = grad_mse ? gsum : nullptr;
   p.msep = msep;
   p.status = status;
+  p.spin_limit = wait_limit(kSpin);
+  p.stall = take_stall(GC_STALL_COMBINE) ? 1 : 0;
   const bool one_block = p.nkb == 1;
   p.parts_per_row = nnt * (one_block ? 2 : 1);
   const int sms = device_sm_count();

@@ -126,3 +126,11 @@ def test_workspace_sizes_monotone():
     assert 0 < a < b
     assert L.gc_chunk_grads_workspace(20, 512, 4096, 0) > 256
     assert L.gc_coeff_workspace(6, 6, 3, 9, 4) == 0   # unsupported -> 0
+
+
+def test_wait_limit_knob_validation():
+    gc = _lib()
+    assert gc.lib.gc_set_wait_limit(-1) == -1
+    assert gc.lib.gc_set_wait_limit(0) == 0
+    assert gc.lib.gc_inject_stall(4) == -1
+    assert gc.lib.gc_inject_stall(0) == 0
