@@ -187,6 +187,33 @@ __device__ __forceinline__ void consumer_sync(int nthreads) {
   asm volatile("bar.sync 1, %0;" ::"r"(nthreads) : "memory");
 }
 
+// Warp sums of R row partials with a halving butterfly: log2(R) exchange
+// levels that each halve the vector, then plain xor levels -- 5 + R - 1
+// shuffles instead of 5 R.  Lane l ends with the warp sum of row l >> (5 - log2 R).
+template <int R>
+__device__ __forceinline__ float warp_sum_rows(const float (&p)[R], int lane) {
+  constexpr int LR = R >= 4 ? 2 : (R >= 2 ? 1 : 0);
+  static_assert((1 << LR) == R, "rows per batch must be 1, 2 or 4");
+  float v[R];
+#pragma unroll
+  for (int j = 0; j < R; ++j) v[j] = p[j];
+#pragma unroll
+  for (int lvl = 0; lvl < LR; ++lvl) {
+    const int off = 16 >> lvl;
+    const int half = R >> (lvl + 1);
+    const bool hi = (lane & off) != 0;
+#pragma unroll
+    for (int j = 0; j < half; ++j) {
+      const float keep = hi ? v[half + j] : v[j];
+      const float send = hi ? v[j] : v[half + j];
+      v[j] = keep + __shfl_xor_sync(0xffffffffu, send, off);
+    }
+  }
+#pragma unroll
+  for (int lvl = LR; lvl < 5; ++lvl) v[0] += __shfl_xor_sync(0xffffffffu, v[0], 16 >> lvl);
+  return v[0];
+}
+
 // NT consumer threads (warps 0 .. NW-1) plus one producer warp (warp NW).
 template <typename T, int CL, int NT, int NVT, int RBM>
 __global__ void __launch_bounds__(NT + 32, 1) k_chunkgrad(CGArgs a) {
@@ -323,24 +350,26 @@ __global__ void __launch_bounds__(NT + 32, 1) k_chunkgrad(CGArgs a) {
           }
         }
       }
-#pragma unroll
-      for (int r = 0; r < RBM; ++r)
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) pd[r] += __shfl_xor_sync(0xffffffffu, pd[r], o);
+      constexpr int kRowShift = 5 - (RBM >= 4 ? 2 : (RBM >= 2 ? 1 : 0));
+      const float ws_ = warp_sum_rows<RBM>(pd, lane);
       float* redn = red + (n & 1) * NW * RBM;
-      if (lane == 0)
-#pragma unroll
-        for (int r = 0; r < RBM; ++r) redn[warp * RBM + r] = pd[r];
+      if ((lane & ((1 << kRowShift) - 1)) == 0) redn[warp * RBM + (lane >> kRowShift)] = ws_;
       consumer_sync(NT);
-      // every warp reduces the NW partials redundantly (lane w holds warp w's,
-      // zeros past NW), then a full xor tree: identical sums in every lane
+      // CTA sums: the NW x RBM partials are spread over the lanes (entry
+      // j*32 + lane is warp (idx % NW) of row idx / NW), summed over aligned
+      // groups of NW lanes, then row r is read from the first lane of its group.
+      constexpr int E = NW * RBM, NCH = (E + 31) / 32;
+      float cs[NCH];
 #pragma unroll
-      for (int r = 0; r < RBM; ++r) {
-        float t = lane < NW ? redn[lane * RBM + r] : 0.f;
+      for (int j = 0; j < NCH; ++j) {
+        const int idx = j * 32 + lane;
+        float t = idx < E ? redn[(idx % NW) * RBM + idx / NW] : 0.f;
 #pragma unroll
-        for (int o = 16; o > 0; o >>= 1) t += __shfl_xor_sync(0xffffffffu, t, o);
-        z[r] = t;
+        for (int o = NW / 2; o > 0; o >>= 1) t += __shfl_xor_sync(0xffffffffu, t, o);
+        cs[j] = t;
       }
+#pragma unroll
+      for (int r = 0; r < RBM; ++r) z[r] = __shfl_sync(0xffffffffu, cs[(r * NW) / 32], (r * NW) % 32);
       if (CL > 1 && tid < CL && !*abort_flag) {
         // thread p writes the CTA sums into peer p's slot and arrives there
         // (release).  After a failed wait the CTA sends no more: a peer then
@@ -354,6 +383,12 @@ __global__ void __launch_bounds__(NT + 32, 1) k_chunkgrad(CGArgs a) {
       }
     };
 
+    // y of batch n for lane r < RB, loaded two batches ahead (off the
+    // critical path between the dot products and the residuals)
+    auto load_y = [&](int n) {
+      return (lane < a.RB && n < nb) ? __ldg(a.y + r0 + (long long)n * a.RB + lane) : 0.f;
+    };
+    float y0 = load_y(0), y1 = load_y(1);
     float znext[RBM];
     if (nb > 0) pass1(0, znext);
     for (int n = 0; n < nb; ++n) {
@@ -386,6 +421,9 @@ __global__ void __launch_bounds__(NT + 32, 1) k_chunkgrad(CGArgs a) {
         cur = chunk;
       }
       const T* st = stages + s * stage_elems;
+      const float yv = y0;
+      y0 = y1;
+      y1 = load_y(n + 2);
       // ---- residuals: lane r takes row r, then broadcast
       float res[RBM];
       {
@@ -393,7 +431,6 @@ __global__ void __launch_bounds__(NT + 32, 1) k_chunkgrad(CGArgs a) {
 #pragma unroll
         for (int r = 0; r < RBM; ++r) {
           if (lane == r && r < a.RB) {
-            const float yv = __ldg(a.y + row0 + r);
             if (a.loss == GC_LSQ) {
               mine = z[r] - yv;
             } else {
@@ -411,7 +448,6 @@ __global__ void __launch_bounds__(NT + 32, 1) k_chunkgrad(CGArgs a) {
 #pragma unroll
         for (int r = 0; r < RBM; ++r) {
           if (r < a.RB && lane == r) {
-            const float yv = __ldg(a.y + row0 + r);
             if (a.loss == GC_LSQ) {
               const float e = z[r] - yv;
               lr = 0.5f * e * e;
@@ -444,6 +480,9 @@ __global__ void __launch_bounds__(NT + 32, 1) k_chunkgrad(CGArgs a) {
       __syncwarp();
       if (lane == 0) mbar_arrive_local(&empty[s]);
     }
+    // the reduction kernel may be scheduled now (it waits for this grid to
+    // finish); not earlier, so that work on other streams keeps the SMs' room
+    if (tid == 0) asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
     if (cur >= 0) flush(cur);
     if (tid == 0 && rank == 0) a.loss_parts[q] = loss_acc;
   }
@@ -451,8 +490,10 @@ __global__ void __launch_bounds__(NT + 32, 1) k_chunkgrad(CGArgs a) {
 }
 
 // G[i][col] = sum of the partials of chunk i, clusters in increasing order.
-// Block (x, i): chunk i, columns [x*1024, (x+1)*1024); the contributing
-// clusters and their slot offsets are computed once per block.
+// Block (x, i): chunk i, columns [x*256, (x+1)*256), one column per thread;
+// the contributing clusters and their slot offsets are computed once per
+// block.  Launched as a programmatic dependent of k_chunkgrad: the blocks are
+// resident before the gradient kernel ends and wait for it here.
 constexpr int kRedMaxParts = 256;
 __global__ void __launch_bounds__(256) k_chunkgrad_reduce(const float* __restrict__ parts,
                                                           const double* __restrict__ loss_parts,
@@ -473,16 +514,21 @@ __global__ void __launch_bounds__(256) k_chunkgrad_reduce(const float* __restric
     s_np = np;
   }
   __syncthreads();
+  asm volatile("griddepcontrol.wait;" ::: "memory");  // k_chunkgrad has completed
   const int np = s_np;
-  const int c0 = blockIdx.x * 1024;
+  const int col = blockIdx.x * 256 + threadIdx.x;
+  if (col < d) {
+    // independent loads in groups of 8, added in increasing cluster order
+    float acc = 0.f;
+    for (int t0 = 0; t0 < np; t0 += 8) {
+      float v[8];
 #pragma unroll
-  for (int k = 0; k < 4; ++k) {
-    const int col = c0 + k * 256 + threadIdx.x;
-    if (col < d) {
-      float acc = 0.f;
-      for (int t = 0; t < np; ++t) acc += __ldg(parts + s_off[t] + col);
-      G[(size_t)i * d + col] = acc;
+      for (int k = 0; k < 8; ++k) v[k] = t0 + k < np ? __ldg(parts + s_off[t0 + k] + col) : 0.f;
+#pragma unroll
+      for (int k = 0; k < 8; ++k)
+        if (t0 + k < np) acc += v[k];
     }
+    G[(size_t)i * d + col] = acc;
   }
   if (loss_out && blockIdx.x == 0 && blockIdx.y == 0 && threadIdx.x < 32) {
     // lane l adds clusters l, l + 32, ...; then a fixed xor tree
@@ -701,16 +747,27 @@ int launch_chunkgrad(const void* X, int x_dtype, const float* y, const float* w,
   a.parts = ws.take<float>((size_t)p.nclusters * p.maxt * d);
   a.loss_parts = ws.take<double>(p.nclusters);
   a.status = status;
-  int rc = x_dtype == GC_BF16 ? dispatch_cl<__nv_bfloat16>(p, a, s) : dispatch_cl<float>(p, a, s);
-  if (rc != GC_OK) return rc;
   if (p.rpc < 1 || (long long)n_c / p.rpc + 2 > kRedMaxParts)
     return fail(GC_ERR_UNSUPPORTED, "chunk of %d rows spans too many row blocks", n_c);
   if (N > 65535) return fail(GC_ERR_UNSUPPORTED, "N=%d exceeds 65535 chunks", N);
-  dim3 grid((d + 1023) / 1024, N);
-  k_chunkgrad_reduce<<<grid, 256, 0, s>>>(a.parts, a.loss_parts, G, loss_out, N, n_c, d, p.rpc,
-                                          p.maxt, p.nclusters, a.Ntil);
+  int rc = x_dtype == GC_BF16 ? dispatch_cl<__nv_bfloat16>(p, a, s) : dispatch_cl<float>(p, a, s);
+  if (rc != GC_OK) return rc;
+  // the reduction as a programmatic dependent launch (it waits in-kernel)
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = dim3((d + 255) / 256, N);
+  cfg.blockDim = dim3(256);
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  cudaError_t e = cudaLaunchKernelEx(&cfg, k_chunkgrad_reduce, (const float*)a.parts,
+                                     (const double*)a.loss_parts, G, loss_out, N, n_c, d, p.rpc,
+                                     p.maxt, p.nclusters, a.Ntil);
+  if (e != cudaSuccess) return cuda_check(e, "cudaLaunchKernelEx(k_chunkgrad_reduce)");
   count_launches(1);
-  return cuda_check(cudaGetLastError(), "k_chunkgrad_reduce");
+  return GC_OK;
 }
 
 }  // namespace gc

@@ -25,7 +25,11 @@
 //               per row; the accumulator is handed back as soon as it is
 //               read, so the epilogue of tile t overlaps the MMAs of t + 1.
 // Tiles are visited n-tile-major so that concurrently running CTAs share the
-// same B tile through L2.  Every mbarrier wait is bounded; on expiry the
+// same B tile through L2.  When one 64-wide block holds all of K the output
+// write bounds the kernel and the B tile is what the copies would mostly
+// move, so each CTA keeps its B tile resident over a contiguous range of
+// tiles and streams only A (the BRES shape below).
+// Every mbarrier wait is bounded; on expiry the
 // kernel flags GC_ERR_TIMEOUT in the status word, drains its own copies and
 // MMAs (with bounded waits) and frees TMEM.
 #include <cuda.h>
@@ -47,15 +51,22 @@ constexpr int STAGE_BYTES = 2 * A_PLANE + 2 * B_PLANE;  // 96 KB
 constexpr uint32_t TMEM_COLS = 512;
 constexpr long long kSpin = 1LL << 32;  // clock cycles per wait (~2 s)
 constexpr int OUT_BUF = 32 * 32 * 4;                 // one 32 x 32 fp32 store box (4 KB)
-// Two shapes: STAGES = 2 smem stages with 4 epilogue warps when K spans
-// several 64-wide blocks (MMA-bound), STAGES = 1 with 8 epilogue warps (two
-// per TMEM lane quarter, half the columns each) when one block holds all of
-// K and the output write bounds the kernel.
-template <int STAGES, int EPI>
+// Two shapes.  Several 64-wide K blocks (MMA-bound): STAGES = 2 ring stages
+// holding A and B, 4 epilogue warps, tiles dealt round-robin.  One K block
+// (the output write bounds the kernel; BRES): each CTA takes a contiguous
+// n-tile-major range of tiles, keeps the B tile of its current n-tile resident
+// (reloaded only when the n-tile changes), streams A through STAGES = 3 ring
+// stages, and runs 8 epilogue warps (two per TMEM lane quarter).
+constexpr int A_STAGE = 2 * A_PLANE;  // 32 KB
+constexpr int kBresStages = 2;        // A ring stages of the BRES shape
+constexpr int B_TILE = 2 * B_PLANE;   // 64 KB
+template <int STAGES, int EPI, bool BRES>
 struct Shape {
   static constexpr int THREADS = 64 + 32 * EPI;
   static constexpr int OUT_BYTES = EPI * 2 * OUT_BUF;  // 2 staging boxes per epilogue warp
-  static constexpr size_t SMEM = (size_t)STAGES * STAGE_BYTES + OUT_BYTES + 1024 + 256;
+  static constexpr int RING = BRES ? STAGES * A_STAGE + B_TILE : STAGES * STAGE_BYTES;
+  static constexpr size_t SMEM = (size_t)RING + OUT_BYTES + 1024 + 256;
+  static_assert(SMEM <= 232448, "shared memory per CTA");
 };
 
 struct Params {
@@ -189,22 +200,36 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
   for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(r[j]);
 }
 
-template <int STAGES, int EPI>
+template <int STAGES, int EPI, bool BRES>
 __global__ void __launch_bounds__(64 + 32 * EPI, 1)
     k_combine_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                  const __grid_constant__ CUtensorMap tmC, Params p) {
-  constexpr int OUT_BYTES = Shape<STAGES, EPI>::OUT_BYTES;
+  using Sh = Shape<STAGES, EPI, BRES>;
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
-  float* outbuf = reinterpret_cast<float*>(smem + STAGES * STAGE_BYTES);  // 1024-aligned
-  uint64_t* full = reinterpret_cast<uint64_t*>(smem + STAGES * STAGE_BYTES + OUT_BYTES);
+  uint8_t* bres = smem + STAGES * A_STAGE;                       // BRES: resident B tile
+  float* outbuf = reinterpret_cast<float*>(smem + Sh::RING);     // 1024-aligned
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + Sh::RING + Sh::OUT_BYTES);
   uint64_t* empty = full + STAGES;
   uint64_t* tfull = empty + STAGES;   // [2]
   uint64_t* tempty = tfull + 2;       // [2]
   uint64_t* done = tempty + 2;        // MMA drain
-  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(done + 1);
+  uint64_t* bfull = done + 1;         // BRES: B tile landed
+  uint64_t* bempty = bfull + 1;       // BRES: MMAs on the B tile finished
+  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(bempty + 1);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_holder + 1);
+  // this CTA's tiles: t = t_first, t_first + t_step, ... < t_last
+  long long t_first, t_last, t_step;
+  if (BRES) {
+    t_first = (long long)blockIdx.x * p.num_tiles / gridDim.x;
+    t_last = (long long)(blockIdx.x + 1) * p.num_tiles / gridDim.x;
+    t_step = 1;
+  } else {
+    t_first = blockIdx.x;
+    t_last = p.num_tiles;
+    t_step = gridDim.x;
+  }
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
@@ -217,6 +242,8 @@ __global__ void __launch_bounds__(64 + 32 * EPI, 1)
       mbar_init(&tempty[a], EPI);
     }
     mbar_init(done, 1);
+    mbar_init(bfull, 1);
+    mbar_init(bempty, 1);
     *abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
@@ -231,13 +258,45 @@ __global__ void __launch_bounds__(64 + 32 * EPI, 1)
   __syncthreads();
   fence_after();
   const uint32_t tmem_base = *tmem_holder;
+  // launched as a programmatic dependent of the operand split: the prologue
+  // above overlaps its tail, the operands are read only after this point
+  asm volatile("griddepcontrol.wait;" ::: "memory");
 
   if (warp == 0) {
     // ------------------------------------------------------------- producer
-    if (lane == 0) {
+    if (lane == 0 && BRES) {
+      uint32_t it = 0, nb_loads = 0;
+      int cur_nt = -1;
+      bool ok = !p.stall;
+      for (long long t = t_first; t < t_last && ok; t += t_step) {
+        const int nt = (int)(t / p.num_m_tiles), mt = (int)(t % p.num_m_tiles);
+        if (nt != cur_nt) {
+          // the MMAs on the previous B tile have finished before it is replaced
+          if (nb_loads > 0 &&
+              !mbar_wait(bempty, (nb_loads - 1) & 1, abort_flag, p.status, p.spin_limit))
+            break;
+          mbar_expect_tx(bfull, B_TILE);
+          tma_load_3d(bres, &tmB, 0, nt * BN, 0, bfull);
+          cur_nt = nt;
+          ++nb_loads;
+        }
+        const int s = it % STAGES;
+        const uint32_t ph = (it / STAGES) & 1;
+        if (!mbar_wait(&empty[s], ph ^ 1, abort_flag, p.status, p.spin_limit)) break;
+        uint8_t* st = smem + s * A_STAGE;
+        mbar_expect_tx(&full[s], A_STAGE);
+        tma_load_3d(st, &tmA, 0, mt * BM, 0, &full[s]);
+        ++it;
+      }
+      // drain: every issued copy has landed before the CTA may exit
+      volatile int no_abort = 0;
+      for (uint32_t k = (it > (uint32_t)STAGES ? it - STAGES : 0); k < it; ++k)
+        mbar_wait(&full[k % STAGES], (k / STAGES) & 1, &no_abort, p.status, 1LL << 28);
+      if (nb_loads > 0) mbar_wait(bfull, (nb_loads - 1) & 1, &no_abort, p.status, 1LL << 28);
+    } else if (lane == 0) {
       uint32_t it = 0;
       bool ok = !p.stall;
-      for (long long t = blockIdx.x; t < p.num_tiles && ok; t += gridDim.x) {
+      for (long long t = t_first; t < t_last && ok; t += t_step) {
         const int nt = (int)(t / p.num_m_tiles), mt = (int)(t % p.num_m_tiles);
         for (int kb = 0; kb < p.nkb; ++kb, ++it) {
           const int s = it % STAGES;
@@ -261,10 +320,46 @@ __global__ void __launch_bounds__(64 + 32 * EPI, 1)
     }
   } else if (warp == 1) {
     // ------------------------------------------------------------- MMA issuer
-    if (lane == 0) {
+    if (lane == 0 && BRES) {
+      uint32_t it = 0, tile_it = 0, nb_used = 0;
+      int cur_nt = -1;
+      for (long long t = t_first; t < t_last; t += t_step, ++tile_it) {
+        const int nt = (int)(t / p.num_m_tiles);
+        if (nt != cur_nt) {
+          if (!mbar_wait(bfull, nb_used & 1, abort_flag, p.status, p.spin_limit)) break;
+          ++nb_used;
+          cur_nt = nt;
+        }
+        const int ab = tile_it & 1;
+        if (!mbar_wait(&tempty[ab], ((tile_it >> 1) & 1) ^ 1, abort_flag, p.status, p.spin_limit))
+          break;
+        const int s = it % STAGES;
+        if (!mbar_wait(&full[s], (it / STAGES) & 1, abort_flag, p.status, p.spin_limit)) break;
+        fence_after();
+        const uint32_t d_tmem = tmem_base + (uint32_t)(ab * BN);
+        const uint32_t a_hi = smem_u32(smem + s * A_STAGE), a_lo = a_hi + A_PLANE;
+        const uint32_t b_hi = smem_u32(bres), b_lo = b_hi + B_PLANE;
+        const int nks = p.K >= BK ? BK / 16 : (p.K + 15) / 16;
+        for (int ks = 0; ks < nks; ++ks) {
+          const uint32_t off = ks * 32;
+          mma_bf16(d_tmem, sdesc(a_hi + off), sdesc(b_hi + off), ks > 0 ? 1u : 0u);
+          mma_bf16(d_tmem, sdesc(a_hi + off), sdesc(b_lo + off), 1u);
+          mma_bf16(d_tmem, sdesc(a_lo + off), sdesc(b_hi + off), 1u);
+        }
+        mma_commit(&empty[s]);
+        ++it;
+        mma_commit(&tfull[ab]);
+        // last tile on this B tile: hand it back once these MMAs complete
+        const bool last_on_b = t + t_step >= t_last || (int)((t + t_step) / p.num_m_tiles) != nt;
+        if (last_on_b) mma_commit(bempty);
+      }
+      mma_commit(done);
+      volatile int no_abort = 0;
+      mbar_wait(done, 0, &no_abort, p.status, 1LL << 28);
+    } else if (lane == 0) {
       uint32_t it = 0, tile_it = 0;
       bool ok = true;
-      for (long long t = blockIdx.x; t < p.num_tiles && ok; t += gridDim.x, ++tile_it) {
+      for (long long t = t_first; t < t_last && ok; t += t_step, ++tile_it) {
         const int ab = tile_it & 1;
         if (!mbar_wait(&tempty[ab], ((tile_it >> 1) & 1) ^ 1, abort_flag, p.status, p.spin_limit))
           break;
@@ -309,7 +404,7 @@ __global__ void __launch_bounds__(64 + 32 * EPI, 1)
     const int cbeg = (e / 4) * SPAN;
     float* wbuf = outbuf + e * 2 * (OUT_BUF / 4);
     uint32_t tile_it = 0, chunk_it = 0;
-    for (long long t = blockIdx.x; t < p.num_tiles; t += gridDim.x, ++tile_it) {
+    for (long long t = t_first; t < t_last; t += t_step, ++tile_it) {
       const int ab = tile_it & 1;
       const int nt = (int)(t / p.num_m_tiles), mt = (int)(t % p.num_m_tiles);
       // warp-uniform: the TMEM loads below are warp-collective
@@ -410,6 +505,9 @@ __global__ void __launch_bounds__(64 + 32 * EPI, 1)
   }
   fence_before();
   __syncthreads();
+  // every role is done: the MSE reduction may be scheduled (it waits for
+  // this grid to finish); earlier, its waiting blocks would hold SM room
+  if (threadIdx.x == 0) asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   if (warp == 1) {
     fence_after();
     asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem_base),
@@ -438,6 +536,8 @@ __global__ void k_split_c(const float* __restrict__ C, int M, int K, int Kp,
 // gsum[k'*L + c] = sum_i g_{D_i}[k'*L + c] (chunks in order) when gsum != 0.
 __global__ void k_split_gt(const float* __restrict__ G, int N, int d, int ell, int L, int Kp,
                            __nv_bfloat16* __restrict__ out, float* __restrict__ gsum) {
+  // the combine kernel may be scheduled now; it waits for this grid to finish
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   __shared__ float tile[32][33];
   const int c0 = blockIdx.x * 32, k0 = blockIdx.y * 32;
   const int tx = threadIdx.x, ty = threadIdx.y;  // 32 x 8
@@ -476,16 +576,23 @@ __global__ void k_split_gt(const float* __restrict__ G, int N, int d, int ell, i
   }
 }
 
+// grad_mse[b] = (sum of the partial squared errors of rows b*ell .. b*ell+ell-1) / d:
+// one warp per pattern (its ell * parts partials are contiguous), lanes
+// stride over them, then a fixed xor tree in fp64.  Launched as a
+// programmatic dependent of the combine kernel.
 __global__ void k_mse_reduce_tiles(const float* __restrict__ msep, int npat, int ell,
                                    int parts, int d, double* __restrict__ grad_mse) {
-  const int b = blockIdx.x * blockDim.x + threadIdx.x;
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  const long long b = ((long long)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const int lane = threadIdx.x & 31;
   if (b >= npat) return;
+  const float* r = msep + (size_t)b * ell * parts;
+  const int n = ell * parts;
   double s = 0.0;
-  for (int k = 0; k < ell; ++k) {
-    const float* r = msep + ((size_t)b * ell + k) * parts;
-    for (int t = 0; t < parts; ++t) s += (double)r[t];
-  }
-  grad_mse[b] = s / (double)d;
+  for (int t = lane; t < n; t += 32) s += (double)__ldg(r + t);
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+  if (lane == 0) grad_mse[b] = s / (double)d;
 }
 
 PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
@@ -534,18 +641,29 @@ int make_map(CUtensorMap* map, const void* base, int rows, int Kp, int box_rows)
 
 }  // namespace tc
 
-template <int STAGES, int EPI>
+template <int STAGES, int EPI, bool BRES>
 int launch_tc(int grid, const CUtensorMap& mA, const CUtensorMap& mB, const CUtensorMap& mC,
               const tc::Params& p, cudaStream_t s) {
-  using Sh = tc::Shape<STAGES, EPI>;
+  using Sh = tc::Shape<STAGES, EPI, BRES>;
   static bool attr_set = false;
   if (!attr_set) {
-    cudaError_t e = cudaFuncSetAttribute(tc::k_combine_tc<STAGES, EPI>,
+    cudaError_t e = cudaFuncSetAttribute(tc::k_combine_tc<STAGES, EPI, BRES>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, (int)Sh::SMEM);
     if (e != cudaSuccess) return cuda_check(e, "cudaFuncSetAttribute(k_combine_tc)");
     attr_set = true;
   }
-  tc::k_combine_tc<STAGES, EPI><<<grid, Sh::THREADS, Sh::SMEM, s>>>(mA, mB, mC, p);
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = dim3(grid);
+  cfg.blockDim = dim3(Sh::THREADS);
+  cfg.dynamicSmemBytes = Sh::SMEM;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  cudaError_t e = cudaLaunchKernelEx(&cfg, tc::k_combine_tc<STAGES, EPI, BRES>, mA, mB, mC, p);
+  if (e != cudaSuccess) return cuda_check(e, "cudaLaunchKernelEx(k_combine_tc)");
   count_launches(1);
   return cuda_check(cudaGetLastError(), "k_combine_tc");
 }
@@ -623,14 +741,23 @@ int launch_apply(const __nv_bfloat16* Cs, const float* G, int N, int ell, int np
   p.parts_per_row = nnt * (one_block ? 2 : 1);
   const int sms = device_sm_count();
   const int grid = (int)std::min<long long>(p.num_tiles, sms);
-  rc = one_block ? launch_tc<1, 8>(grid, mA, mB, mC, p, s) : launch_tc<2, 4>(grid, mA, mB, mC, p, s);
+  rc = one_block ? launch_tc<kBresStages, 8, true>(grid, mA, mB, mC, p, s)
+                 : launch_tc<2, 4, false>(grid, mA, mB, mC, p, s);
   if (rc) return rc;
   if (grad_mse) {
-    k_mse_reduce_tiles<<<(npat + 255) / 256, 256, 0, s>>>(msep, npat, ell, p.parts_per_row, d,
-                                                         grad_mse);
+    cudaLaunchConfig_t cfg{};
+    cfg.gridDim = dim3((unsigned)(((long long)npat * 32 + 255) / 256));
+    cfg.blockDim = dim3(256);
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    cudaError_t e = cudaLaunchKernelEx(&cfg, k_mse_reduce_tiles, (const float*)msep, npat, ell,
+                                       p.parts_per_row, d, grad_mse);
+    if (e != cudaSuccess) return cuda_check(e, "cudaLaunchKernelEx(k_mse_reduce_tiles)");
     count_launches(1);
-    cudaError_t e = cudaGetLastError();
-    if (e != cudaSuccess) return cuda_check(e, "k_mse_reduce_tiles");
   }
   return GC_OK;
 }

@@ -10,13 +10,15 @@ namespace gc {
 // T[b][j][c] = sum_{p < psi[b][j]} sum_k E[b][j][p][k] * g_{order[j][p]}[k*L + c]
 // (g zero past d).  Block = (column tile, worker j, pattern b); worker j's
 // coefficients and chunk list are staged in shared memory (fp32) once per
-// block.
+// block -- delta * (ell + 1) words of dynamic shared memory, so the kernel
+// still fits beside a resident kernel that holds nearly all of an SM's.
 __global__ void k_encode(const double* __restrict__ E, const int32_t* __restrict__ order,
                          const int32_t* __restrict__ psi, int N, int m, int delta, int ell,
                          int npat, const float* __restrict__ G, int d, int L,
                          float* __restrict__ T) {
-  __shared__ float s_e[GC_MAX_DELTA * GC_MAX_ELL];
-  __shared__ int s_chunk[GC_MAX_DELTA];
+  extern __shared__ float s_dyn[];
+  float* s_e = s_dyn;                                          // [delta * ell]
+  int* s_chunk = reinterpret_cast<int*>(s_dyn + delta * ell);  // [delta]
   const int j = blockIdx.y, b = blockIdx.z;
   int np = psi[(size_t)b * m + j];
   np = np < 0 ? 0 : (np > delta ? delta : np);  // bad values are flagged by the solve
@@ -47,18 +49,20 @@ int launch_encode(const double* E, const int32_t* order, const int32_t* psi, int
   if (npat > 65535 || m > 65535) return fail(GC_ERR_UNSUPPORTED, "encode grid: npat and m <= 65535");
   const int threads = 256;
   dim3 grid((L + threads - 1) / threads, m, npat);
-  k_encode<<<grid, threads, 0, s>>>(E, order, psi, N, m, delta, ell, npat, G, d, L, T);
+  const size_t smem = (size_t)delta * (ell + 1) * sizeof(float);
+  k_encode<<<grid, threads, smem, s>>>(E, order, psi, N, m, delta, ell, npat, G, d, L, T);
   count_launches(1);
   return cuda_check(cudaGetLastError(), "k_encode");
 }
 
 // ghat[b][k*L + c] = sum_j R[k][j] * T[b][j][c].  One thread per (b, c); R is
-// staged in shared memory as fp32 (m <= kDecodeSmemM) or read as fp64.
+// staged in dynamic shared memory as fp32 (ELL * m words, m <= kDecodeSmemM)
+// or read as fp64.
 constexpr int kDecodeSmemM = 1024;
 template <int ELL>
 __global__ void k_decode_tx(const double* __restrict__ R, int m, const float* __restrict__ T,
                             int npat, int d, int L, float* __restrict__ ghat) {
-  __shared__ float s_r[ELL * kDecodeSmemM];
+  extern __shared__ float s_r[];
   const bool staged = m <= kDecodeSmemM;
   if (staged)
     for (int t = threadIdx.x; t < ELL * m; t += blockDim.x) s_r[t] = (float)R[t];
@@ -94,15 +98,16 @@ int launch_decode_tx(const double* R, int ell, int m, const float* T, int npat, 
   if (tot == 0) return GC_OK;
   const int threads = 256;
   const unsigned blocks = (unsigned)((tot + threads - 1) / threads);
+  const size_t sm = m <= kDecodeSmemM ? (size_t)ell * m * sizeof(float) : 0;
   switch (ell) {
-    case 1: k_decode_tx<1><<<blocks, threads, 0, s>>>(R, m, T, npat, d, L, ghat); break;
-    case 2: k_decode_tx<2><<<blocks, threads, 0, s>>>(R, m, T, npat, d, L, ghat); break;
-    case 3: k_decode_tx<3><<<blocks, threads, 0, s>>>(R, m, T, npat, d, L, ghat); break;
-    case 4: k_decode_tx<4><<<blocks, threads, 0, s>>>(R, m, T, npat, d, L, ghat); break;
-    case 5: k_decode_tx<5><<<blocks, threads, 0, s>>>(R, m, T, npat, d, L, ghat); break;
-    case 6: k_decode_tx<6><<<blocks, threads, 0, s>>>(R, m, T, npat, d, L, ghat); break;
-    case 7: k_decode_tx<7><<<blocks, threads, 0, s>>>(R, m, T, npat, d, L, ghat); break;
-    case 8: k_decode_tx<8><<<blocks, threads, 0, s>>>(R, m, T, npat, d, L, ghat); break;
+    case 1: k_decode_tx<1><<<blocks, threads, sm, s>>>(R, m, T, npat, d, L, ghat); break;
+    case 2: k_decode_tx<2><<<blocks, threads, sm, s>>>(R, m, T, npat, d, L, ghat); break;
+    case 3: k_decode_tx<3><<<blocks, threads, sm, s>>>(R, m, T, npat, d, L, ghat); break;
+    case 4: k_decode_tx<4><<<blocks, threads, sm, s>>>(R, m, T, npat, d, L, ghat); break;
+    case 5: k_decode_tx<5><<<blocks, threads, sm, s>>>(R, m, T, npat, d, L, ghat); break;
+    case 6: k_decode_tx<6><<<blocks, threads, sm, s>>>(R, m, T, npat, d, L, ghat); break;
+    case 7: k_decode_tx<7><<<blocks, threads, sm, s>>>(R, m, T, npat, d, L, ghat); break;
+    case 8: k_decode_tx<8><<<blocks, threads, sm, s>>>(R, m, T, npat, d, L, ghat); break;
     default: return fail(GC_ERR_UNSUPPORTED, "ell=%d exceeds GC_MAX_ELL", ell);
   }
   count_launches(1);
