@@ -126,6 +126,56 @@ int gc_status(void* ws, void* stream);
 int gc_make_assignment(int N, int m, int delta, int kind, const int32_t* explicit_order_h,
                        uint8_t* A_h, int32_t* order_h, uint8_t* O_h);
 
+/* ---- chunk ordering (Sec. III, Algorithm 2) ------------------------------
+ * Host only.  Given an assignment matrix with N == m in which every row and
+ * every column holds exactly delta non-zeros (e.g. the adjacency matrix of a
+ * delta-regular graph), find an ordering that minimises
+ * Q_max(O) = max_i sum_j O[i][j] + (m - delta - 1) * delta: the bipartite
+ * graph of A is split into delta disjoint perfect matchings P_1..P_delta
+ * (Claim 1 guarantees each exists) and O = sum_p p * P_p, so that every row
+ * sum equals the lower bound delta (delta + 1) / 2.  Each matching is found
+ * by augmenting paths with rows taken in increasing order and each row's
+ * columns in increasing order, so the result is deterministic.
+ *   A_h      N x m uint8 (non-zero = assigned), N == m.
+ * Outputs (host, caller-owned, any may be NULL): order_h (m x delta int32,
+ * W_j's chunks top to bottom) and O_h (N x m uint8) as in gc_make_assignment;
+ * the order is accepted by gc_make_assignment(GC_EXPLICIT).
+ * Errors: GC_ERR_SHAPE (N != m, or a row or column sum differs from delta),
+ * GC_ERR_UNSUPPORTED (delta > GC_MAX_DELTA), GC_ERR_DATA (no perfect matching;
+ * impossible for a valid input).
+ */
+int gc_chunk_ordering(const uint8_t* A_h, int N, int m, int delta, int32_t* order_h, uint8_t* O_h);
+
+/* ---- completion times and the encode-and-transmit trigger (Sec. IV) ----
+ * Batched simulation of the cluster: realization r gives every worker a
+ * time per chunk tau[r][j] (> 0, +inf for a failed worker); W_j finishes
+ * the chunk in its slot p (1-based) at p * tau_j.  With n_i(T) the number of
+ * processed copies of D_i at time T, the PS's error estimate is
+ * est(T) = sum_i max(0, ell - n_i(T)) (eq. (7) and the sentence after it).
+ * For each realization:
+ *   T[r]       the first time with est(T) <= theta: the (N ell - theta)-th
+ *              smallest of the N ell values t_i^(k) (k-th smallest completion
+ *              time of D_i, k <= ell; +inf when too few copies can finish).
+ *              theta = 0: every chunk processed ell times (exact recovery).
+ *   psi[r][j]  chunks W_j has processed by T[r]: #{p <= delta_j : p tau_j <= T}
+ *              (0 for a failed worker) -- the state the PS decodes from.
+ *   T_full[r]  the same time when a copy counts only once its worker has
+ *              finished all delta_j of its chunks (at delta_j tau_j), i.e.
+ *              the original protocol's completion time (Sec. IV).
+ * Times are formed with one double multiply each, exactly as defined, so
+ * results are reproducible bit for bit.
+ *   order   device m x delta int32 (as gc_make_assignment / gc_chunk_ordering).
+ *   tau     device nsim x m fp64.
+ *   T, psi, T_full  device outputs (nsim fp64, nsim x m int32, nsim fp64),
+ *           each nullable.
+ *   Limits: 1 <= ell <= GC_MAX_ELL, 0 <= theta, N * ell <= 2048, m <= 32767.
+ * Workspace: gc_trigger_workspace(N) bytes.
+ */
+size_t gc_trigger_workspace(int N);
+int gc_trigger_times(const int32_t* order, int N, int m, int delta, const double* tau, int64_t nsim,
+                     int ell, int theta, double* T, int32_t* psi, double* T_full, void* ws,
+                     size_t ws_bytes, void* stream);
+
 /* ---- chunk gradients (Sec. I: g_{D_j} = sum_{i in D_j} grad l) --------
  * X        N~ x d, element type x_dtype, row-major, 16-byte aligned; chunk i
  *          is rows [i*n_c, (i+1)*n_c).

@@ -80,6 +80,89 @@ def q_metric(O: np.ndarray, delta: int) -> np.ndarray:
     return Q
 
 
+def chunk_ordering(A: np.ndarray) -> np.ndarray:
+    """Algorithm 2 (Sec. III): for an N == m assignment with every row and
+    column sum delta, peel delta perfect matchings P_1..P_delta off the
+    bipartite graph of A (each exists by Claim 1) and return the ordering
+    matrix O = sum_p p * P_p (N x m uint8).  The matching step is a library
+    maximum bipartite matching; which optimal O comes out depends on it."""
+    from scipy.sparse import csr_matrix
+    from scipy.sparse.csgraph import maximum_bipartite_matching
+
+    At = (np.asarray(A) != 0).astype(np.int64)
+    N, m = At.shape
+    assert N == m, "Algorithm 2 needs N == m"
+    delta = int(At[0].sum())
+    assert np.all(At.sum(axis=0) == delta) and np.all(At.sum(axis=1) == delta)
+    O = np.zeros((N, m), dtype=np.uint8)
+    for p in range(1, delta + 1):
+        match = maximum_bipartite_matching(csr_matrix(At), perm_type="column")  # row i -> column
+        assert np.all(match >= 0), "Claim 1: a perfect matching exists"
+        P = np.zeros_like(At)
+        P[np.arange(N), match] = 1
+        O[P == 1] = p
+        At = At - P
+    assert At.sum() == 0
+    return O
+
+
+def order_from_O(O: np.ndarray) -> np.ndarray:
+    """Per-worker processing order (m x delta, -1 padded) from an ordering
+    matrix: column j lists D_i by increasing O_ij."""
+    N, m = O.shape
+    delta = int(max((O[:, j] > 0).sum() for j in range(m)))
+    order = -np.ones((m, delta), dtype=np.int32)
+    for j in range(m):
+        for i in range(N):
+            if O[i, j]:
+                order[j, int(O[i, j]) - 1] = i
+    return order
+
+
+def completion_times(order: np.ndarray, tau: np.ndarray, N: int, ell: int, theta: int = 0):
+    """Completion-time simulation of Sec. IV.  Realization r: W_j needs
+    tau[r, j] per chunk (+inf = failed) and finishes its p-th chunk (1-based)
+    at p * tau_j.  Returns, per realization,
+      T      the first time at which the error estimate sum_i max(0, ell -
+             n_i(T)) is <= theta, n_i(T) = copies of D_i processed by T
+             (theta = 0: every chunk processed ell times);
+      psi    chunks each worker has processed by T;
+      T_full the same time when a copy counts only once its worker has
+             processed all of its chunks (the original protocol of Sec. IV).
+    The estimate only drops at the ell earliest completion times of each
+    chunk, so T is the (N ell - theta)-th smallest of those N ell times."""
+    tau = np.asarray(tau, dtype=np.float64)
+    m, delta = order.shape
+    dj = [int((order[j] >= 0).sum()) for j in range(m)]
+    nsim = tau.shape[0]
+    T = np.zeros(nsim)
+    TF = np.zeros(nsim)
+    psi = np.zeros((nsim, m), dtype=np.int32)
+    k = N * ell - theta
+    for r in range(nsim):
+        times = [[] for _ in range(N)]
+        times_full = [[] for _ in range(N)]
+        for j in range(m):
+            t = float(tau[r, j])
+            if not math.isfinite(t):
+                continue
+            for p in range(dj[j]):
+                i = int(order[j, p])
+                times[i].append(float(p + 1) * t)
+                times_full[i].append(float(dj[j]) * t)
+        vals, vals_full = [], []
+        for i in range(N):
+            vals += (sorted(times[i]) + [math.inf] * ell)[:ell]
+            vals_full += (sorted(times_full[i]) + [math.inf] * ell)[:ell]
+        T[r] = sorted(vals)[k - 1] if k >= 1 else 0.0
+        TF[r] = sorted(vals_full)[k - 1] if k >= 1 else 0.0
+        for j in range(m):
+            t = float(tau[r, j])
+            if math.isfinite(t):
+                psi[r, j] = sum(1 for p in range(1, dj[j] + 1) if float(p) * t <= T[r])
+    return T, psi, TF
+
+
 # --------------------------------------------------------------------------
 # Chunk gradients (Sec. I): g_{D_j} = sum_{i in D_j} grad l(x_i, y_i, w)
 # --------------------------------------------------------------------------

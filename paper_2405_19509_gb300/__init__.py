@@ -36,6 +36,8 @@ from .binding import (  # noqa: F401
     gc_mse,
     gc_mse_workspace,
     gc_set_wait_limit,
+    gc_chunk_ordering,
+    gc_trigger_times,
     gc_inject_stall,
     GC_STALL_CHUNK_GRADS,
     GC_STALL_COMBINE,

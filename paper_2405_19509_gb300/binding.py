@@ -44,6 +44,9 @@ _sig("gc_inject_stall", _i, _i)
 _sig("gc_workspace_init", _i, _p, _sz, _p)
 _sig("gc_status", _i, _p, _p)
 _sig("gc_make_assignment", _i, _i, _i, _i, _i, _p, _p, _p, _p)
+_sig("gc_chunk_ordering", _i, _p, _i, _i, _i, _p, _p)
+_sig("gc_trigger_workspace", _sz, _i)
+_sig("gc_trigger_times", _i, _p, _i, _i, _i, _p, _i64, _i, _i, _p, _p, _p, _p, _sz, _p)
 _sig("gc_chunk_grads_workspace", _sz, _i, _i, _i, _i)
 _sig("gc_chunk_grads", _i, _p, _i, _p, _p, _i, _i, _i, _i, _p, _p, _p, _sz, _p)
 _sig("gc_coeff_workspace", _sz, _i, _i, _i, _i, _i)
@@ -157,6 +160,44 @@ def gc_make_assignment(N: int, m: int, delta: int, kind: int = GC_CYCLIC, explic
     _check(lib.gc_make_assignment(N, m, delta, kind, None if ex is None else ex.ctypes.data,
                                   A.ctypes.data, order.ctypes.data, O.ctypes.data))
     return A, order, O
+
+
+def gc_chunk_ordering(A):
+    """Host-only Algorithm 2: A (N x N, every row and column sum delta) ->
+    (order m x delta int32, O N x m uint8) with every row sum of O equal to
+    delta (delta + 1) / 2."""
+    A = np.ascontiguousarray(np.asarray(A) != 0, dtype=np.uint8)
+    N, m = A.shape
+    delta = int(A[0].sum()) if N else 0
+    order = np.zeros((m, max(delta, 1)), dtype=np.int32)
+    O = np.zeros((N, m), dtype=np.uint8)
+    _check(lib.gc_chunk_ordering(A.ctypes.data, N, m, delta, order.ctypes.data, O.ctypes.data))
+    return order, O
+
+
+def gc_trigger_times(order, N: int, m: int, delta: int, tau, ell: int, theta: int = 0, T=True,
+                     psi=True, T_full=True, ws: Workspace | None = None):
+    """Completion times and the encode-and-transmit trigger for nsim simulated
+    realizations (tau: nsim x m float64 on the device, +inf = failed worker).
+    Returns dict T (nsim float64), psi (nsim x m int32), T_full (nsim float64);
+    pass a tensor to write into it or False to skip an output."""
+    nsim = tau.shape[0]
+    dev = tau.device
+
+    def out(x, shape, dt):
+        if x is True:
+            return torch.empty(shape, dtype=dt, device=dev)
+        return x if isinstance(x, torch.Tensor) else None
+    T = out(T, (nsim,), torch.float64)
+    psi = out(psi, (nsim, m), torch.int32)
+    T_full = out(T_full, (nsim,), torch.float64)
+    ws, (wp, wn) = _ws(ws, lib.gc_trigger_workspace(N), dev)
+    _check(lib.gc_trigger_times(
+        _dev(order, torch.int32, "order", (m, delta)), N, m, delta,
+        _dev(tau, torch.float64, "tau", (nsim, m)), nsim, ell, theta,
+        _dev(T, torch.float64, "T", (nsim,)), _dev(psi, torch.int32, "psi", (nsim, m)),
+        _dev(T_full, torch.float64, "T_full", (nsim,)), wp, wn, _stream()))
+    return {"T": T, "psi": psi, "T_full": T_full}
 
 
 # ---------------------------------------------------------------- chunk gradients

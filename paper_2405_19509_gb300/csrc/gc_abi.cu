@@ -110,6 +110,33 @@ int gc_inject_stall(int kernels) {
   return GC_OK;
 }
 
+size_t gc_trigger_workspace(int N) {
+  if (N < 1) return 0;
+  Carve c(nullptr);
+  carve_holders(c, N);
+  return c.bytes();
+}
+
+int gc_trigger_times(const int32_t* order, int N, int m, int delta, const double* tau, int64_t nsim,
+                     int ell, int theta, double* T, int32_t* psi, double* T_full, void* ws,
+                     size_t ws_bytes, void* stream) {
+  if (N < 1 || m < 1 || delta < 1 || nsim < 0) return fail(GC_ERR_SHAPE, "N, m, delta >= 1, nsim >= 0");
+  if (ell < 1 || ell > GC_MAX_ELL) return fail(GC_ERR_UNSUPPORTED, "ell=%d outside [1, %d]", ell, GC_MAX_ELL);
+  if (delta > GC_MAX_DELTA) return fail(GC_ERR_UNSUPPORTED, "delta=%d exceeds %d", delta, GC_MAX_DELTA);
+  if (theta < 0) return fail(GC_ERR_ARG, "theta=%d must be >= 0", theta);
+  if ((long long)N * ell > kTriggerMaxKeys)
+    return fail(GC_ERR_UNSUPPORTED, "N*ell=%lld exceeds %d", (long long)N * ell, kTriggerMaxKeys);
+  if (m > 32767) return fail(GC_ERR_UNSUPPORTED, "m=%d exceeds 32767", m);
+  if (nsim == 0) return GC_OK;
+  if (!order || !tau) return fail(GC_ERR_ARG, "order and tau must be non-NULL");
+  if (!ws || ws_bytes < gc_trigger_workspace(N)) return fail(GC_ERR_WORKSPACE, "workspace too small");
+  cudaStream_t s = as_stream(stream);
+  Carve c(ws);
+  Holders h = carve_holders(c, N);
+  launch_holders(order, N, m, delta, h, status_of(ws), s);
+  return launch_trigger(order, h, N, m, delta, tau, nsim, ell, theta, T, psi, T_full, s);
+}
+
 int gc_set_wait_limit(int64_t cycles) {
   if (cycles < 0) return fail(GC_ERR_ARG, "cycles=%lld must be >= 0", (long long)cycles);
   g_wait_limit.store(cycles, std::memory_order_relaxed);

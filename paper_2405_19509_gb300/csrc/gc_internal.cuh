@@ -70,6 +70,12 @@ Holders carve_holders(Carve& c, int N);
 void launch_holders(const int32_t* order, int N, int m, int delta, Holders h, uint32_t* status,
                     cudaStream_t s);
 
+// ---- completion times and trigger (k_trigger.cu) --------------------------
+constexpr int kTriggerMaxKeys = 2048;  // N * ell per realization
+int launch_trigger(const int32_t* order, Holders h, int N, int m, int delta, const double* tau,
+                   long long nsim, int ell, int theta, double* T, int32_t* psi, double* TF,
+                   cudaStream_t s);
+
 // ---- Algorithm 1 batched (k_solve.cu) -----------------------------------
 struct SolveOut {
   double* E;          // npat x m x delta x ell (nullable)

@@ -1,0 +1,177 @@
+// Completion times and the encode-and-transmit trigger (Sec. II-A and
+// Sec. IV), batched over simulated realizations of the cluster.
+//
+// Realization r gives every worker a time per chunk tau[r][j] (+inf for a
+// failed worker).  W_j finishes the chunk in its slot p (1-based) at p *
+// tau_j, so chunk D_i has been processed n_i(T) = #{holders j : O_ij tau_j
+// <= T} times by time T, and the PS's error estimate (eq. (7) and the
+// sentence after it) is est(T) = sum_i max(0, ell - n_i(T)).  With t_i^(k)
+// the k-th smallest completion time of D_i, est(T) = #{(i, k <= ell) :
+// t_i^(k) > T}; the first time the estimate reaches theta or less is
+// therefore the (N ell - theta)-th smallest of the N ell values t_i^(k).
+// theta = 0 gives the time at which every chunk has been processed ell
+// times, i.e. exact recovery becomes possible.  The same time counting a
+// copy only when its worker has finished all of its chunks (at delta_j
+// tau_j) is the completion time of the original protocol (Sec. IV).
+//
+// GB300 design: one warp per realization.  Lanes take chunks, gather their
+// holders' completion times from the holder table and keep the ell
+// smallest in registers; the N ell values go to shared memory as 64-bit
+// keys (the bit patterns of non-negative doubles order like the values),
+// and a most-significant-digit radix select (4-bit digits, per-lane packed
+// counters summed with warp reductions) finds the order statistic without
+// sorting.  All arithmetic is the same double multiply the definition uses,
+// so times and psi are bit-exact.
+#include <math.h>
+
+#include <algorithm>
+
+#include "gc_internal.cuh"
+
+namespace gc {
+namespace {
+
+constexpr int kWarpsPerBlock = 4;
+
+// k-th smallest (1-based, 1 <= k <= n) of n keys in shared memory, by warp.
+__device__ unsigned long long warp_select(const unsigned long long* keys, int n, int k, int lane) {
+  unsigned long long prefix = 0, mask = 0;
+  for (int shift = 60; shift >= 0; shift -= 4) {
+    unsigned long long lo = 0, hi = 0;  // 8-bit counters for digits 0..7 and 8..15
+    for (int t = lane; t < n; t += 32) {
+      const unsigned long long key = keys[t];
+      if ((key & mask) == prefix) {
+        const int dg = (int)((key >> shift) & 15u);
+        if (dg < 8) lo += 1ull << (8 * dg);
+        else hi += 1ull << (8 * (dg - 8));
+      }
+    }
+    int cum = 0, digit = 15;
+    for (int dg = 0; dg < 16; ++dg) {
+      const unsigned c = (unsigned)(((dg < 8 ? lo : hi) >> (8 * (dg & 7))) & 255u);
+      const int tot = (int)__reduce_add_sync(0xffffffffu, c);
+      if (cum + tot >= k) {
+        digit = dg;
+        break;
+      }
+      cum += tot;
+    }
+    k -= cum;
+    prefix |= (unsigned long long)digit << shift;
+    mask |= 15ull << shift;
+  }
+  return prefix;
+}
+
+template <int ELL>
+__device__ __forceinline__ void insert_smallest(double (&b)[ELL], double v) {
+  if (!(v < b[ELL - 1])) return;
+  int q = ELL - 1;
+  while (q > 0 && b[q - 1] > v) {
+    b[q] = b[q - 1];
+    --q;
+  }
+  b[q] = v;
+}
+
+template <int ELL>
+__global__ void __launch_bounds__(32 * kWarpsPerBlock)
+    k_trigger(const int32_t* __restrict__ order, Holders h, int N, int m, int delta,
+              const double* __restrict__ tau, long long nsim, int theta, double* __restrict__ T_out,
+              int32_t* __restrict__ psi_out, double* __restrict__ Tfull_out) {
+  extern __shared__ unsigned long long s_dyn[];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  // per block: delta_j of every worker, then per warp 2 N ELL keys
+  int8_t* s_dj = reinterpret_cast<int8_t*>(s_dyn);
+  const size_t dj_words = ((size_t)m + 7) / 8;
+  unsigned long long* keys = s_dyn + dj_words + (size_t)warp * 2 * N * ELL;
+  unsigned long long* keysF = keys + (size_t)N * ELL;
+  for (int j = threadIdx.x; j < m; j += blockDim.x) {
+    int c = 0;
+    for (int p = 0; p < delta; ++p) c += order[(size_t)j * delta + p] >= 0;
+    s_dj[j] = (int8_t)c;
+  }
+  __syncthreads();
+  const int n = N * ELL;
+  const int kth = n - theta;
+  for (long long r = (long long)blockIdx.x * kWarpsPerBlock + warp; r < nsim;
+       r += (long long)gridDim.x * kWarpsPerBlock) {
+    const double* tr = tau + r * m;
+    for (int i = lane; i < N; i += 32) {
+      double b[ELL], bf[ELL];
+#pragma unroll
+      for (int k = 0; k < ELL; ++k) b[k] = bf[k] = INFINITY;
+      const int cnt = h.cnt[i];
+      for (int q = 0; q < cnt; ++q) {
+        const int j = h.w[(size_t)i * GC_MAX_REPL + q];
+        const int p = h.p[(size_t)i * GC_MAX_REPL + q];
+        const double tj = tr[j];
+        if (isfinite(tj)) {
+          insert_smallest<ELL>(b, (double)(p + 1) * tj);
+          insert_smallest<ELL>(bf, (double)s_dj[j] * tj);
+        }
+      }
+#pragma unroll
+      for (int k = 0; k < ELL; ++k) {
+        keys[(size_t)i * ELL + k] = (unsigned long long)__double_as_longlong(b[k]);
+        keysF[(size_t)i * ELL + k] = (unsigned long long)__double_as_longlong(bf[k]);
+      }
+    }
+    __syncwarp();
+    double T = 0.0, TF = 0.0;
+    if (kth >= 1) {
+      T = __longlong_as_double((long long)warp_select(keys, n, kth, lane));
+      TF = __longlong_as_double((long long)warp_select(keysF, n, kth, lane));
+    }
+    if (lane == 0) {
+      if (T_out) T_out[r] = T;
+      if (Tfull_out) Tfull_out[r] = TF;
+    }
+    if (psi_out)
+      for (int j = lane; j < m; j += 32) {
+        const double tj = tr[j];
+        int c = 0;
+        if (isfinite(tj))
+          for (int p = 1; p <= s_dj[j]; ++p) c += (double)p * tj <= T;
+        psi_out[r * m + j] = c;
+      }
+    __syncwarp();
+  }
+}
+
+template <int ELL>
+int launch_one(const int32_t* order, Holders h, int N, int m, int delta, const double* tau,
+               long long nsim, int theta, double* T, int32_t* psi, double* TF, cudaStream_t s) {
+  const size_t smem = (((size_t)m + 7) / 8 + (size_t)kWarpsPerBlock * 2 * N * ELL) * 8;
+  if (smem > 48 * 1024) {
+    cudaError_t e = cudaFuncSetAttribute(k_trigger<ELL>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)smem);
+    if (e != cudaSuccess) return cuda_check(e, "cudaFuncSetAttribute(k_trigger)");
+  }
+  const long long blocks_needed = (nsim + kWarpsPerBlock - 1) / kWarpsPerBlock;
+  const int blocks = (int)std::min<long long>(blocks_needed, (long long)device_sm_count() * 16);
+  k_trigger<ELL><<<blocks, 32 * kWarpsPerBlock, smem, s>>>(order, h, N, m, delta, tau, nsim, theta,
+                                                           T, psi, TF);
+  count_launches(1);
+  return cuda_check(cudaGetLastError(), "k_trigger");
+}
+
+}  // namespace
+
+int launch_trigger(const int32_t* order, Holders h, int N, int m, int delta, const double* tau,
+                   long long nsim, int ell, int theta, double* T, int32_t* psi, double* TF,
+                   cudaStream_t s) {
+  switch (ell) {
+    case 1: return launch_one<1>(order, h, N, m, delta, tau, nsim, theta, T, psi, TF, s);
+    case 2: return launch_one<2>(order, h, N, m, delta, tau, nsim, theta, T, psi, TF, s);
+    case 3: return launch_one<3>(order, h, N, m, delta, tau, nsim, theta, T, psi, TF, s);
+    case 4: return launch_one<4>(order, h, N, m, delta, tau, nsim, theta, T, psi, TF, s);
+    case 5: return launch_one<5>(order, h, N, m, delta, tau, nsim, theta, T, psi, TF, s);
+    case 6: return launch_one<6>(order, h, N, m, delta, tau, nsim, theta, T, psi, TF, s);
+    case 7: return launch_one<7>(order, h, N, m, delta, tau, nsim, theta, T, psi, TF, s);
+    case 8: return launch_one<8>(order, h, N, m, delta, tau, nsim, theta, T, psi, TF, s);
+    default: return fail(GC_ERR_UNSUPPORTED, "ell=%d exceeds GC_MAX_ELL", ell);
+  }
+}
+
+}  // namespace gc

@@ -15,4 +15,8 @@ from .gen import (  # noqa: F401
     make_chunk_grads,
     make_patterns,
     all_patterns,
+    random_regular_graph,
+    second_eigenvalue,
+    random_order,
+    make_worker_times,
 )

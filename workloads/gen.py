@@ -16,7 +16,8 @@ import torch
 
 from .configs import Config
 
-_TAG_R, _TAG_WSTAR, _TAG_W, _TAG_X, _TAG_NOISE, _TAG_LABEL, _TAG_PSI, _TAG_G = range(8)
+(_TAG_R, _TAG_WSTAR, _TAG_W, _TAG_X, _TAG_NOISE, _TAG_LABEL, _TAG_PSI, _TAG_G, _TAG_GRAPH,
+ _TAG_ORDER, _TAG_TIMES) = range(11)
 
 
 def _np_rng(*key: int) -> np.random.Generator:
@@ -134,3 +135,77 @@ def make_patterns(cfg: Config, npat: int | None = None, p: float | None = None,
 def all_patterns(m: int, delta: int) -> np.ndarray:
     """Every psi in {0..delta}^m, in lexicographic order (brute force)."""
     return np.array(list(itertools.product(range(delta + 1), repeat=m)), dtype=np.int32)
+
+
+def random_regular_graph(m: int, nu: int, seed: int) -> np.ndarray:
+    """Adjacency matrix (m x m uint8, symmetric, zero diagonal) of a random
+    nu-regular simple graph: the pairing model with pairs drawn among the
+    points that can still be joined (no loop, no repeated edge), restarted
+    when it gets stuck (Steger and Wormald, 1999).  Used as the assignment
+    matrix A of the approximate-GC workloads (Sec. IV: N = m, every row and
+    column sum nu)."""
+    assert (m * nu) % 2 == 0 and nu < m
+    rng = _np_rng(seed, _TAG_GRAPH, m, nu)
+    while True:
+        A = np.zeros((m, m), dtype=np.uint8)
+        pts = list(np.repeat(np.arange(m), nu))
+        stuck = False
+        while pts:
+            n = len(pts)
+            done = False
+            for _ in range(64):
+                a, b = rng.integers(0, n, size=2)
+                u, v = pts[a], pts[b]
+                if a != b and u != v and not A[u, v]:
+                    done = True
+                    break
+            if not done:
+                # exhaustive search for any suitable pair before giving up
+                cand = [(a, b) for a in range(n) for b in range(a + 1, n)
+                        if pts[a] != pts[b] and not A[pts[a], pts[b]]]
+                if not cand:
+                    stuck = True
+                    break
+                a, b = cand[rng.integers(0, len(cand))]
+                u, v = pts[a], pts[b]
+            A[u, v] = A[v, u] = 1
+            for k in sorted((a, b), reverse=True):
+                pts[k] = pts[-1]
+                pts.pop()
+        if not stuck:
+            return A
+
+
+def second_eigenvalue(A: np.ndarray) -> float:
+    """Second-largest absolute eigenvalue of a symmetric adjacency matrix
+    (a nu-regular graph is Ramanujan when it is below 2 sqrt(nu - 1))."""
+    ev = np.sort(np.abs(np.linalg.eigvalsh(A.astype(np.float64))))
+    return float(ev[-2])
+
+
+def random_order(A: np.ndarray, seed: int, index: int = 0) -> np.ndarray:
+    """A uniformly random processing order for assignment A: worker j takes
+    its chunks {i : A_ij != 0} in a random permutation (m x delta int32,
+    -1 padded).  Sec. IV compares the optimal ordering with the best of 100
+    such orderings."""
+    N, m = A.shape
+    delta = int((A != 0).sum(axis=0).max())
+    rng = _np_rng(seed, _TAG_ORDER, index)
+    order = -np.ones((m, delta), dtype=np.int32)
+    for j in range(m):
+        ch = np.flatnonzero(A[:, j])
+        order[j, :len(ch)] = rng.permutation(ch)
+    return order
+
+
+def make_worker_times(m: int, nsim: int, seed: int, alpha: int = 0, shift: float = 0.0):
+    """Per-realization worker speeds for the completion-time simulation of
+    Sec. IV: tau[r, j] = time W_j takes per chunk, i.i.d. shift + Exp(1); in
+    every realization alpha workers chosen uniformly at random have failed
+    (tau = +inf).  Returns float64 nsim x m."""
+    rng = _np_rng(seed, _TAG_TIMES, m, alpha)
+    tau = shift + rng.exponential(1.0, size=(nsim, m))
+    for r in range(nsim):
+        if alpha:
+            tau[r, rng.choice(m, size=alpha, replace=False)] = np.inf
+    return tau
