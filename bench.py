@@ -56,6 +56,10 @@ def parse():
     ap.add_argument("--warmup", type=int, default=20)
     ap.add_argument("--impl", choices=["gc", "reference"], default="gc")
     ap.add_argument("--ell", type=int, default=2)
+    ap.add_argument("--workload", default="logistic",
+                    choices=["logistic", "decode", "sweep", "sgd", "trigger"],
+                    help="logistic: the headline step (default).  The others measure the "
+                         "remaining configurations, one JSON line each (1 GPU)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--min-warm-seconds", type=float, default=1.5,
                     help="keep warming up at least this long (steady clocks, clock samples)")
@@ -482,8 +486,211 @@ def gpu_arm(args, rank, world, local_rank):
         print(json.dumps(line), flush=True)
 
 
+# ------------------------------------------------------------------ other workloads
+def _time_ms(torch, f, reps, warm=2, flush=None):
+    """Mean CUDA-event time of f() (ms); the L2 is flushed before each rep."""
+    for _ in range(warm):
+        f()
+    torch.cuda.synchronize()
+    tot = 0.0
+    for _ in range(reps):
+        if flush is not None:
+            flush.zero_()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        f()
+        e1.record()
+        torch.cuda.synchronize()
+        tot += e0.elapsed_time(e1)
+    return tot / reps
+
+
+def extra_workload(args):
+    """One JSON line for a non-headline configuration (single GPU)."""
+    import torch
+
+    import paper_2405_19509_gb300 as gc
+    from workloads import (get, make_R, make_chunk_grads, make_data, make_patterns,
+                           make_worker_times, random_regular_graph)
+
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    pk, pk_src = peaks()
+    hbm, bf16 = float(pk["hbm_gbs"]), float(pk["bf16_tflops"])
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+    n0 = gc.gc_kernel_launches()
+    ell = args.ell
+    line = {"workload": args.workload, "n_gpus": 1, "data": "synthetic", "dtype": "f32"}
+    if args.workload == "decode":
+        cfg = get("decode")
+        N, m, delta, d, npat = cfg.N, cfg.m, cfg.delta, cfg.d, cfg.npat
+        G = make_chunk_grads(cfg, dev)
+        _, order, _ = gc.gc_make_assignment(N, m, delta)
+        Rd = torch.from_numpy(make_R(cfg, ell)).to(dev)
+        od = torch.from_numpy(order).to(dev)
+        pd = torch.from_numpy(make_patterns(cfg)).to(dev)
+        plan = torch.empty(int(gc.lib.gc_decode_plan_bytes(N, ell, npat)), dtype=torch.uint8, device=dev)
+        Gh = torch.empty(npat, d, device=dev)
+        ce = torch.empty(npat, dtype=torch.float64, device=dev)
+        es = torch.empty_like(ce)
+        wsB, wsC = gc.Workspace(dev), gc.Workspace(dev)
+        t_plan = _time_ms(torch, lambda: gc.gc_decode_plan(Rd, ell, od, N, m, delta, pd, plan=plan,
+                                                           coef_err=ce, est=es, ws=wsB), 5)
+        t_apply = _time_ms(torch, lambda: gc.gc_decode_apply(plan, ell, N, npat, G, Ghat=Gh,
+                                                             grad_mse=False, ws=wsC), 5)
+        gc.gc_status(wsB)
+        gc.gc_status(wsC)
+        L = -(-d // ell)
+        Kp = -(-N * ell // 64) * 64
+        useful = 2.0 * npat * ell * (N * ell) * L
+        issued = 3 * 2.0 * npat * ell * Kp * L
+        line.update({
+            "metric": f"decoded gradients/sec (m=N=256, delta=16, d=2^20, 4096 patterns, l={ell})",
+            "value": npat / ((t_plan + t_apply) / 1e3), "unit": "decoded gradients/s",
+            "ms_plan": t_plan, "ms_apply": t_apply,
+            "roofline": {"kernel": "k_combine_tc", "bound": "tensor", "unit": "TFLOP/s",
+                         "achieved": issued / (t_apply / 1e3) / 1e12, "peak": bf16,
+                         "frac": issued / (t_apply / 1e3) / 1e12 / bf16,
+                         "useful_tflops": useful / (t_apply / 1e3) / 1e12,
+                         "note": "issued = three bf16 MMAs per K step (hi/lo split) over the padded K; "
+                                 "timed gc_decode_apply includes the operand split",
+                         "peak_source": f"{pk_src} bf16_tflops"},
+            "config": {"workload": f"decode m=N=256 delta=16 d=2^20 npat=4096 ell={ell}",
+                       "l2": "inputs larger than L2 (G 1.07 GB, Ghat 17.2 GB)"}})
+    elif args.workload == "sweep":
+        cfg = get("mse_sweep")
+        N, m, delta, d, npat = cfg.N, cfg.m, cfg.delta, cfg.d, cfg.npat
+        data = make_data(cfg, dev)
+        G = torch.empty(N, d, device=dev)
+        wsA = gc.Workspace(dev)
+        t_cg = _time_ms(torch, lambda: gc.gc_chunk_grads(data["X"], data["y"], data["w"], N, cfg.n_c,
+                                                         gc.GC_LSQ, G=G, ws=wsA), 5)
+        del data
+        torch.cuda.empty_cache()
+        _, order, _ = gc.gc_make_assignment(N, m, delta)
+        Rd = torch.from_numpy(make_R(cfg, ell)).to(dev)
+        od = torch.from_numpy(order).to(dev)
+        wsM = gc.Workspace(dev)
+        res = {}
+        t_mse_tot = 0.0
+        for p in (0.3, 0.5, 0.7):
+            pd = torch.from_numpy(make_patterns(cfg, p=p)).to(dev)
+            t = _time_ms(torch, lambda: gc.gc_mse(Rd, ell, od, N, m, delta, pd, G, ws=wsM), 3)
+            out = gc.gc_mse(Rd, ell, od, N, m, delta, pd, G, ws=wsM)
+            gc.gc_status(wsM)
+            res[str(p)] = {"ms": t, "mean_grad_mse": float(out["grad_mse"].mean()),
+                           "mean_coef_err": float(out["coef_err"].mean()),
+                           "mean_est": float(out["est"].mean())}
+            t_mse_tot += t
+        L = -(-d // ell)
+        useful = 2.0 * npat * ell * (N * ell) * L
+        Kp = -(-N * ell // 64) * 64
+        issued = 3 * 2.0 * npat * ell * Kp * L
+        t_mse = t_mse_tot / 3
+        line.update({
+            "metric": f"patterns/sec (MSE only, m=N=64, delta=8, d=65536, 10^5 patterns, l={ell})",
+            "value": npat / (t_mse / 1e3), "unit": "patterns/s",
+            "chunk_grads": {"ms": t_cg, "GB/s": cfg.Ntil * d * 2 / (t_cg / 1e3) / 1e9,
+                            "frac_of_hbm": cfg.Ntil * d * 2 / (t_cg / 1e3) / 1e9 / hbm,
+                            "TFLOP/s": 4.0 * cfg.Ntil * d / (t_cg / 1e3) / 1e12},
+            "per_p": res,
+            "roofline": {"kernel": "k_combine_tc (MSE only)", "bound": "tensor", "unit": "TFLOP/s",
+                         "achieved": issued / (t_mse / 1e3) / 1e12, "peak": bf16,
+                         "frac": issued / (t_mse / 1e3) / 1e12 / bf16,
+                         "useful_tflops": useful / (t_mse / 1e3) / 1e12,
+                         "note": "timed gc_mse includes Algorithm 1 for the 10^5 patterns",
+                         "peak_source": f"{pk_src} bf16_tflops"},
+            "dtype": "bf16 X, f32 otherwise",
+            "config": {"workload": f"sweep m=N=64 delta=8 d=65536 n_c=1024 bf16 npat=10^5 ell={ell}",
+                       "l2": "inputs larger than L2 (X 8.6 GB)"}})
+    elif args.workload == "sgd":
+        cfg = get("sgd")
+        N, m, delta, d = cfg.N, cfg.m, cfg.delta, cfg.d
+        data = make_data(cfg, dev, w_which="zero")
+        X, y, w = data["X"], data["y"], data["w"].clone()
+        _, order, _ = gc.gc_make_assignment(N, m, delta)
+        Rd = torch.from_numpy(make_R(cfg, ell)).to(dev)
+        od = torch.from_numpy(order).to(dev)
+        psi = torch.from_numpy(np.stack([make_patterns(cfg, npat=1, stream=t)[0]
+                                         for t in range(cfg.iters)])).to(dev)
+        G = torch.empty(N, d, device=dev)
+        loss = torch.zeros(cfg.iters, dtype=torch.float64, device=dev)
+        ws = gc.Workspace(dev)
+        L = -(-d // ell)
+        T = torch.empty(1, m, L, device=dev)
+        gh = torch.empty(1, d, device=dev)
+
+        def run():
+            for it in range(cfg.iters):
+                gc.gc_chunk_grads(X, y, w, N, cfg.n_c, gc.GC_LOGISTIC, G=G, loss_out=loss[it:it + 1], ws=ws)
+                gc.gc_encode(Rd, ell, od, N, m, delta, psi[it:it + 1], G, T=T, ws=ws)
+                gc.gc_decode_tx(Rd, ell, m, T, d, ghat=gh)
+                gc.gc_sgd_step(w, gh[0], cfg.lr, cfg.Ntil)
+        w0 = w.clone()
+        t = _time_ms(torch, run, 2, warm=1)
+        w.copy_(w0)
+        t_cg = _time_ms(torch, lambda: gc.gc_chunk_grads(X, y, w, N, cfg.n_c, gc.GC_LOGISTIC, G=G, ws=ws), 5)
+        gc.gc_status(ws)
+        line.update({
+            "metric": f"coded SGD iterations/sec (m=N=128, delta=6, d=8192, n_c=2048, l={ell})",
+            "value": cfg.iters / (t / 1e3), "unit": "iterations/s", "ms_64_iterations": t,
+            "roofline": {"kernel": "k_chunkgrad", "bound": "hbm", "unit": "GB/s",
+                         "achieved": cfg.Ntil * d * 4 / (t_cg / 1e3) / 1e9, "peak": hbm,
+                         "frac": cfg.Ntil * d * 4 / (t_cg / 1e3) / 1e9 / hbm,
+                         "ms_chunk_grads": t_cg, "peak_source": f"{pk_src} hbm_gbs"},
+            "config": {"workload": f"sgd m=N=128 delta=6 d=8192 n_c=2048 64 iterations ell={ell}",
+                       "l2": "inputs larger than L2 (X 8.6 GB)"}})
+    elif args.workload == "trigger":
+        nsim = 100_000
+        rows = {}
+        for name, N, nu, alpha_of in (("cyclic N=m=200 delta=8", 200, 8, lambda l: 8 - l),
+                                      ("random 8-regular m=200 (Alg. 2 order)", 200, 8, lambda l: 7)):
+            if name.startswith("cyclic"):
+                _, order, _ = gc.gc_make_assignment(N, N, nu)
+                t_alg2 = None
+            else:
+                A = random_regular_graph(N, nu, 1)
+                t0 = time.perf_counter()
+                order, _ = gc.gc_chunk_ordering(A)
+                t_alg2 = (time.perf_counter() - t0) * 1e3
+            od = torch.from_numpy(order).to(dev)
+            ws = gc.Workspace(dev)
+            for l in (1, 2, 3, 4):
+                tau = torch.from_numpy(make_worker_times(N, nsim, 20 + l, alpha=alpha_of(l))).to(dev)
+                T = torch.empty(nsim, dtype=torch.float64, device=dev)
+                TF = torch.empty_like(T)
+                psi = torch.empty(nsim, N, dtype=torch.int32, device=dev)
+                t = _time_ms(torch, lambda: gc.gc_trigger_times(od, N, N, nu, tau, l, 0, T=T, psi=psi,
+                                                                T_full=TF, ws=ws), 5, flush=flush)
+                fin = torch.isfinite(T) & torch.isfinite(TF)
+                rows[f"{name}, l={l}"] = {
+                    "ms": t, "realizations/s": nsim / (t / 1e3),
+                    "mean_T": float(T[fin].mean()), "mean_T_full": float(TF[fin].mean()),
+                    "mean_ratio_T_full_over_T": float((TF[fin] / T[fin]).mean()),
+                    "alg2_host_ms": t_alg2}
+        r0 = rows["cyclic N=m=200 delta=8, l=2"]
+        bytes_r = 200 * 8 + 200 * 4 + 16  # tau read, psi written, two times written
+        line.update({
+            "metric": "simulated realizations/sec (completion time + trigger + psi, N=m=200, delta=8, l=2)",
+            "value": r0["realizations/s"], "unit": "realizations/s", "per_case": rows,
+            "roofline": {"kernel": "k_trigger", "bound": "hbm", "unit": "GB/s",
+                         "achieved": bytes_r * r0["realizations/s"] / 1e9, "peak": hbm,
+                         "frac": bytes_r * r0["realizations/s"] / 1e9 / hbm,
+                         "note": "latency/ALU-bound selection; bytes = tau read + outputs",
+                         "peak_source": f"{pk_src} hbm_gbs"},
+            "dtype": "f64",
+            "config": {"workload": "trigger cyclic N=m=200 delta=8 alpha=delta-l, 10^5 realizations; "
+                                   "and 8-regular m=200 alpha=7",
+                       "l2": "L2 flushed before each timed call (tau 160 MB)"}})
+    line["gpu_launches_total"] = int(gc.gc_kernel_launches() - n0)
+    print(json.dumps(line), flush=True)
+
+
 def main():
     args = parse()
+    if args.workload != "logistic" and args.impl == "gc":
+        extra_workload(args)
+        return
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
     local_rank = int(os.environ.get("LOCAL_RANK", "0"))
