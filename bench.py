@@ -57,7 +57,7 @@ def parse():
     ap.add_argument("--impl", choices=["gc", "reference"], default="gc")
     ap.add_argument("--ell", type=int, default=2)
     ap.add_argument("--workload", default="logistic",
-                    choices=["logistic", "decode", "sweep", "sgd", "trigger"],
+                    choices=["logistic", "decode", "sweep", "sgd", "trigger", "batched"],
                     help="logistic: the headline step (default).  The others measure the "
                          "remaining configurations, one JSON line each (1 GPU)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
@@ -639,6 +639,37 @@ def extra_workload(args):
                          "frac": cfg.Ntil * d * 4 / (t_cg / 1e3) / 1e9 / hbm,
                          "ms_chunk_grads": t_cg, "peak_source": f"{pk_src} hbm_gbs"},
             "config": {"workload": f"sgd m=N=128 delta=6 d=8192 n_c=2048 64 iterations ell={ell}",
+                       "l2": "inputs larger than L2 (X 8.6 GB)"}})
+    elif args.workload == "batched":
+        cfg = get("mse_sweep")
+        N, d, n_c = cfg.N, cfg.d, cfg.n_c
+        data = make_data(cfg, dev)
+        X, y = data["X"], data["y"]
+        res = {}
+        for n_w in (128, 256):
+            W = torch.randn(n_w, d, generator=torch.Generator(device=dev).manual_seed(n_w),
+                            device=dev) / d ** 0.5
+            G = torch.empty(n_w, N, d, device=dev)
+            ws = gc.Workspace(dev)
+            t = _time_ms(torch, lambda: gc.gc_chunk_grads_batched(X, y, W, N, n_c, gc.GC_LSQ, G=G, ws=ws), 3)
+            gc.gc_status(ws)
+            useful = 4.0 * cfg.Ntil * d * n_w
+            res[n_w] = {"ms": t, "useful_tflops": useful / (t / 1e3) / 1e12,
+                        "issued_tflops": 2 * useful / (t / 1e3) / 1e12,
+                        "X_read_GBps": 2 * cfg.Ntil * d * 2 / (t / 1e3) / 1e9}
+            del G
+            torch.cuda.empty_cache()
+        r = res[256]
+        line.update({
+            "metric": "chunk-gradient TFLOP/s, n_w parameter vectors at once (m=N=64, d=65536, n_c=1024, bf16 X)",
+            "value": r["useful_tflops"], "unit": "TFLOP/s (useful)", "per_n_w": res,
+            "roofline": {"kernel": "k_gemm_w (two GEMMs)", "bound": "tensor", "unit": "TFLOP/s",
+                         "achieved": r["issued_tflops"], "peak": bf16, "frac": r["issued_tflops"] / bf16,
+                         "note": "issued = two bf16 MMAs per K step (hi/lo parts of W, R); X is read "
+                                 "twice (once per GEMM)",
+                         "peak_source": f"{pk_src} bf16_tflops"},
+            "dtype": "bf16 X, f32 accumulate",
+            "config": {"workload": "batched chunk gradients N=64 n_c=1024 d=65536 bf16, n_w=128 and 256, lsq",
                        "l2": "inputs larger than L2 (X 8.6 GB)"}})
     elif args.workload == "trigger":
         nsim = 100_000

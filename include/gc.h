@@ -146,6 +146,25 @@ int gc_make_assignment(int N, int m, int delta, int kind, const int32_t* explici
  */
 int gc_chunk_ordering(const uint8_t* A_h, int N, int m, int delta, int32_t* order_h, uint8_t* O_h);
 
+/* ---- chunk gradients for several parameter vectors (tensor cores) -------
+ * For n_w parameter vectors at once (replicas, a learning-rate sweep):
+ *   G[w][i] = X_i^T (f(X_i w_w) - y01_i)       (Sec. I, one per w_w)
+ * computed as two tcgen05 GEMMs, Z = X W^T (K = d) with the residual
+ * R = f(Z) - y01 formed in the epilogue, then G_i = X_i^T R_i (K = n_c).
+ * W and R enter the MMAs as bf16 hi + lo parts (fp32 accumulation), X as
+ * bf16 (exact).  f and y01 as in gc_chunk_grads.
+ *   X    device N~ x d bf16, row-major, 16-byte aligned.
+ *   y    device N~ fp32.   W  device n_w x d fp32 (row w = w_w).
+ *   G    device output n_w x N x d fp32 (G[w] is the N x d chunk-gradient
+ *        matrix of w_w, the layout the decode entry points take).
+ *   Limits: 32 <= n_w <= 256, n_w % 32 == 0; d % 128 == 0; n_c % 64 == 0;
+ *   N * n_c % 128 == 0.  No loss output.
+ * Workspace: gc_chunk_grads_batched_workspace(N, n_c, d, n_w) bytes.
+ */
+size_t gc_chunk_grads_batched_workspace(int N, int n_c, int d, int n_w);
+int gc_chunk_grads_batched(const void* X, const float* y, const float* W, int N, int n_c, int d,
+                           int n_w, int loss, float* G, void* ws, size_t ws_bytes, void* stream);
+
 /* ---- completion times and the encode-and-transmit trigger (Sec. IV) ----
  * Batched simulation of the cluster: realization r gives every worker a
  * time per chunk tau[r][j] (> 0, +inf for a failed worker); W_j finishes

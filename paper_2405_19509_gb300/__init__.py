@@ -38,6 +38,7 @@ from .binding import (  # noqa: F401
     gc_set_wait_limit,
     gc_chunk_ordering,
     gc_trigger_times,
+    gc_chunk_grads_batched,
     gc_inject_stall,
     GC_STALL_CHUNK_GRADS,
     GC_STALL_COMBINE,

@@ -46,6 +46,8 @@ _sig("gc_status", _i, _p, _p)
 _sig("gc_make_assignment", _i, _i, _i, _i, _i, _p, _p, _p, _p)
 _sig("gc_chunk_ordering", _i, _p, _i, _i, _i, _p, _p)
 _sig("gc_trigger_workspace", _sz, _i)
+_sig("gc_chunk_grads_batched_workspace", _sz, _i, _i, _i, _i)
+_sig("gc_chunk_grads_batched", _i, _p, _p, _p, _i, _i, _i, _i, _i, _p, _p, _sz, _p)
 _sig("gc_trigger_times", _i, _p, _i, _i, _i, _p, _i64, _i, _i, _p, _p, _p, _p, _sz, _p)
 _sig("gc_chunk_grads_workspace", _sz, _i, _i, _i, _i)
 _sig("gc_chunk_grads", _i, _p, _i, _p, _p, _i, _i, _i, _i, _p, _p, _p, _sz, _p)
@@ -198,6 +200,23 @@ def gc_trigger_times(order, N: int, m: int, delta: int, tau, ell: int, theta: in
         _dev(T, torch.float64, "T", (nsim,)), _dev(psi, torch.int32, "psi", (nsim, m)),
         _dev(T_full, torch.float64, "T_full", (nsim,)), wp, wn, _stream()))
     return {"T": T, "psi": psi, "T_full": T_full}
+
+
+def gc_chunk_grads_batched(X, y, W, N: int, n_c: int, loss: int, G=None,
+                           ws: Workspace | None = None):
+    """Chunk gradients for n_w parameter vectors (rows of W) on the tensor
+    cores: G (n_w x N x d float32).  X must be bfloat16."""
+    n_w, d = W.shape
+    if X.dtype != torch.bfloat16:
+        raise TypeError("X must be bfloat16")
+    if G is None:
+        G = torch.empty(n_w, N, d, dtype=torch.float32, device=X.device)
+    ws, (wp, wn) = _ws(ws, lib.gc_chunk_grads_batched_workspace(N, n_c, d, n_w), X.device)
+    _check(lib.gc_chunk_grads_batched(
+        _dev(X, torch.bfloat16, "X", (N * n_c, d)), _dev(y, torch.float32, "y", (N * n_c,)),
+        _dev(W, torch.float32, "W", (n_w, d)), N, n_c, d, n_w, loss,
+        _dev(G, torch.float32, "G", (n_w, N, d)), wp, wn, _stream()))
+    return G
 
 
 # ---------------------------------------------------------------- chunk gradients

@@ -110,6 +110,30 @@ int gc_inject_stall(int kernels) {
   return GC_OK;
 }
 
+size_t gc_chunk_grads_batched_workspace(int N, int n_c, int d, int n_w) {
+  if (N < 1 || n_c < 1 || d < 1 || n_w < 1) return 0;
+  return kHeaderBytes + gemmw_ws_bytes(N, n_c, d, n_w);
+}
+
+int gc_chunk_grads_batched(const void* X, const float* y, const float* W, int N, int n_c, int d,
+                           int n_w, int loss, float* G, void* ws, size_t ws_bytes, void* stream) {
+  if (N < 1 || n_c < 1 || d < 1 || n_w < 1) return fail(GC_ERR_SHAPE, "N, n_c, d, n_w must be >= 1");
+  if (n_w % 32 != 0 || n_w > 256)
+    return fail(GC_ERR_UNSUPPORTED, "n_w=%d must be a multiple of 32 in [32, 256]", n_w);
+  if (d % 128 != 0) return fail(GC_ERR_UNSUPPORTED, "d=%d must be a multiple of 128", d);
+  if (n_c % 64 != 0) return fail(GC_ERR_UNSUPPORTED, "n_c=%d must be a multiple of 64", n_c);
+  if (((long long)N * n_c) % 128 != 0) return fail(GC_ERR_UNSUPPORTED, "N*n_c must be a multiple of 128");
+  if ((long long)N * n_c > (1LL << 31) - 1) return fail(GC_ERR_UNSUPPORTED, "N*n_c too large");
+  if (loss != GC_LSQ && loss != GC_LOGISTIC) return fail(GC_ERR_ARG, "unknown loss %d", loss);
+  if (!X || !y || !W || !G) return fail(GC_ERR_ARG, "X, y, W and G must be non-NULL");
+  if (reinterpret_cast<uintptr_t>(X) % 16 != 0) return fail(GC_ERR_ARG, "X must be 16-byte aligned");
+  if (!ws || ws_bytes < gc_chunk_grads_batched_workspace(N, n_c, d, n_w))
+    return fail(GC_ERR_WORKSPACE, "workspace too small");
+  Carve c(ws);
+  return launch_chunkgrad_batched(X, y, W, N, n_c, d, n_w, loss, G, c, status_of(ws),
+                                  as_stream(stream));
+}
+
 size_t gc_trigger_workspace(int N) {
   if (N < 1) return 0;
   Carve c(nullptr);

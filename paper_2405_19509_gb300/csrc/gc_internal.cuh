@@ -70,6 +70,12 @@ Holders carve_holders(Carve& c, int N);
 void launch_holders(const int32_t* order, int N, int m, int delta, Holders h, uint32_t* status,
                     cudaStream_t s);
 
+// ---- batched chunk gradients on the tensor cores (k_gemm_w.cu) -----------
+size_t gemmw_ws_bytes(int N, int n_c, int d, int n_w);
+int launch_chunkgrad_batched(const void* X, const float* y, const float* W, int N, int n_c, int d,
+                             int n_w, int loss, float* G, Carve& ws, uint32_t* status,
+                             cudaStream_t s);
+
 // ---- completion times and trigger (k_trigger.cu) --------------------------
 constexpr int kTriggerMaxKeys = 2048;  // N * ell per realization
 int launch_trigger(const int32_t* order, Holders h, int N, int m, int delta, const double* tau,

@@ -134,3 +134,15 @@ def test_wait_limit_knob_validation():
     assert gc.lib.gc_set_wait_limit(0) == 0
     assert gc.lib.gc_inject_stall(4) == -1
     assert gc.lib.gc_inject_stall(0) == 0
+
+
+def test_batched_chunk_grads_validation():
+    gc = _lib()
+    L = gc.lib
+    nul = None
+    # unsupported shapes are rejected on the host before anything runs
+    assert L.gc_chunk_grads_batched(nul, nul, nul, 2, 128, 256, 48, 0, nul, nul, 0, nul) == -3
+    assert L.gc_chunk_grads_batched(nul, nul, nul, 2, 128, 200, 32, 0, nul, nul, 0, nul) == -3
+    assert L.gc_chunk_grads_batched(nul, nul, nul, 2, 100, 256, 32, 0, nul, nul, 0, nul) == -3
+    assert L.gc_chunk_grads_batched(nul, nul, nul, 2, 128, 256, 32, 0, nul, nul, 0, nul) == -1
+    assert L.gc_chunk_grads_batched_workspace(2, 128, 256, 32) > 256
