@@ -97,13 +97,25 @@ struct Vec<float> {
     const float4 v = *reinterpret_cast<const float4*>(p);
     o[0] = v.x; o[1] = v.y; o[2] = v.z; o[3] = v.w;
   }
+  __device__ static __forceinline__ uint4 load_raw(const float* p) {
+    return *reinterpret_cast<const uint4*>(p);
+  }
+  __device__ static __forceinline__ void unpack(const uint4& u, float (&o)[4]) {
+    o[0] = __uint_as_float(u.x); o[1] = __uint_as_float(u.y);
+    o[2] = __uint_as_float(u.z); o[3] = __uint_as_float(u.w);
+  }
   __device__ static __forceinline__ float scalar(const float* p) { return *p; }
 };
 template <>
 struct Vec<__nv_bfloat16> {
   static constexpr int V = 8;
   __device__ static __forceinline__ void load(const __nv_bfloat16* p, float (&o)[8]) {
-    const uint4 u = *reinterpret_cast<const uint4*>(p);
+    unpack(load_raw(p), o);
+  }
+  __device__ static __forceinline__ uint4 load_raw(const __nv_bfloat16* p) {
+    return *reinterpret_cast<const uint4*>(p);
+  }
+  __device__ static __forceinline__ void unpack(const uint4& u, float (&o)[8]) {
     const uint32_t w[4] = {u.x, u.y, u.z, u.w};
 #pragma unroll
     for (int k = 0; k < 4; ++k) {
@@ -327,27 +339,46 @@ __global__ void __launch_bounds__(NT + 32, 1) k_chunkgrad(CGArgs a) {
       }
     };
 
-    // Pass 1 of batch n: partial dot products, CTA reduction and (clusters)
-    // the send to every peer.  Returns the CTA sums in every lane.
-    auto pass1 = [&](int n, float (&z)[RBM]) {
-      const int s = n % a.S;
-      bounded_wait(&full[s], (uint32_t)((n / a.S) & 1), abort_flag, a.status, a.spin_limit);
-      const T* st = stages + s * stage_elems;
+    // x vectors of batch n: raw 16-byte words straight from its stage (zero
+    // for rows past RB and vectors past the slice) ...
+    auto wait_stage = [&](int n) {
+      bounded_wait(&full[n % a.S], (uint32_t)((n / a.S) & 1), abort_flag, a.status, a.spin_limit);
+    };
+    auto from_stage = [&](int n) {
+      const T* st = stages + (n % a.S) * stage_elems;
+      return [=](int r, int u) {
+        const int v = tid + u * NT;
+        return (r < a.RB && v < nvs) ? Vec<T>::load_raw(st + (size_t)r * a.ld_s + v * V)
+                                     : make_uint4(0u, 0u, 0u, 0u);
+      };
+    };
+    // ... or copied to registers once (kept from the dot products to pass 2)
+    auto load_x = [&](int n, uint4 (&xr)[RBM][NVT]) {
+      auto src = from_stage(n);
+#pragma unroll
+      for (int r = 0; r < RBM; ++r)
+#pragma unroll
+        for (int u = 0; u < NVT; ++u) xr[r][u] = src(r, u);
+    };
+    // hand stage n back to the producer (every lane of the warp is done reading it)
+    auto release = [&](int n) {
+      __syncwarp();
+      if (lane == 0) mbar_arrive_local(&empty[n % a.S]);
+    };
+    // Dot products of batch n, reduced over the CTA (warp butterfly, then
+    // lane-parallel over (warp, row) pairs) and, with clusters, sent to every
+    // peer.  Returns the CTA sums in every lane.
+    auto dots = [&](int n, auto&& xget, float (&z)[RBM]) {
       float pd[RBM];
 #pragma unroll
       for (int r = 0; r < RBM; ++r) {
         pd[r] = 0.f;
-        if (r < a.RB) {
 #pragma unroll
-          for (int u = 0; u < NVT; ++u) {
-            const int v = tid + u * NT;
-            if (v < nvs) {
-              float x[V];
-              Vec<T>::load(st + (size_t)r * a.ld_s + v * V, x);
+        for (int u = 0; u < NVT; ++u) {
+          float x[V];
+          Vec<T>::unpack(xget(r, u), x);
 #pragma unroll
-              for (int e = 0; e < V; ++e) pd[r] = fmaf(x[e], wv[u][e], pd[r]);
-            }
-          }
+          for (int e = 0; e < V; ++e) pd[r] = fmaf(x[e], wv[u][e], pd[r]);
         }
       }
       constexpr int kRowShift = 5 - (RBM >= 4 ? 2 : (RBM >= 2 ? 1 : 0));
@@ -389,29 +420,9 @@ __global__ void __launch_bounds__(NT + 32, 1) k_chunkgrad(CGArgs a) {
       return (lane < a.RB && n < nb) ? __ldg(a.y + r0 + (long long)n * a.RB + lane) : 0.f;
     };
     float y0 = load_y(0), y1 = load_y(1);
-    float znext[RBM];
-    if (nb > 0) pass1(0, znext);
-    for (int n = 0; n < nb; ++n) {
-      const int s = n % a.S;
-      const long long row0 = r0 + (long long)n * a.RB;
-      const long long chunk = row0 / a.n_c;
-      float z[RBM];
-#pragma unroll
-      for (int r = 0; r < RBM; ++r) z[r] = znext[r];
-      // software pipelining: batch n + 1's pass 1 (and its send) before the
-      // wait for batch n's cluster sums
-      if (n + 1 < nb) pass1(n + 1, znext);
-      if (CL > 1) {
-        bounded_wait(&zfull[n % kZSlots], (uint32_t)((n / kZSlots) & 1), abort_flag, a.status,
-                     a.spin_limit, true);
-        const float* zc = zcl + (n % kZSlots) * CL * RBM;
-#pragma unroll
-        for (int r = 0; r < RBM; ++r) {
-          float t = 0.f;
-          for (int p = 0; p < CL; ++p) t += zc[p * RBM + r];
-          z[r] = t;
-        }
-      }
+    // Residuals, loss and pass 2 (acc += r * x) of batch n from its row sums z.
+    auto finish = [&](int n, const float (&z)[RBM], auto&& xget) {
+      const long long chunk = (r0 + (long long)n * a.RB) / a.n_c;
       if (chunk != cur) {
         if (cur >= 0) flush(cur);
 #pragma unroll
@@ -420,7 +431,6 @@ __global__ void __launch_bounds__(NT + 32, 1) k_chunkgrad(CGArgs a) {
           for (int e = 0; e < V; ++e) acc[u][e] = 0.f;
         cur = chunk;
       }
-      const T* st = stages + s * stage_elems;
       const float yv = y0;
       y0 = y1;
       y1 = load_y(n + 2);
@@ -461,24 +471,72 @@ __global__ void __launch_bounds__(NT + 32, 1) k_chunkgrad(CGArgs a) {
         for (int o = 2; o > 0; o >>= 1) lr += __shfl_xor_sync(0xffffffffu, lr, o);
         if (lane == 0) loss_acc += (double)lr;
       }
-      // ---- pass 2: acc += r * x, then hand the stage back to the producer
+      // ---- pass 2
 #pragma unroll
       for (int r = 0; r < RBM; ++r) {
-        if (r < a.RB) {
 #pragma unroll
-          for (int u = 0; u < NVT; ++u) {
-            const int v = tid + u * NT;
-            if (v < nvs) {
-              float x[V];
-              Vec<T>::load(st + (size_t)r * a.ld_s + v * V, x);
+        for (int u = 0; u < NVT; ++u) {
+          float x[V];
+          Vec<T>::unpack(xget(r, u), x);
 #pragma unroll
-              for (int e = 0; e < V; ++e) acc[u][e] = fmaf(res[r], x[e], acc[u][e]);
-            }
-          }
+          for (int e = 0; e < V; ++e) acc[u][e] = fmaf(res[r], x[e], acc[u][e]);
         }
       }
-      __syncwarp();
-      if (lane == 0) mbar_arrive_local(&empty[s]);
+    };
+
+    // x in registers when they fit beside acc and w (fp32 rows; not bf16,
+    // whose unpacked vectors would spill)
+    constexpr bool kXRegs = NVT * RBM * V <= 32;
+    if (CL == 1 && kXRegs) {
+      // One pass over the stage: x stays in registers from the dot products to
+      // pass 2, so the stage goes back to the producer as soon as it is read.
+      for (int n = 0; n < nb; ++n) {
+        uint4 xr[RBM][NVT];
+        float z[RBM];
+        wait_stage(n);
+        load_x(n, xr);
+        release(n);
+        auto xget = [&](int r, int u) { return xr[r][u]; };
+        dots(n, xget, z);
+        finish(n, z, xget);
+      }
+    } else if (CL == 1) {
+      for (int n = 0; n < nb; ++n) {
+        float z[RBM];
+        wait_stage(n);
+        dots(n, from_stage(n), z);
+        finish(n, z, from_stage(n));
+        release(n);
+      }
+    } else {
+      // Clusters: batch n + 1's dot products and send run before the wait for
+      // batch n's cluster sums (software pipelining); pass 2 re-reads the
+      // stage, which is handed back afterwards.
+      float znext[RBM];
+      if (nb > 0) {
+        wait_stage(0);
+        dots(0, from_stage(0), znext);
+      }
+      for (int n = 0; n < nb; ++n) {
+        float z[RBM];
+#pragma unroll
+        for (int r = 0; r < RBM; ++r) z[r] = znext[r];
+        if (n + 1 < nb) {
+          wait_stage(n + 1);
+          dots(n + 1, from_stage(n + 1), znext);
+        }
+        bounded_wait(&zfull[n % kZSlots], (uint32_t)((n / kZSlots) & 1), abort_flag, a.status,
+                     a.spin_limit, true);
+        const float* zc = zcl + (n % kZSlots) * CL * RBM;
+#pragma unroll
+        for (int r = 0; r < RBM; ++r) {
+          float t = 0.f;
+          for (int p = 0; p < CL; ++p) t += zc[p * RBM + r];
+          z[r] = t;
+        }
+        finish(n, z, from_stage(n));
+        release(n);
+      }
     }
     // the reduction kernel may be scheduled now (it waits for this grid to
     // finish); not earlier, so that work on other streams keeps the SMs' room
