@@ -253,43 +253,48 @@ def gpu_arm(args, rank, world, local_rank):
     psi_all = torch.from_numpy(psi_host).to(dev)
     live_all = torch.from_numpy(live_host).to(dev)
     # static buffers
-    psi_s = torch.empty(npat, m, dtype=torch.int32, device=dev)
-    live_s = torch.empty(1, m, dtype=torch.int32, device=dev)
+    # step inputs and per-step results are double-buffered (index t % 2) so
+    # that step t + 1's inputs are copied in, and step t - 1's results out,
+    # on a copy stream while step t runs
+    psi_b = [torch.empty(npat, m, dtype=torch.int32, device=dev) for _ in range(2)]
+    live_b = [torch.empty(1, m, dtype=torch.int32, device=dev) for _ in range(2)]
+    loss_b = [torch.zeros(1, dtype=torch.float64, device=dev) for _ in range(2)]
+    ce_b = [torch.empty(npat, dtype=torch.float64, device=dev) for _ in range(2)]
+    est_b = [torch.empty(npat, dtype=torch.float64, device=dev) for _ in range(2)]
+    mse_b = [torch.empty(npat, dtype=torch.float64, device=dev) for _ in range(2)]
     G_s = torch.empty(N, d, dtype=torch.float32, device=dev)
-    loss_s = torch.zeros(1, dtype=torch.float64, device=dev)
     plan_s = torch.empty(int(gc.lib.gc_decode_plan_bytes(N, ell, npat)), dtype=torch.uint8, device=dev)
-    ce_s = torch.empty(npat, dtype=torch.float64, device=dev)
-    est_s = torch.empty(npat, dtype=torch.float64, device=dev)
     Gh_s = torch.empty(npat, d, dtype=torch.float32, device=dev)
-    mse_s = torch.empty(npat, dtype=torch.float64, device=dev)
     T_s = torch.empty(1, m, L, dtype=torch.float32, device=dev)
     E_s = torch.empty(1, m, delta, ell, dtype=torch.float64, device=dev)
     gh_s = torch.empty(1, d, dtype=torch.float32, device=dev)
     wsA, wsB, wsC, wsD = (gc.Workspace(dev) for _ in range(4))
 
+    bi = [0]  # buffer the stage functions use (set before each capture / eager call)
+
     def stage_a():
-        gc.gc_chunk_grads(X, y, w, N, n_c, gc.GC_LOGISTIC, G=G_s, loss_out=loss_s, ws=wsA)
+        gc.gc_chunk_grads(X, y, w, N, n_c, gc.GC_LOGISTIC, G=G_s, loss_out=loss_b[bi[0]], ws=wsA)
 
     def stage_b():  # Algorithm 1 for the batch -> decode plan (psi side, no G needed)
-        gc.gc_decode_plan(Rd, ell, od, N, m, delta, psi_s, plan=plan_s, coef_err=ce_s, est=est_s,
-                          ws=wsB)
+        gc.gc_decode_plan(Rd, ell, od, N, m, delta, psi_b[bi[0]], plan=plan_s,
+                          coef_err=ce_b[bi[0]], est=est_b[bi[0]], ws=wsB)
 
     def stage_c():  # batched decode-combine from the plan and G
-        gc.gc_decode_apply(plan_s, ell, N, npat, G_s, Ghat=Gh_s, grad_mse=mse_s, ws=wsC)
+        gc.gc_decode_apply(plan_s, ell, N, npat, G_s, Ghat=Gh_s, grad_mse=mse_b[bi[0]], ws=wsC)
 
     def stage_d1():  # Algorithm 1 for the live realization (independent of G)
-        gc.gc_find_encoding_coeff(Rd, ell, od, N, m, delta, live_s, E=E_s, C=False, delta_out=False,
-                                  support=False, coef_err=False, est=False, ws=wsD)
+        gc.gc_find_encoding_coeff(Rd, ell, od, N, m, delta, live_b[bi[0]], E=E_s, C=False,
+                                  delta_out=False, support=False, coef_err=False, est=False, ws=wsD)
 
     def stage_d2():  # eq. (2) encode, PS decode, update
-        gc.gc_encode_with_coeffs(E_s, ell, od, N, m, delta, live_s, G_s, T=T_s)
+        gc.gc_encode_with_coeffs(E_s, ell, od, N, m, delta, live_b[bi[0]], G_s, T=T_s)
         gc.gc_decode_tx(Rd, ell, m, T_s, d, ghat=gh_s)
         gc.gc_sgd_step(w, gh_s[0], cfg.lr, cfg.Ntil)
 
     stages = [stage_a, stage_b, stage_c, stage_d1, stage_d2]
     # eager run: allocates workspaces, checks the device status words
-    psi_s.copy_(psi_all[0])
-    live_s.copy_(live_all[0])
+    psi_b[0].copy_(psi_all[0])
+    live_b[0].copy_(live_all[0])
     for f in stages:
         f()
     for ws in (wsA, wsB, wsC, wsD):
@@ -327,34 +332,65 @@ def gpu_arm(args, rank, world, local_rank):
             join.record(cap_hi)
         cap_stream.wait_event(join)
 
-    g1, g2 = torch.cuda.CUDAGraph(), torch.cuda.CUDAGraph()
-    with torch.cuda.graph(g1, stream=cap_stream):
-        two_streams([stage_a], [stage_d1, stage_b])
-    with torch.cuda.graph(g2, stream=cap_stream):
-        two_streams([stage_c], [stage_d2])
-    launches_per_step = gc.gc_kernel_launches() - n0
+    g1, g2 = [], []
+    for b in range(2):
+        bi[0] = b
+        g1.append(torch.cuda.CUDAGraph())
+        g2.append(torch.cuda.CUDAGraph())
+        with torch.cuda.graph(g1[b], stream=cap_stream):
+            two_streams([stage_a], [stage_d1, stage_b])
+        with torch.cuda.graph(g2[b], stream=cap_stream):
+            two_streams([stage_c], [stage_d2])
+        if b == 0:
+            launches_per_step = gc.gc_kernel_launches() - n0
     torch.cuda.synchronize()
 
     stream = torch.cuda.current_stream(dev)
 
-    def run_step(t, evs=None, host=None):
-        """One step: the step's realizations are copied into the static
-        buffers, then g1 and g2.  evs[0..3] bracket g1 and g2."""
+    copy_stream = torch.cuda.Stream(dev)
+    ev_ready = [torch.cuda.Event() for _ in range(2)]  # inputs of the buffer's next step are in
+    ev_done = [torch.cuda.Event() for _ in range(2)]   # the buffer's step has finished
+    ev_out = [torch.cuda.Event() for _ in range(2)]    # the buffer's results have been read out
+
+    def put_inputs(t, b, src):
+        """Copy step t's realizations into buffer b on the copy stream, once
+        the step that last used buffer b has finished."""
+        with torch.cuda.stream(copy_stream):
+            copy_stream.wait_event(ev_done[b])
+            psi_b[b].copy_(src[0][t], non_blocking=True)
+            live_b[b].copy_(src[1][t], non_blocking=True)
+            ev_ready[b].record(copy_stream)
+
+    def run_step(k, t, t_next, src, evs=None, outs=None):
+        """Step k on realization batch t (buffer k % 2, whose inputs are
+        already being copied in); queues the copy of batch t_next into the
+        other buffer, runs g1 and g2 and, with `outs`, copies the step's
+        results to host memory on the copy stream.  evs[0..3] bracket g1
+        and g2."""
+        b = k % 2
+
         def rec(i):
             if evs is not None:
                 evs[i].record(stream)
-        if host is None:
-            psi_s.copy_(psi_all[t], non_blocking=True)
-            live_s.copy_(live_all[t], non_blocking=True)
-        else:
-            psi_s.copy_(host[0][t], non_blocking=True)
-            live_s.copy_(host[1][t], non_blocking=True)
+        if t_next is not None:
+            put_inputs(t_next, 1 - b, src)
+        stream.wait_event(ev_ready[b])
+        stream.wait_event(ev_out[b])  # results of step k - 2 have been read out
         rec(0)
-        g1.replay()
+        g1[b].replay()
         rec(1)
         rec(2)
-        g2.replay()
+        g2[b].replay()
         rec(3)
+        ev_done[b].record(stream)
+        if outs is not None:
+            with torch.cuda.stream(copy_stream):
+                copy_stream.wait_event(ev_done[b])
+                outs[0][k].copy_(ce_b[b], non_blocking=True)
+                outs[1][k].copy_(est_b[b], non_blocking=True)
+                outs[2][k].copy_(mse_b[b], non_blocking=True)
+                outs[3][k].copy_(loss_b[b], non_blocking=True)
+                ev_out[b].record(copy_stream)
 
     import torch.distributed as tdist
 
@@ -367,25 +403,32 @@ def gpu_arm(args, rank, world, local_rank):
     clocks = Clocks(f"GPU-{uuid}" if uuid is not None else None)
     clocks.start()
     # warm-up: at least W steps and at least --min-warm-seconds
+    src_dev = (psi_all, live_all)
     t_w = time.perf_counter()
-    t = 0
-    while t < args.warmup or time.perf_counter() - t_w < args.min_warm_seconds:
-        run_step(t % S)
-        t += 1
-        if t % 64 == 0:
+    put_inputs(0, 0, src_dev)
+    k = 0
+    while k < args.warmup or time.perf_counter() - t_w < args.min_warm_seconds:
+        run_step(k, k % S, (k + 1) % S, src_dev)
+        k += 1
+        if k % 64 == 0:
             torch.cuda.synchronize()
     torch.cuda.synchronize()
 
     K = args.steps
-    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(K)]
+    # the stage events bracket g1 and g2 of every 8th timed step
+    EVERY = 8
+    evs = {k: [torch.cuda.Event(enable_timing=True) for _ in range(4)] for k in range(0, K, EVERY)}
+    batch = [(args.warmup + k) % S for k in range(K)]
     barrier()
     torch.cuda.synchronize()
     t_start = torch.cuda.Event(enable_timing=True)
     t_end = torch.cuda.Event(enable_timing=True)
     wall0 = time.perf_counter()
     t_start.record(stream)
+    copy_stream.wait_stream(stream)
+    put_inputs(batch[0], 0, src_dev)
     for k in range(K):
-        run_step(args.warmup + k if args.warmup + k < S else k % S, evs[k])
+        run_step(k, batch[k], batch[k + 1] if k + 1 < K else None, src_dev, evs.get(k))
     t_end.record(stream)
     torch.cuda.synchronize()
     barrier()
@@ -393,10 +436,10 @@ def gpu_arm(args, rank, world, local_rank):
     clk = clocks.stop()
     total_ms = t_start.elapsed_time(t_end)
     stage_ms = np.zeros(2)
-    for k in range(K):
+    for k, ev in evs.items():
         for si in range(2):
-            stage_ms[si] += evs[k][2 * si].elapsed_time(evs[k][2 * si + 1])
-    stage_ms /= K
+            stage_ms[si] += ev[2 * si].elapsed_time(ev[2 * si + 1])
+    stage_ms /= len(evs)
     for ws in (wsA, wsB, wsC, wsD):
         gc.gc_status(ws)
 
@@ -411,14 +454,14 @@ def gpu_arm(args, rank, world, local_rank):
     torch.cuda.synchronize()
     e0 = torch.cuda.Event(enable_timing=True)
     e1 = torch.cuda.Event(enable_timing=True)
+    src_host = (pin_psi, pin_live)
+    outs = (out_ce, out_est, out_mse, out_loss)
     e0.record(stream)
+    copy_stream.wait_stream(stream)
+    put_inputs(batch[0], 0, src_host)
     for k in range(K):
-        t = (args.warmup + k) % S
-        run_step(t, host=(pin_psi, pin_live))
-        out_ce[k].copy_(ce_s, non_blocking=True)
-        out_est[k].copy_(est_s, non_blocking=True)
-        out_mse[k].copy_(mse_s, non_blocking=True)
-        out_loss[k].copy_(loss_s, non_blocking=True)
+        run_step(k, batch[k], batch[k + 1] if k + 1 < K else None, src_host, None, outs)
+    stream.wait_stream(copy_stream)  # the last step's results are in host memory
     e1.record(stream)
     torch.cuda.synchronize()
     barrier()
