@@ -20,8 +20,9 @@
 // keys (the bit patterns of non-negative doubles order like the values),
 // and a most-significant-digit radix select (4-bit digits, per-lane packed
 // counters summed with warp reductions) finds the order statistic without
-// sorting.  All arithmetic is the same double multiply the definition uses,
-// so times and psi are bit-exact.
+// sorting; for theta = 0 the statistic is the largest value, a warp max
+// (and no keys are stored).  All arithmetic is the same double multiply the
+// definition uses, so times and psi are bit-exact.
 #include <math.h>
 
 #include <algorithm>
@@ -63,8 +64,12 @@ __device__ unsigned long long warp_select(const unsigned long long* keys, int n,
   return prefix;
 }
 
+// Keep the ELL smallest keys seen so far (ascending).  Keys are the bit
+// patterns of non-negative doubles, which order like the values, so the
+// comparisons are integer ones (GB300's fp64 pipe is 1/64 of fp32; only the
+// multiplies that define the times stay in fp64).
 template <int ELL>
-__device__ __forceinline__ void insert_smallest(double (&b)[ELL], double v) {
+__device__ __forceinline__ void insert_smallest(unsigned long long (&b)[ELL], unsigned long long v) {
   if (!(v < b[ELL - 1])) return;
   int q = ELL - 1;
   while (q > 0 && b[q - 1] > v) {
@@ -72,6 +77,9 @@ __device__ __forceinline__ void insert_smallest(double (&b)[ELL], double v) {
     --q;
   }
   b[q] = v;
+}
+__device__ __forceinline__ unsigned long long dbits(double x) {
+  return (unsigned long long)__double_as_longlong(x);
 }
 
 template <int ELL>
@@ -81,10 +89,13 @@ __global__ void __launch_bounds__(32 * kWarpsPerBlock)
               int32_t* __restrict__ psi_out, double* __restrict__ Tfull_out) {
   extern __shared__ unsigned long long s_dyn[];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  // per block: delta_j of every worker, then per warp 2 N ELL keys
+  // per block: delta_j of every worker; per warp: the finishing time of every
+  // worker (m keys) and, for theta > 0, 2 N ELL completion keys
   int8_t* s_dj = reinterpret_cast<int8_t*>(s_dyn);
   const size_t dj_words = ((size_t)m + 7) / 8;
-  unsigned long long* keys = s_dyn + dj_words + (size_t)warp * 2 * N * ELL;
+  unsigned long long* fin = s_dyn + dj_words + (size_t)warp * m;
+  unsigned long long* keys = s_dyn + dj_words + (size_t)kWarpsPerBlock * m +
+                             (size_t)warp * 2 * N * ELL;
   unsigned long long* keysF = keys + (size_t)N * ELL;
   for (int j = threadIdx.x; j < m; j += blockDim.x) {
     int c = 0;
@@ -97,42 +108,68 @@ __global__ void __launch_bounds__(32 * kWarpsPerBlock)
   for (long long r = (long long)blockIdx.x * kWarpsPerBlock + warp; r < nsim;
        r += (long long)gridDim.x * kWarpsPerBlock) {
     const double* tr = tau + r * m;
+    const unsigned long long kInf = dbits(INFINITY);
+    // each worker's finishing time delta_j tau_j (+inf for a failed worker)
+    for (int j = lane; j < m; j += 32) {
+      const double tj = tr[j];
+      fin[j] = isfinite(tj) ? dbits((double)s_dj[j] * tj) : kInf;
+    }
+    __syncwarp();
+    // theta = 0: the order statistic is the largest of the N ell values, i.e.
+    // the largest ell-th completion time -- a max, no selection needed
+    unsigned long long lmax = 0, lmaxF = 0;
     for (int i = lane; i < N; i += 32) {
-      double b[ELL], bf[ELL];
+      unsigned long long b[ELL], bf[ELL];
 #pragma unroll
-      for (int k = 0; k < ELL; ++k) b[k] = bf[k] = INFINITY;
+      for (int k = 0; k < ELL; ++k) b[k] = bf[k] = kInf;
       const int cnt = h.cnt[i];
       for (int q = 0; q < cnt; ++q) {
         const int j = h.w[(size_t)i * GC_MAX_REPL + q];
         const int p = h.p[(size_t)i * GC_MAX_REPL + q];
         const double tj = tr[j];
         if (isfinite(tj)) {
-          insert_smallest<ELL>(b, (double)(p + 1) * tj);
-          insert_smallest<ELL>(bf, (double)s_dj[j] * tj);
+          insert_smallest<ELL>(b, dbits((double)(p + 1) * tj));
+          insert_smallest<ELL>(bf, fin[j]);
         }
       }
+      if (theta == 0) {
+        lmax = max(lmax, b[ELL - 1]);
+        lmaxF = max(lmaxF, bf[ELL - 1]);
+      } else {
 #pragma unroll
-      for (int k = 0; k < ELL; ++k) {
-        keys[(size_t)i * ELL + k] = (unsigned long long)__double_as_longlong(b[k]);
-        keysF[(size_t)i * ELL + k] = (unsigned long long)__double_as_longlong(bf[k]);
+        for (int k = 0; k < ELL; ++k) {
+          keys[(size_t)i * ELL + k] = b[k];
+          keysF[(size_t)i * ELL + k] = bf[k];
+        }
       }
     }
     __syncwarp();
-    double T = 0.0, TF = 0.0;
-    if (kth >= 1) {
-      T = __longlong_as_double((long long)warp_select(keys, n, kth, lane));
-      TF = __longlong_as_double((long long)warp_select(keysF, n, kth, lane));
+    unsigned long long Tb = 0, TFb = 0;
+    if (theta == 0) {
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) {
+        lmax = max(lmax, (unsigned long long)__shfl_xor_sync(0xffffffffu, lmax, o));
+        lmaxF = max(lmaxF, (unsigned long long)__shfl_xor_sync(0xffffffffu, lmaxF, o));
+      }
+      Tb = lmax;
+      TFb = lmaxF;
+    } else if (kth >= 1) {
+      Tb = warp_select(keys, n, kth, lane);
+      TFb = warp_select(keysF, n, kth, lane);
     }
+    const double T = __longlong_as_double((long long)Tb);
+    const double TF = __longlong_as_double((long long)TFb);
     if (lane == 0) {
       if (T_out) T_out[r] = T;
       if (Tfull_out) Tfull_out[r] = TF;
     }
     if (psi_out)
       for (int j = lane; j < m; j += 32) {
+        // slots finish in order: count p while p tau_j <= T
         const double tj = tr[j];
         int c = 0;
         if (isfinite(tj))
-          for (int p = 1; p <= s_dj[j]; ++p) c += (double)p * tj <= T;
+          while (c < s_dj[j] && dbits((double)(c + 1) * tj) <= Tb) ++c;
         psi_out[r * m + j] = c;
       }
     __syncwarp();
@@ -142,7 +179,8 @@ __global__ void __launch_bounds__(32 * kWarpsPerBlock)
 template <int ELL>
 int launch_one(const int32_t* order, Holders h, int N, int m, int delta, const double* tau,
                long long nsim, int theta, double* T, int32_t* psi, double* TF, cudaStream_t s) {
-  const size_t smem = (((size_t)m + 7) / 8 + (size_t)kWarpsPerBlock * 2 * N * ELL) * 8;
+  const size_t keys = theta == 0 ? 0 : (size_t)kWarpsPerBlock * 2 * N * ELL;
+  const size_t smem = (((size_t)m + 7) / 8 + (size_t)kWarpsPerBlock * m + keys) * 8;
   if (smem > 48 * 1024) {
     cudaError_t e = cudaFuncSetAttribute(k_trigger<ELL>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          (int)smem);
