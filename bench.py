@@ -60,6 +60,10 @@ def parse():
                     choices=["logistic", "decode", "sweep", "sgd", "trigger", "batched"],
                     help="logistic: the headline step (default).  The others measure the "
                          "remaining configurations, one JSON line each (1 GPU)")
+    ap.add_argument("--small", action="store_true",
+                    help="with --workload batched: a 134 MB case (N=64, n_c=1024, d=1024: the "
+                         "same tile counts, short K for GEMM 1) for profiler captures instead of "
+                         "the 8.6 GB one")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--min-warm-seconds", type=float, default=1.5,
                     help="keep warming up at least this long (steady clocks, clock samples)")
@@ -685,11 +689,14 @@ def extra_workload(args):
                        "l2": "inputs larger than L2 (X 8.6 GB)"}})
     elif args.workload == "batched":
         cfg = get("mse_sweep")
+        if args.small:
+            import dataclasses
+            cfg = dataclasses.replace(cfg, N=64, m=64, n_c=1024, d=1024)
         N, d, n_c = cfg.N, cfg.d, cfg.n_c
         data = make_data(cfg, dev)
         X, y = data["X"], data["y"]
         res = {}
-        for n_w in (128, 256):
+        for n_w in ((256,) if args.small else (128, 256)):
             W = torch.randn(n_w, d, generator=torch.Generator(device=dev).manual_seed(n_w),
                             device=dev) / d ** 0.5
             G = torch.empty(n_w, N, d, device=dev)
@@ -704,7 +711,7 @@ def extra_workload(args):
             torch.cuda.empty_cache()
         r = res[256]
         line.update({
-            "metric": "chunk-gradient TFLOP/s, n_w parameter vectors at once (m=N=64, d=65536, n_c=1024, bf16 X)",
+            "metric": f"chunk-gradient TFLOP/s, n_w parameter vectors at once (m=N={N}, d={d}, n_c={n_c}, bf16 X)",
             "value": r["useful_tflops"], "unit": "TFLOP/s (useful)", "per_n_w": res,
             "roofline": {"kernel": "k_gemm_w (two GEMMs)", "bound": "tensor", "unit": "TFLOP/s",
                          "achieved": r["issued_tflops"], "peak": bf16, "frac": r["issued_tflops"] / bf16,
@@ -712,8 +719,9 @@ def extra_workload(args):
                                  "twice (once per GEMM)",
                          "peak_source": f"{pk_src} bf16_tflops"},
             "dtype": "bf16 X, f32 accumulate",
-            "config": {"workload": "batched chunk gradients N=64 n_c=1024 d=65536 bf16, n_w=128 and 256, lsq",
-                       "l2": "inputs larger than L2 (X 8.6 GB)"}})
+            "config": {"workload": f"batched chunk gradients N={N} n_c={n_c} d={d} bf16, "
+                                   f"n_w={'256' if args.small else '128 and 256'}, lsq",
+                       "l2": f"inputs larger than L2 (X {cfg.Ntil * d * 2 / 1e9:.2f} GB)"}})
     elif args.workload == "trigger":
         nsim = 100_000
         rows = {}
