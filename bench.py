@@ -9,7 +9,8 @@ communication factor l = 2.
 One step (every row of the hot path once):
   1. chunk gradients g_{D_i} at the current w            (gc_chunk_grads)
   2. Algorithm 1 for all 10^4 patterns -> decode plan,
-     coefficient error and estimate                       (gc_decode_plan)
+     coefficient error and estimate, by lookup in the
+     per-(chunk, holder subset) solutions prepared once   (gc_decode_plan_prepared)
   3. batched decode-combine Ghat = C . G (10^4 decoded
      gradients written) with the fused gradient MSE       (gc_decode_apply)
   4. the live realization: worker encoding (eq. 2), PS
@@ -279,9 +280,13 @@ def gpu_arm(args, rank, world, local_rank):
     def stage_a():
         gc.gc_chunk_grads(X, y, w, N, n_c, gc.GC_LOGISTIC, G=G_s, loss_out=loss_b[bi[0]], ws=wsA)
 
+    # set-up, once per (R, assignment) like the assignment itself: the holder
+    # table and Algorithm 1's solution for every (chunk, holder subset)
+    prep = gc.gc_decode_prepare(Rd, ell, od, N, m, delta)
+
     def stage_b():  # Algorithm 1 for the batch -> decode plan (psi side, no G needed)
-        gc.gc_decode_plan(Rd, ell, od, N, m, delta, psi_b[bi[0]], plan=plan_s,
-                          coef_err=ce_b[bi[0]], est=est_b[bi[0]], ws=wsB)
+        gc.gc_decode_plan_prepared(prep, Rd, ell, N, m, delta, psi_b[bi[0]], plan=plan_s,
+                                   coef_err=ce_b[bi[0]], est=est_b[bi[0]], ws=wsB)
 
     def stage_c():  # batched decode-combine from the plan and G
         gc.gc_decode_apply(plan_s, ell, N, npat, G_s, Ghat=Gh_s, grad_mse=mse_b[bi[0]], ws=wsC)

@@ -328,6 +328,33 @@ size_t gc_decode_plan_workspace(int N, int m, int delta, int ell, int npat);
 int gc_decode_plan(const double* R, int ell, const int32_t* order, int N, int m, int delta,
                    const int32_t* psi, int npat, void* plan, size_t plan_bytes, double* coef_err,
                    double* est, void* ws, size_t ws_bytes, void* stream);
+/* ---- prepared decode: the parts of Algorithm 1 that depend only on R and
+ * the assignment, computed once -----------------------------------------
+ * Every block problem of Algorithm 1 is X = R[:, S] for S a subset of the
+ * holders of one chunk (Sec. II), so for an assignment with delta <= 14
+ * chunks per worker all of them -- one per (chunk, subset of its holders) --
+ * can be solved once and looked up for every pattern.  gc_decode_prepare
+ * writes the holder table and, when delta <= 14, that memo table (the block
+ * R_S X^+ and its error ||I - R_S X^+||_F^2 per subset) into a caller-owned
+ * device buffer `prep` of gc_decode_prepare_bytes(N, m, delta, ell) bytes
+ * (256-byte aligned; its first 256 bytes are a status header, read with
+ * gc_status).  gc_decode_plan_prepared then does the psi side of the decode
+ * for a batch as gc_decode_plan does, without recomputing them: the same
+ * plan, coefficient error and estimate bit for bit whenever gc_decode_plan
+ * itself uses its memo table (npat >= 2^delta), equal to rounding otherwise;
+ * with delta > 14 it solves every block directly.  `prep` must come from the same R, ell,
+ * order, N, m and delta; it is read-only afterwards and may serve any number
+ * of calls.  ws needs gc_decode_plan_prepared_workspace() bytes (a status
+ * header only). */
+size_t gc_decode_prepare_bytes(int N, int m, int delta, int ell);
+int gc_decode_prepare(const double* R, int ell, const int32_t* order, int N, int m, int delta,
+                      void* prep, size_t prep_bytes, void* stream);
+size_t gc_decode_plan_prepared_workspace(void);
+int gc_decode_plan_prepared(const void* prep, const double* R, int ell, int N, int m, int delta,
+                            const int32_t* psi, int npat, void* plan, size_t plan_bytes,
+                            double* coef_err, double* est, void* ws, size_t ws_bytes,
+                            void* stream);
+
 size_t gc_decode_apply_workspace(int N, int ell, int npat, int d);
 int gc_decode_apply(const void* plan, int ell, int N, int npat, const float* G, int d,
                     float* Ghat, double* grad_mse, void* ws, size_t ws_bytes, void* stream);

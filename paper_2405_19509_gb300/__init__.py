@@ -39,6 +39,8 @@ from .binding import (  # noqa: F401
     gc_chunk_ordering,
     gc_trigger_times,
     gc_chunk_grads_batched,
+    gc_decode_prepare,
+    gc_decode_plan_prepared,
     gc_inject_stall,
     GC_STALL_CHUNK_GRADS,
     GC_STALL_COMBINE,

@@ -65,6 +65,10 @@ _sig("gc_decode_batch", _i, _p, _i, _p, _i, _i, _i, _p, _i, _p, _i, _p, _p, _p, 
 _sig("gc_decode_plan_bytes", _sz, _i, _i, _i)
 _sig("gc_decode_plan_workspace", _sz, _i, _i, _i, _i, _i)
 _sig("gc_decode_plan", _i, _p, _i, _p, _i, _i, _i, _p, _i, _p, _sz, _p, _p, _p, _sz, _p)
+_sig("gc_decode_prepare_bytes", _sz, _i, _i, _i, _i)
+_sig("gc_decode_prepare", _i, _p, _i, _p, _i, _i, _i, _p, _sz, _p)
+_sig("gc_decode_plan_prepared_workspace", _sz)
+_sig("gc_decode_plan_prepared", _i, _p, _p, _i, _i, _i, _i, _p, _i, _p, _sz, _p, _p, _p, _sz, _p)
 _sig("gc_decode_apply_workspace", _sz, _i, _i, _i, _i)
 _sig("gc_decode_apply", _i, _p, _i, _i, _i, _p, _i, _p, _p, _p, _sz, _p)
 _sig("gc_decode_combine_workspace", _sz, _i, _i, _i, _i)
@@ -381,6 +385,43 @@ def gc_decode_plan(R, ell, order, N, m, delta, psi, plan=None, coef_err=True, es
                               _dev(plan, torch.uint8, "plan"), plan.numel(),
                               _dev(ce, torch.float64, "coef_err"), _dev(es, torch.float64, "est"),
                               wp, wn, _stream()))
+    return {"plan": plan, "coef_err": ce, "est": es}
+
+
+def gc_decode_prepare(R, ell, order, N, m, delta, prep=None):
+    """Holders and the Algorithm 1 memo table for (R, assignment), once:
+    a uint8 device buffer for gc_decode_plan_prepared."""
+    nb = int(lib.gc_decode_prepare_bytes(N, m, delta, ell))
+    if nb == 0:
+        raise ValueError("unsupported shape for gc_decode_prepare")
+    if prep is None:
+        prep = torch.empty(nb, dtype=torch.uint8, device=R.device)
+    _check(lib.gc_decode_prepare(_dev(R, torch.float64, "R", (ell, m)), ell,
+                                 _dev(order, torch.int32, "order", (m, delta)), N, m, delta,
+                                 _dev(prep, torch.uint8, "prep"), prep.numel(), _stream()))
+    return prep
+
+
+def gc_decode_plan_prepared(prep, R, ell, N, m, delta, psi, plan=None, coef_err=True, est=True,
+                            ws: Workspace | None = None):
+    """gc_decode_plan from a gc_decode_prepare buffer.  Returns dict with
+    plan, coef_err, est."""
+    npat = psi.shape[0]
+    dev = psi.device
+    nb = lib.gc_decode_plan_bytes(N, ell, npat)
+    if plan is None:
+        plan = torch.empty(max(int(nb), 256), dtype=torch.uint8, device=dev)
+    ce = coef_err if isinstance(coef_err, torch.Tensor) else (
+        torch.empty(npat, dtype=torch.float64, device=dev) if coef_err else None)
+    es = est if isinstance(est, torch.Tensor) else (
+        torch.empty(npat, dtype=torch.float64, device=dev) if est else None)
+    ws, (wp, wn) = _ws(ws, lib.gc_decode_plan_prepared_workspace(), dev)
+    _check(lib.gc_decode_plan_prepared(_dev(prep, torch.uint8, "prep"),
+                                       _dev(R, torch.float64, "R", (ell, m)), ell, N, m, delta,
+                                       _dev(psi, torch.int32, "psi", (npat, m)), npat,
+                                       _dev(plan, torch.uint8, "plan"), plan.numel(),
+                                       _dev(ce, torch.float64, "coef_err"),
+                                       _dev(es, torch.float64, "est"), wp, wn, _stream()))
     return {"plan": plan, "coef_err": ce, "est": es}
 
 

@@ -373,6 +373,68 @@ int gc_decode_plan(const double* R, int ell, const int32_t* order, int N, int m,
                            status_of(ws), s);
 }
 
+// Layout of a prepared buffer: status header, holders, memo table (delta <= 14).
+static int prep_bits(int delta) { return delta <= 14 ? delta : -1; }
+
+size_t gc_decode_prepare_bytes(int N, int m, int delta, int ell) {
+  if (N < 1 || m < 1 || delta < 1 || ell < 1 || ell > GC_MAX_ELL || delta > GC_MAX_DELTA) return 0;
+  Carve c(nullptr);
+  carve_holders(c, N);
+  c.take<char>(solve_table_bytes(N, ell, prep_bits(delta)));
+  return c.bytes();
+}
+
+int gc_decode_prepare(const double* R, int ell, const int32_t* order, int N, int m, int delta,
+                      void* prep, size_t prep_bytes, void* stream) {
+  int rc = check_dims(N, m, delta, ell, 0);
+  if (rc) return rc;
+  if (!R || !order) return fail(GC_ERR_ARG, "R and order must be non-NULL");
+  if (!prep || reinterpret_cast<uintptr_t>(prep) % 256 != 0)
+    return fail(GC_ERR_WORKSPACE, "prep must be a 256-byte aligned device buffer");
+  if (prep_bytes < gc_decode_prepare_bytes(N, m, delta, ell))
+    return fail(GC_ERR_WORKSPACE, "prep buffer too small: %zu < %zu bytes", prep_bytes,
+                gc_decode_prepare_bytes(N, m, delta, ell));
+  cudaStream_t s = as_stream(stream);
+  GC_CUDA(cudaMemsetAsync(prep, 0, kHeaderBytes, s));
+  Carve c(prep);
+  Holders h = carve_holders(c, N);
+  const int bits = prep_bits(delta);
+  void* table = bits >= 0 ? c.take<char>(solve_table_bytes(N, ell, bits)) : nullptr;
+  launch_holders(order, N, m, delta, h, status_of(prep), s);
+  if (bits < 0) return cuda_check(cudaGetLastError(), "k_holders");
+  SolveOut out{nullptr, nullptr, nullptr, nullptr, nullptr, nullptr, nullptr, combine_kp(N, ell)};
+  return launch_solve_impl(R, ell, nullptr, h, N, m, delta, 0, out, table, bits, status_of(prep),
+                           s, true);
+}
+
+size_t gc_decode_plan_prepared_workspace(void) { return kHeaderBytes; }
+
+int gc_decode_plan_prepared(const void* prep, const double* R, int ell, int N, int m, int delta,
+                            const int32_t* psi, int npat, void* plan, size_t plan_bytes_,
+                            double* coef_err, double* est, void* ws, size_t ws_bytes,
+                            void* stream) {
+  int rc = check_dims(N, m, delta, ell, npat);
+  if (rc) return rc;
+  if (!prep || !R || (!psi && npat > 0)) return fail(GC_ERR_ARG, "prep, R and psi must be non-NULL");
+  if (npat == 0) return GC_OK;
+  if (!plan) return fail(GC_ERR_ARG, "plan is NULL");
+  if (plan_bytes_ < plan_bytes(N, ell, npat))
+    return fail(GC_ERR_WORKSPACE, "plan buffer too small: %zu < %zu bytes", plan_bytes_,
+                plan_bytes(N, ell, npat));
+  if (reinterpret_cast<uintptr_t>(plan) % 256 != 0)
+    return fail(GC_ERR_WORKSPACE, "plan buffer must be 256-byte aligned");
+  rc = check_ws(ws, ws_bytes, kHeaderBytes);
+  if (rc) return rc;
+  Carve c(const_cast<void*>(prep));
+  Holders h = carve_holders(c, N);
+  const int bits = prep_bits(delta);
+  void* table = bits >= 0 ? c.take<char>(solve_table_bytes(N, ell, bits)) : nullptr;
+  SolveOut out{nullptr, nullptr, nullptr, nullptr, coef_err, est,
+               static_cast<__nv_bfloat16*>(plan), combine_kp(N, ell)};
+  return launch_solve_impl(R, ell, psi, h, N, m, delta, npat, out, table, bits, status_of(ws),
+                           as_stream(stream), false);
+}
+
 size_t gc_decode_apply_workspace(int N, int ell, int npat, int d) {
   if (N < 1 || ell < 1 || ell > GC_MAX_ELL || npat < 0 || d < 1) return 0;
   return kHeaderBytes + apply_ws_bytes(N, ell, npat, d);

@@ -98,7 +98,7 @@ int solve_table_bits(int N, int m, int delta, int npat);
 size_t solve_table_bytes(int N, int ell, int bits);
 int launch_solve_impl(const double* R, int ell, const int32_t* psi, Holders h, int N, int m,
                       int delta, int npat, SolveOut out, void* table_mem, int bits,
-                      uint32_t* status, cudaStream_t s);
+                      uint32_t* status, cudaStream_t s, bool build_table = true);
 
 // ---- chunk gradients (k_chunkgrad.cu) -----------------------------------
 size_t chunkgrad_ws_bytes(int N, int n_c, int d, int x_dtype);

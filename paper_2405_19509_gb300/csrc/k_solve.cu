@@ -674,15 +674,16 @@ __global__ void __launch_bounds__(128) k_patterns_warp(const double* __restrict_
 
 template <int ELL>
 static void run_solve(const double* R, const int32_t* psi, Holders h, int N, int m, int delta,
-                      int npat, SolveOut out, Table tb, bool use_table, uint32_t* status,
-                      cudaStream_t s) {
-  if (use_table) {
+                      int npat, SolveOut out, Table tb, bool use_table, bool build_table,
+                      uint32_t* status, cudaStream_t s) {
+  if (use_table && build_table) {
     // one warp per block: the fp64 pipe is narrow, so spread the solves over SMs
     const long long nent = (long long)N << tb.bits;
     const int blocks = (int)((nent + 31) / 32);
     k_table<ELL><<<blocks, 32, 0, s>>>(R, h, N, m, tb, out.E != nullptr, status);
     count_launches(1);
   }
+  if (npat == 0) return;
   if (!out.E && N <= 32) {
     const int warps = 4;  // per 128-thread block
     const int blocks = std::max(1, std::min((npat + warps - 1) / warps, 8 * device_sm_count()));
@@ -706,10 +707,12 @@ static void run_solve(const double* R, const int32_t* psi, Holders h, int N, int
                                                        status);
 }
 
-// The table region is carved by the caller right after the holders.
+// The table region is carved by the caller right after the holders.  With
+// build_table = false the table already holds every entry (gc_decode_prepare)
+// and npat may be 0 with build_table = true to build it alone.
 int launch_solve_impl(const double* R, int ell, const int32_t* psi, Holders h, int N, int m,
                       int delta, int npat, SolveOut out, void* table_mem, int bits,
-                      uint32_t* status, cudaStream_t s) {
+                      uint32_t* status, cudaStream_t s, bool build_table) {
   Table tb{bits < 0 ? 0 : bits, nullptr, nullptr, nullptr};
   const bool use_table = bits >= 0 && table_mem != nullptr;
   if (use_table) {
@@ -726,14 +729,14 @@ int launch_solve_impl(const double* R, int ell, const int32_t* psi, Holders h, i
     if (e != cudaSuccess) return cuda_check(e, "cudaMemsetAsync(E)");
   }
   switch (ell) {
-    case 1: run_solve<1>(R, psi, h, N, m, delta, npat, out, tb, use_table, status, s); break;
-    case 2: run_solve<2>(R, psi, h, N, m, delta, npat, out, tb, use_table, status, s); break;
-    case 3: run_solve<3>(R, psi, h, N, m, delta, npat, out, tb, use_table, status, s); break;
-    case 4: run_solve<4>(R, psi, h, N, m, delta, npat, out, tb, use_table, status, s); break;
-    case 5: run_solve<5>(R, psi, h, N, m, delta, npat, out, tb, use_table, status, s); break;
-    case 6: run_solve<6>(R, psi, h, N, m, delta, npat, out, tb, use_table, status, s); break;
-    case 7: run_solve<7>(R, psi, h, N, m, delta, npat, out, tb, use_table, status, s); break;
-    case 8: run_solve<8>(R, psi, h, N, m, delta, npat, out, tb, use_table, status, s); break;
+    case 1: run_solve<1>(R, psi, h, N, m, delta, npat, out, tb, use_table, build_table, status, s); break;
+    case 2: run_solve<2>(R, psi, h, N, m, delta, npat, out, tb, use_table, build_table, status, s); break;
+    case 3: run_solve<3>(R, psi, h, N, m, delta, npat, out, tb, use_table, build_table, status, s); break;
+    case 4: run_solve<4>(R, psi, h, N, m, delta, npat, out, tb, use_table, build_table, status, s); break;
+    case 5: run_solve<5>(R, psi, h, N, m, delta, npat, out, tb, use_table, build_table, status, s); break;
+    case 6: run_solve<6>(R, psi, h, N, m, delta, npat, out, tb, use_table, build_table, status, s); break;
+    case 7: run_solve<7>(R, psi, h, N, m, delta, npat, out, tb, use_table, build_table, status, s); break;
+    case 8: run_solve<8>(R, psi, h, N, m, delta, npat, out, tb, use_table, build_table, status, s); break;
     default: return fail(GC_ERR_UNSUPPORTED, "ell=%d exceeds GC_MAX_ELL", ell);
   }
   return cuda_check(cudaGetLastError(), "solve kernels");

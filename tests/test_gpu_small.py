@@ -318,3 +318,52 @@ def test_decode_plan_then_apply(gc, ell):
     for b in range(0, psi.shape[0], 7):
         r = O.run_pattern(R, order, psi[b], N, G.astype(np.float64), want_transmit=False)
         assert_grad_close(to_np(ap["Ghat"][b]), r.ghat, f"plan/apply b={b}")
+
+
+@pytest.mark.parametrize("cfg_name,ell,npat", [("tiny", 2, 256), ("tiny", 3, 5), ("logistic", 2, 2000)])
+def test_prepared_plan_matches_plan(gc, cfg_name, ell, npat):
+    """gc_decode_plan_prepared equals gc_decode_plan bit for bit when the
+    latter uses its memo table (npat >= 2^delta), to rounding otherwise; the
+    prepared buffer serves several batches."""
+    from workloads import get, make_R, make_patterns
+    cfg = get(cfg_name)
+    N, m, delta = cfg.N, cfg.m, cfg.delta
+    order = O.cyclic_order(N, m, delta)
+    dev = torch.device("cuda")
+    Rd = torch.from_numpy(make_R(cfg, ell)).to(dev)
+    od = torch.from_numpy(order).to(dev)
+    prep = gc.gc_decode_prepare(Rd, ell, od, N, m, delta)
+    for stream in (0, 1):
+        psi = torch.from_numpy(make_patterns(cfg, npat=npat, stream=stream)).to(dev)
+        a = gc.gc_decode_plan(Rd, ell, od, N, m, delta, psi)
+        b = gc.gc_decode_plan_prepared(prep, Rd, ell, N, m, delta, psi)
+        torch.cuda.synchronize()
+        assert torch.equal(a["est"], b["est"])
+        if npat >= 2 ** delta:
+            assert torch.equal(a["plan"], b["plan"])
+            assert torch.equal(a["coef_err"], b["coef_err"])
+        else:
+            assert torch.allclose(a["coef_err"], b["coef_err"], rtol=0, atol=1e-9)
+            pa = a["plan"].view(torch.bfloat16).float()
+            pb = b["plan"].view(torch.bfloat16).float()
+            assert torch.allclose(pa, pb, rtol=2 ** -7, atol=1e-6)
+
+
+def test_prepared_plan_direct_solves_for_large_delta(gc):
+    """delta = 16 > 14: no memo table; the prepared call solves every block
+    directly and agrees with the oracle's coefficient error."""
+    from workloads import get, make_R, make_patterns
+    cfg = get("decode")
+    N, m, delta, ell = 64, 64, 16, 2
+    order = O.cyclic_order(N, m, delta)
+    dev = torch.device("cuda")
+    R = np.random.default_rng(5).standard_normal((ell, m))
+    Rd, od = torch.from_numpy(R).to(dev), torch.from_numpy(order).to(dev)
+    psi_np = np.random.default_rng(6).integers(0, delta + 1, size=(40, m)).astype(np.int32)
+    prep = gc.gc_decode_prepare(Rd, ell, od, N, m, delta)
+    b = gc.gc_decode_plan_prepared(prep, Rd, ell, N, m, delta, torch.from_numpy(psi_np).to(dev))
+    ce = b["coef_err"].cpu().numpy()
+    for i in range(0, 40, 7):
+        r = O.run_pattern(R, order, psi_np[i], N, None, want_transmit=False)
+        assert abs(ce[i] - r.coef_err) <= 1e-9 * max(1.0, r.coef_err)
+        assert b["est"][i].item() == r.est
