@@ -57,16 +57,18 @@ int launch_encode(const double* E, const int32_t* order, const int32_t* psi, int
 
 // ghat[b][k*L + c] = sum_j R[k][j] * T[b][j][c].  One thread per (b, c); R is
 // staged in dynamic shared memory as fp32 (ELL * m words, m <= kDecodeSmemM)
-// or read as fp64.
+// or read as fp64.  The transmissions are loaded eight workers at a time, so
+// that eight independent loads are in flight per thread (the kernel is
+// latency-bound at the sizes of one live realization).
 constexpr int kDecodeSmemM = 1024;
-template <int ELL>
+template <int ELL, bool STAGED>
 __global__ void k_decode_tx(const double* __restrict__ R, int m, const float* __restrict__ T,
                             int npat, int d, int L, float* __restrict__ ghat) {
   extern __shared__ float s_r[];
-  const bool staged = m <= kDecodeSmemM;
-  if (staged)
+  if (STAGED) {
     for (int t = threadIdx.x; t < ELL * m; t += blockDim.x) s_r[t] = (float)R[t];
-  __syncthreads();
+    __syncthreads();
+  }
   const long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;
   if (idx >= (long long)npat * L) return;
   const int c = (int)(idx % L);
@@ -75,13 +77,19 @@ __global__ void k_decode_tx(const double* __restrict__ R, int m, const float* __
 #pragma unroll
   for (int k = 0; k < ELL; ++k) acc[k] = 0.f;
   const float* Tb = T + (size_t)b * m * L + c;
-#pragma unroll 8
-  for (int j = 0; j < m; ++j) {
-    const float t = __ldg(Tb + (size_t)j * L);
+  for (int j0 = 0; j0 < m; j0 += 8) {
+    float t[8];
 #pragma unroll
-    for (int k = 0; k < ELL; ++k) {
-      const float r = staged ? s_r[k * m + j] : (float)__ldg(R + (size_t)k * m + j);
-      acc[k] = fmaf(r, t, acc[k]);
+    for (int u = 0; u < 8; ++u) t[u] = j0 + u < m ? __ldg(Tb + (size_t)(j0 + u) * L) : 0.f;
+#pragma unroll
+    for (int u = 0; u < 8; ++u) {
+      if (j0 + u < m) {
+#pragma unroll
+        for (int k = 0; k < ELL; ++k) {
+          const float r = STAGED ? s_r[k * m + j0 + u] : (float)__ldg(R + (size_t)k * m + j0 + u);
+          acc[k] = fmaf(r, t[u], acc[k]);
+        }
+      }
     }
   }
 #pragma unroll
@@ -96,20 +104,29 @@ int launch_decode_tx(const double* R, int ell, int m, const float* T, int npat, 
   const int L = (d + ell - 1) / ell;
   const long long tot = (long long)npat * L;
   if (tot == 0) return GC_OK;
-  const int threads = 256;
+  const int threads = 128;
   const unsigned blocks = (unsigned)((tot + threads - 1) / threads);
-  const size_t sm = m <= kDecodeSmemM ? (size_t)ell * m * sizeof(float) : 0;
+  const bool staged = m <= kDecodeSmemM;
+  const size_t sm = staged ? (size_t)ell * m * sizeof(float) : 0;
+#define GC_DTX(E)                                                                              \
+  case E:                                                                                      \
+    if (staged)                                                                                \
+      k_decode_tx<E, true><<<blocks, threads, sm, s>>>(R, m, T, npat, d, L, ghat);             \
+    else                                                                                       \
+      k_decode_tx<E, false><<<blocks, threads, 0, s>>>(R, m, T, npat, d, L, ghat);             \
+    break;
   switch (ell) {
-    case 1: k_decode_tx<1><<<blocks, threads, sm, s>>>(R, m, T, npat, d, L, ghat); break;
-    case 2: k_decode_tx<2><<<blocks, threads, sm, s>>>(R, m, T, npat, d, L, ghat); break;
-    case 3: k_decode_tx<3><<<blocks, threads, sm, s>>>(R, m, T, npat, d, L, ghat); break;
-    case 4: k_decode_tx<4><<<blocks, threads, sm, s>>>(R, m, T, npat, d, L, ghat); break;
-    case 5: k_decode_tx<5><<<blocks, threads, sm, s>>>(R, m, T, npat, d, L, ghat); break;
-    case 6: k_decode_tx<6><<<blocks, threads, sm, s>>>(R, m, T, npat, d, L, ghat); break;
-    case 7: k_decode_tx<7><<<blocks, threads, sm, s>>>(R, m, T, npat, d, L, ghat); break;
-    case 8: k_decode_tx<8><<<blocks, threads, sm, s>>>(R, m, T, npat, d, L, ghat); break;
+    GC_DTX(1)
+    GC_DTX(2)
+    GC_DTX(3)
+    GC_DTX(4)
+    GC_DTX(5)
+    GC_DTX(6)
+    GC_DTX(7)
+    GC_DTX(8)
     default: return fail(GC_ERR_UNSUPPORTED, "ell=%d exceeds GC_MAX_ELL", ell);
   }
+#undef GC_DTX
   count_launches(1);
   return cuda_check(cudaGetLastError(), "k_decode_tx");
 }
