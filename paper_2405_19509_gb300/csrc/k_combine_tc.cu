@@ -531,47 +531,84 @@ __global__ void k_split_c(const float* __restrict__ C, int M, int K, int Kp,
 }
 
 // G (N x d fp32) -> planes [2][L][Kp] bf16 of Gv^T: element (c, i*ell + k') =
-// g_{D_i}[k'*L + c] (zero past d and for padding columns), 32 x 32 tiles
-// transposed through shared memory; blocks with blockIdx.y == 0 also write
+// g_{D_i}[k'*L + c] (zero past d and for padding columns).  Block (x, y)
+// transposes the tile of 32 K-rows (kk = 32 y ..) by COLS columns
+// (c = COLS x ..) through shared memory: 16-byte loads along c, 16-byte
+// stores along kk (COLS = 128 for long rows, 32 when L is short and more
+// blocks are wanted).  Blocks with y == 0 also write
 // gsum[k'*L + c] = sum_i g_{D_i}[k'*L + c] (chunks in order) when gsum != 0.
-__global__ void k_split_gt(const float* __restrict__ G, int N, int d, int ell, int L, int Kp,
-                           __nv_bfloat16* __restrict__ out, float* __restrict__ gsum) {
+template <int COLS>
+__global__ void __launch_bounds__(256) k_split_gt(const float* __restrict__ G, int N, int d,
+                                                  int ell, int L, int Kp,
+                                                  __nv_bfloat16* __restrict__ out,
+                                                  float* __restrict__ gsum) {
+  constexpr int kSplitCols = COLS;
+  constexpr int TPR = COLS / 4;            // threads per row of the load phase
+  constexpr int RPP = 256 / TPR;           // rows per pass
   // the combine kernel may be scheduled now; it waits for this grid to finish
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
-  __shared__ float tile[32][33];
-  const int c0 = blockIdx.x * 32, k0 = blockIdx.y * 32;
-  const int tx = threadIdx.x, ty = threadIdx.y;  // 32 x 8
+  __shared__ float tile[32][kSplitCols + 1];
+  const int c0 = blockIdx.x * kSplitCols, k0 = blockIdx.y * 32;
+  const int t = threadIdx.x;
   const int K = N * ell;
+  const bool vec = (L % 4 == 0) && (d % 4 == 0) && (reinterpret_cast<uintptr_t>(G) % 16 == 0);
+  // load: thread t takes columns 4 (t % TPR) .. +3 of rows t / TPR + RPP r
+#pragma unroll
+  for (int r = 0; r < 32 / RPP; ++r) {
+    const int kr = t / TPR + RPP * r, kk = k0 + kr;
+    const int cc = 4 * (t % TPR), c = c0 + cc;
+    float v[4] = {0.f, 0.f, 0.f, 0.f};
+    if (kk < K) {
+      const int i = kk / ell, kp = kk - i * ell;
+      const float* src = G + (size_t)i * d + (size_t)kp * L + c;
+      if (vec && c + 3 < L && kp * L + c + 3 < d) {
+        const float4 q = __ldg(reinterpret_cast<const float4*>(src));
+        v[0] = q.x; v[1] = q.y; v[2] = q.z; v[3] = q.w;
+      } else {
+#pragma unroll
+        for (int e = 0; e < 4; ++e)
+          if (c + e < L && kp * L + c + e < d) v[e] = __ldg(src + e);
+      }
+    }
+#pragma unroll
+    for (int e = 0; e < 4; ++e) tile[kr][cc + e] = v[e];
+  }
+  __syncthreads();
+  // store: thread t takes column t % COLS and K-rows 16 (t / COLS) .. +15
+  if (t < 2 * kSplitCols) {
+    const int cc = t % kSplitCols, h = t / kSplitCols, c = c0 + cc;
+    if (c < L) {
+      uint32_t hw[8], lw[8];
+#pragma unroll
+      for (int e = 0; e < 16; e += 2) {
+        const float a = tile[16 * h + e][cc], b = tile[16 * h + e + 1][cc];
+        const __nv_bfloat16 ha = __float2bfloat16_rn(a), hb = __float2bfloat16_rn(b);
+        const __nv_bfloat16 la = __float2bfloat16_rn(a - __bfloat162float(ha));
+        const __nv_bfloat16 lb = __float2bfloat16_rn(b - __bfloat162float(hb));
+        hw[e / 2] = (uint32_t)__bfloat16_as_ushort(ha) | ((uint32_t)__bfloat16_as_ushort(hb) << 16);
+        lw[e / 2] = (uint32_t)__bfloat16_as_ushort(la) | ((uint32_t)__bfloat16_as_ushort(lb) << 16);
+      }
+      const int kk = k0 + 16 * h;
+      if (kk < Kp) {  // Kp is a multiple of 64, so the 16 entries are all inside
+        const size_t plane = (size_t)L * Kp;
+        uint4* dh = reinterpret_cast<uint4*>(out + (size_t)c * Kp + kk);
+        uint4* dl = reinterpret_cast<uint4*>(out + plane + (size_t)c * Kp + kk);
+        dh[0] = make_uint4(hw[0], hw[1], hw[2], hw[3]);
+        dh[1] = make_uint4(hw[4], hw[5], hw[6], hw[7]);
+        dl[0] = make_uint4(lw[0], lw[1], lw[2], lw[3]);
+        dl[1] = make_uint4(lw[4], lw[5], lw[6], lw[7]);
+      }
+    }
+  }
   if (gsum && blockIdx.y == 0) {
-    for (int kp = ty; kp < ell; kp += 8) {
-      const int col = kp * L + c0 + tx;
-      if (c0 + tx < L && col < d) {
+    for (int it = t; it < kSplitCols * ell; it += blockDim.x) {
+      const int cc = it % kSplitCols, kp = it / kSplitCols, c = c0 + cc;
+      const int col = kp * L + c;
+      if (c < L && col < d) {
         float acc = 0.f;
         for (int i = 0; i < N; ++i) acc += __ldg(G + (size_t)i * d + col);
         gsum[col] = acc;
       }
-    }
-  }
-  for (int r = ty; r < 32; r += 8) {
-    const int kk = k0 + r, c = c0 + tx;
-    float v = 0.f;
-    if (kk < K && c < L) {
-      const int i = kk / ell, kp = kk - i * ell;
-      const int col = kp * L + c;
-      if (col < d) v = __ldg(G + (size_t)i * d + col);
-    }
-    tile[r][tx] = v;
-  }
-  __syncthreads();
-  const size_t plane = (size_t)L * Kp;
-  for (int r = ty; r < 32; r += 8) {
-    const int c = c0 + r, kk = k0 + tx;
-    if (c < L && kk < Kp) {
-      const float v = tile[tx][r];
-      const __nv_bfloat16 hi = __float2bfloat16_rn(v);
-      const __nv_bfloat16 lo = __float2bfloat16_rn(v - __bfloat162float(hi));
-      out[(size_t)c * Kp + kk] = hi;
-      out[plane + (size_t)c * Kp + kk] = lo;
     }
   }
 }
@@ -700,8 +737,13 @@ int launch_apply(const __nv_bfloat16* Cs, const float* G, int N, int ell, int np
   float* gsum = ws.take<float>((size_t)d);
   float* msep = grad_mse ? ws.take<float>((size_t)M * nnt * 2) : nullptr;
   {
-    dim3 grid((L + 31) / 32, (Kp + 31) / 32);
-    k_split_gt<<<grid, dim3(32, 8), 0, s>>>(G, N, d, ell, L, Kp, Gs, grad_mse ? gsum : nullptr);
+    if (L >= 16384) {
+      dim3 grid((L + 127) / 128, Kp / 32);
+      k_split_gt<128><<<grid, 256, 0, s>>>(G, N, d, ell, L, Kp, Gs, grad_mse ? gsum : nullptr);
+    } else {
+      dim3 grid((L + 31) / 32, Kp / 32);
+      k_split_gt<32><<<grid, 256, 0, s>>>(G, N, d, ell, L, Kp, Gs, grad_mse ? gsum : nullptr);
+    }
     count_launches(1);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return cuda_check(e, "k_split_gt");
