@@ -615,21 +615,22 @@ __global__ void __launch_bounds__(256) k_split_gt(const float* __restrict__ G, i
 
 // grad_mse[b] = (sum of the partial squared errors of rows b*ell .. b*ell+ell-1) / d:
 // one warp per pattern (its ell * parts partials are contiguous), lanes
-// stride over them, then a fixed xor tree in fp64.  Launched as a
-// programmatic dependent of the combine kernel.
+// stride over them, then a fixed xor tree (fp32: the partials are fp32 sums
+// already; the result is scaled in fp64).  Launched as a programmatic
+// dependent of the combine kernel.
 __global__ void k_mse_reduce_tiles(const float* __restrict__ msep, int npat, int ell,
-                                   int parts, int d, double* __restrict__ grad_mse) {
+                                   int parts, double inv_d, double* __restrict__ grad_mse) {
   asm volatile("griddepcontrol.wait;" ::: "memory");
   const long long b = ((long long)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
   const int lane = threadIdx.x & 31;
   if (b >= npat) return;
   const float* r = msep + (size_t)b * ell * parts;
   const int n = ell * parts;
-  double s = 0.0;
-  for (int t = lane; t < n; t += 32) s += (double)__ldg(r + t);
+  float s = 0.f;
+  for (int t = lane; t < n; t += 32) s += __ldg(r + t);
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
-  if (lane == 0) grad_mse[b] = s / (double)d;
+  if (lane == 0) grad_mse[b] = (double)s * inv_d;
 }
 
 PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
@@ -797,7 +798,7 @@ int launch_apply(const __nv_bfloat16* Cs, const float* G, int N, int ell, int np
     cfg.attrs = attr;
     cfg.numAttrs = 1;
     cudaError_t e = cudaLaunchKernelEx(&cfg, k_mse_reduce_tiles, (const float*)msep, npat, ell,
-                                       p.parts_per_row, d, grad_mse);
+                                       p.parts_per_row, 1.0 / (double)d, grad_mse);
     if (e != cudaSuccess) return cuda_check(e, "cudaLaunchKernelEx(k_mse_reduce_tiles)");
     count_launches(1);
   }
