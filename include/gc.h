@@ -98,6 +98,7 @@ int gc_set_wait_limit(int64_t cycles);
  * CUDA graph (the capture would keep the withheld copy).  Process-wide. */
 #define GC_STALL_CHUNK_GRADS 1 /* the chunk-gradient kernel (gc_chunk_grads)  */
 #define GC_STALL_COMBINE 2     /* the tensor-core combine (decode apply, MSE) */
+#define GC_STALL_BATCHED 4     /* the batched chunk-gradient GEMMs (first one) */
 int gc_inject_stall(int kernels);
 
 /* Zero the status header of a workspace (asynchronous on `stream`). */

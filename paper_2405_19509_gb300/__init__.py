@@ -44,6 +44,7 @@ from .binding import (  # noqa: F401
     gc_inject_stall,
     GC_STALL_CHUNK_GRADS,
     GC_STALL_COMBINE,
+    GC_STALL_BATCHED,
     gc_sgd_step,
     gc_status,
     gc_version,

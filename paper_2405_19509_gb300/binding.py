@@ -448,6 +448,7 @@ def gc_set_wait_limit(cycles: int) -> None:
 
 GC_STALL_CHUNK_GRADS = 1
 GC_STALL_COMBINE = 2
+GC_STALL_BATCHED = 4
 
 
 def gc_inject_stall(kernels: int) -> None:

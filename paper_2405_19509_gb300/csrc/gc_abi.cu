@@ -104,7 +104,7 @@ int gc_version(void) { return 100; }
 uint64_t gc_kernel_launches(void) { return g_launches.load(); }
 
 int gc_inject_stall(int kernels) {
-  if (kernels & ~(GC_STALL_CHUNK_GRADS | GC_STALL_COMBINE))
+  if (kernels & ~(GC_STALL_CHUNK_GRADS | GC_STALL_COMBINE | GC_STALL_BATCHED))
     return fail(GC_ERR_ARG, "kernels=0x%x has unknown bits", kernels);
   g_stall.store(kernels);
   return GC_OK;

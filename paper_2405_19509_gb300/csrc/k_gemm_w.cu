@@ -61,6 +61,7 @@ struct WParams {
   __nv_bfloat16* Rt;  // MODE 0 output: planes [2][n_w][N~]
   float* G;           // MODE 1 output: [n_w][N][d]
   long long spin_limit;
+  int stall;  // failure-path test: the TMA producer issues nothing
   uint32_t* status;
 };
 
@@ -112,7 +113,7 @@ __global__ void __launch_bounds__(kThreadsW, 1)
     // ------------------------------------------------------------- producer
     if (lane == 0) {
       uint32_t it = 0;
-      bool ok = true;
+      bool ok = !p.stall;
       for (long long t = blockIdx.x; t < p.num_tiles && ok; t += gridDim.x) {
         int a_x, a_y;  // MODE 0: (k, row0); MODE 1: (col0, row0)
         if (MODE == 0) {
@@ -365,6 +366,7 @@ int launch_chunkgrad_batched(const void* X, const float* y, const float* W, int 
   p.Rt = Rt;
   p.G = G;
   p.spin_limit = wait_limit(kSpinW);
+  p.stall = take_stall(GC_STALL_BATCHED) ? 1 : 0;
   p.status = status;
   CUtensorMap mA, mB;
   // GEMM 1: Z = X W^T, residual epilogue -> R^T planes
@@ -382,6 +384,7 @@ int launch_chunkgrad_batched(const void* X, const float* y, const float* W, int 
   if (rc) return rc;
   rc = map_planes(&mB, Rt, n_w, Ntil);
   if (rc) return rc;
+  p.stall = 0;
   p.num_m_tiles = (d + TM - 1) / TM;
   p.num_tiles = (long long)N * p.num_m_tiles;
   p.nkb = n_c / BK;

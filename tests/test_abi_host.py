@@ -132,7 +132,7 @@ def test_wait_limit_knob_validation():
     gc = _lib()
     assert gc.lib.gc_set_wait_limit(-1) == -1
     assert gc.lib.gc_set_wait_limit(0) == 0
-    assert gc.lib.gc_inject_stall(4) == -1
+    assert gc.lib.gc_inject_stall(8) == -1
     assert gc.lib.gc_inject_stall(0) == 0
 
 

@@ -103,3 +103,29 @@ def test_stall_bit_is_consumed(gc):
     finally:
         gc.gc_inject_stall(0)
         gc.gc_set_wait_limit(0)
+
+
+def test_batched_gemm_stall_times_out_then_recovers(gc):
+    N, n_c, d, n_w = 4, 128, 256, 32
+    g = torch.Generator().manual_seed(9)
+    X = (torch.randn(N * n_c, d, generator=g) / d ** 0.5).to(torch.bfloat16)
+    y = torch.randn(N * n_c, generator=g)
+    W = torch.randn(n_w, d, generator=g)
+    Xd, yd, Wd = X.cuda(), y.cuda(), W.cuda()
+    ws = gc.Workspace()
+    gc.gc_set_wait_limit(SHORT)
+    try:
+        gc.gc_inject_stall(gc.GC_STALL_BATCHED)
+        gc.gc_chunk_grads_batched(Xd, yd, Wd, N, n_c, O.LSQ, ws=ws)
+        torch.cuda.synchronize()
+        _expect_timeout(gc, ws)
+    finally:
+        gc.gc_inject_stall(0)
+        gc.gc_set_wait_limit(0)
+    G = gc.gc_chunk_grads_batched(Xd, yd, Wd, N, n_c, O.LSQ, ws=ws)
+    gc.gc_status(ws)
+    Xf = X.float().numpy().astype(np.float64)
+    for w in (0, 31):
+        ref = O.chunk_gradients(Xf, y.numpy(), W[w].numpy(), N, n_c, O.LSQ)
+        for i in range(N):
+            assert_grad_close(to_np(G[w, i]), ref[i], f"w {w} chunk {i} after recovery")
