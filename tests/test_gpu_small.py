@@ -367,3 +367,40 @@ def test_prepared_plan_direct_solves_for_large_delta(gc):
         r = O.run_pattern(R, order, psi_np[i], N, None, want_transmit=False)
         assert abs(ce[i] - r.coef_err) <= 1e-9 * max(1.0, r.coef_err)
         assert b["est"][i].item() == r.est
+
+
+def test_maximum_delta_and_replication(gc):
+    """delta = 32 (GC_MAX_DELTA) in the cyclic assignment, so every chunk has
+    32 holders (GC_MAX_REPL); l = 2 (l = 8 is covered above: the oracle's
+    per-worker solve at l = 8 with 32 chunks a worker takes seconds per
+    pattern).  Decode, errors and the transmit path against the oracle; the
+    trigger kernel on the same assignment."""
+    rng = np.random.default_rng(21)
+    N = m = 40
+    delta, ell, d = 32, 2, 48
+    order = O.cyclic_order(N, m, delta)
+    R = rng.standard_normal((ell, m))
+    G = rng.standard_normal((N, d)).astype(np.float32)
+    psi = rng.integers(0, delta + 1, size=(12, m)).astype(np.int32)
+    psi[0] = delta
+    psi[1] = 0
+    psi[2] = rng.integers(0, 2, size=m)  # mostly too few copies: approximate
+    Rd, od, pd = dev_tensors(R, order, psi)
+    Gd = torch.from_numpy(G).cuda()
+    res = gc.gc_decode_batch(Rd, ell, od, N, m, delta, pd, Gd)
+    T = gc.gc_encode(Rd, ell, od, N, m, delta, pd[:4].contiguous(), Gd)
+    gh = gc.gc_decode_tx(Rd, ell, m, T, d)
+    for b in range(psi.shape[0]):
+        r = O.run_pattern(R, order, psi[b], N, G.astype(np.float64), want_transmit=b < 4)
+        assert_grad_close(to_np(res["Ghat"][b]), r.ghat, f"delta=32 b={b}")
+        assert abs(res["coef_err"][b].item() - r.coef_err) <= 1e-8 * max(1.0, r.coef_err)
+        assert res["est"][b].item() == r.est
+        if b < 4:
+            assert_grad_close(to_np(gh[b]), r.ghat, f"delta=32 transmit b={b}")
+    from workloads import make_worker_times
+    tau = make_worker_times(m, 64, 22, alpha=5)
+    out = gc.gc_trigger_times(od, N, m, delta, torch.from_numpy(tau).cuda(), ell, 3)
+    Tn, psin, TFn = O.completion_times(order, tau, N, ell, 3)
+    assert np.array_equal(out["T"].cpu().numpy(), Tn)
+    assert np.array_equal(out["psi"].cpu().numpy(), psin)
+    assert np.array_equal(out["T_full"].cpu().numpy(), TFn)
