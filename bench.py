@@ -58,13 +58,17 @@ def parse():
     ap.add_argument("--impl", choices=["gc", "reference"], default="gc")
     ap.add_argument("--ell", type=int, default=2)
     ap.add_argument("--workload", default="logistic",
-                    choices=["logistic", "decode", "sweep", "sgd", "trigger", "batched"],
+                    choices=["logistic", "decode", "sweep", "sgd", "trigger", "batched", "chunkgrad"],
                     help="logistic: the headline step (default).  The others measure the "
                          "remaining configurations, one JSON line each (1 GPU)")
     ap.add_argument("--small", action="store_true",
                     help="with --workload batched: a 134 MB case (N=64, n_c=1024, d=1024: the "
                          "same tile counts, short K for GEMM 1) for profiler captures instead of "
                          "the 8.6 GB one")
+    ap.add_argument("--shape", default=None,
+                    help="with --workload chunkgrad: one case 'dtype,N,n_c,d' (dtype f32 or bf16) "
+                         "timed over --steps calls after --warmup calls, instead of the table of "
+                         "8.6 GB cases")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--min-warm-seconds", type=float, default=1.5,
                     help="keep warming up at least this long (steady clocks, clock samples)")
@@ -319,27 +323,31 @@ def gpu_arm(args, rank, world, local_rank):
     torch.cuda.synchronize()
     serial_ms = [ser_ev[2 * si].elapsed_time(ser_ev[2 * si + 1]) for si in range(len(stages))]
 
-    # two graphs per step, each over two streams: the main stream runs the
-    # long kernels, a high-priority stream runs the small ones beside them
-    # (their blocks then take free SM room before further CTAs of the long
-    # kernels), joined back at the end of the graph:
-    #   g1: chunk gradients (A)        || Algorithm 1, live (D1) then batch (B)
+    # two graphs per step: the main stream runs the long kernels, high-priority
+    # side streams run the small, independent ones beside them (their blocks
+    # then take free SM room before further CTAs of the long kernels), all
+    # joined back at the end of the graph:
+    #   g1: chunk gradients (A)        || Algorithm 1, live (D1) || Algorithm 1, batch (B)
     #   g2: batched decode-combine (C) || live encode / decode / update (D2)
     n0 = gc.gc_kernel_launches()
     cap_stream = torch.cuda.Stream(dev)
-    cap_hi = torch.cuda.Stream(dev, priority=-1)
+    cap_hi = [torch.cuda.Stream(dev, priority=-1) for _ in range(2)]
 
-    def two_streams(main_fns, side_fns):
-        fork, join = torch.cuda.Event(), torch.cuda.Event()
+    def fork_join(main_fns, *side_lists):
+        fork = torch.cuda.Event()
         fork.record(cap_stream)
-        cap_hi.wait_event(fork)
         for f in main_fns:
             f()
-        with torch.cuda.stream(cap_hi):
-            for f in side_fns:
-                f()
-            join.record(cap_hi)
-        cap_stream.wait_event(join)
+        joins = []
+        for side, fns in zip(cap_hi, side_lists):
+            side.wait_event(fork)
+            with torch.cuda.stream(side):
+                for f in fns:
+                    f()
+                joins.append(torch.cuda.Event())
+                joins[-1].record(side)
+        for j in joins:
+            cap_stream.wait_event(j)
 
     g1, g2 = [], []
     for b in range(2):
@@ -347,9 +355,9 @@ def gpu_arm(args, rank, world, local_rank):
         g1.append(torch.cuda.CUDAGraph())
         g2.append(torch.cuda.CUDAGraph())
         with torch.cuda.graph(g1[b], stream=cap_stream):
-            two_streams([stage_a], [stage_d1, stage_b])
+            fork_join([stage_a], [stage_d1], [stage_b])
         with torch.cuda.graph(g2[b], stream=cap_stream):
-            two_streams([stage_c], [stage_d2])
+            fork_join([stage_c], [stage_d2])
         if b == 0:
             launches_per_step = gc.gc_kernel_launches() - n0
     torch.cuda.synchronize()
@@ -780,6 +788,44 @@ def extra_workload(args):
             "config": {"workload": "trigger cyclic N=m=200 delta=8 alpha=delta-l, 10^5 realizations; "
                                    "and 8-regular m=200 alpha=7",
                        "l2": "L2 flushed before each timed call (tau 160 MB)"}})
+    elif args.workload == "chunkgrad":
+        # chunk-gradient bandwidth over row lengths: every case reads 8.6 GB of X
+        # (one pass), from one CTA per row slice up to clusters of 8
+        shapes = [args.shape] if args.shape else [
+            "bf16,64,1024,65536", "bf16,128,1024,32768", "bf16,256,1024,16384", "bf16,512,1024,8192",
+            "f32,64,512,65536", "f32,128,512,32768", "f32,256,512,16384", "f32,512,512,8192"]
+        gen = torch.Generator(device=dev).manual_seed(5)
+        rows = {}
+        for sh in shapes:
+            dt, N, n_c, d = sh.split(",")
+            N, n_c, d = int(N), int(n_c), int(d)
+            tdt = torch.bfloat16 if dt == "bf16" else torch.float32
+            X = torch.empty(N * n_c, d, dtype=tdt, device=dev).normal_(generator=gen).mul_(d ** -0.5)
+            y = torch.sign(torch.randn(N * n_c, device=dev, generator=gen))
+            w = torch.randn(d, device=dev, generator=gen)
+            G = torch.empty(N, d, device=dev)
+            lo = torch.zeros(1, dtype=torch.float64, device=dev)
+            ws = gc.Workspace(dev)
+            t = _time_ms(torch, lambda: gc.gc_chunk_grads(X, y, w, N, n_c, gc.GC_LOGISTIC, G=G,
+                                                          loss_out=lo, ws=ws),
+                         max(1, args.steps if args.shape else 10), warm=max(1, args.warmup if args.shape else 3),
+                         flush=flush if X.numel() * X.element_size() < (256 << 20) else None)
+            gc.gc_status(ws)
+            nbytes = X.numel() * X.element_size() + N * n_c * 4 + N * d * 4
+            rows[sh] = {"ms": t, "GB/s": nbytes / (t / 1e3) / 1e9, "frac_of_hbm": nbytes / (t / 1e3) / 1e9 / hbm}
+            del X, y, w, G, ws
+            torch.cuda.empty_cache()
+        key = shapes[0]
+        line.update({
+            "metric": f"chunk-gradient bandwidth (logistic, {key})", "value": rows[key]["GB/s"], "unit": "GB/s",
+            "per_shape": rows,
+            "roofline": {"kernel": "k_chunkgrad", "bound": "hbm", "unit": "GB/s",
+                         "achieved": rows[key]["GB/s"], "peak": hbm, "frac": rows[key]["frac_of_hbm"],
+                         "note": "bytes = X and y read, G written; k_chunkgrad plus its reduction",
+                         "peak_source": f"{pk_src} hbm_gbs"},
+            "dtype": "bf16 or f32 X (per shape), f32 accumulate",
+            "config": {"workload": "chunk gradients 'dtype,N,n_c,d': " + ", ".join(shapes),
+                       "l2": "inputs larger than L2 (8.6 GB per case), else flushed"}})
     line["gpu_launches_total"] = int(gc.gc_kernel_launches() - n0)
     print(json.dumps(line), flush=True)
 

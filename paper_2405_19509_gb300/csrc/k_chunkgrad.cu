@@ -226,6 +226,18 @@ __device__ __forceinline__ float warp_sum_rows(const float (&p)[R], int lane) {
   return v[0];
 }
 
+// Position in the ring of stages: the stage index and the parity of its phase.
+struct Ring {
+  int s;
+  uint32_t ph;
+  __device__ __forceinline__ void next(int S) {
+    if (++s == S) {
+      s = 0;
+      ph ^= 1u;
+    }
+  }
+};
+
 // NT consumer threads (warps 0 .. NW-1) plus one producer warp (warp NW).
 template <typename T, int CL, int NT, int NVT, int RBM>
 __global__ void __launch_bounds__(NT + 32, 1) k_chunkgrad(CGArgs a) {
@@ -260,6 +272,19 @@ __global__ void __launch_bounds__(NT + 32, 1) k_chunkgrad(CGArgs a) {
     }
     for (int z = 0; z < kZSlots; ++z) mbar_init(&zfull[z], CL);
     fence_mbar_init();
+  }
+  {
+    // Stage bytes the producer never writes -- rows RB..RBM-1, and with TMA
+    // the vectors past the slice -- are zeroed once, so that the consumers
+    // read whole stages without masks (zeros add nothing to either pass).
+    const int vpr = a.ld_s / V;  // 16-byte vectors per stage row
+    const int vfrom = a.use_tma ? nvs : vpr;
+    for (int s = 0; s < a.S; ++s) {
+      uint4* st = reinterpret_cast<uint4*>(stages + (size_t)s * stage_elems);
+      for (int r = 0; r < RBM; ++r)
+        for (int v = (r < a.RB ? vfrom : 0) + tid; v < vpr; v += blockDim.x)
+          st[(size_t)r * vpr + v] = make_uint4(0u, 0u, 0u, 0u);
+    }
   }
   __syncthreads();
   if (CL > 1) cluster_sync_all();  // every peer has started and initialised its barriers
@@ -322,7 +347,8 @@ __global__ void __launch_bounds__(NT + 32, 1) k_chunkgrad(CGArgs a) {
 #pragma unroll
       for (int e = 0; e < V; ++e) acc[u][e] = 0.f;
     const long long first_chunk = r0 / a.n_c;
-    long long cur = -1;
+    long long cur = -1;     // chunk whose gradient acc holds
+    long long next_row = r0;  // first row past chunk `cur` (a batch never straddles chunks: RB | n_c)
     double loss_acc = 0.0;
     auto flush = [&](long long chunk) {
       float* dst = a.parts + ((size_t)q * a.maxt + (size_t)(chunk - first_chunk)) * a.d;
@@ -339,31 +365,28 @@ __global__ void __launch_bounds__(NT + 32, 1) k_chunkgrad(CGArgs a) {
       }
     };
 
-    // x vectors of batch n: raw 16-byte words straight from its stage (zero
-    // for rows past RB and vectors past the slice) ...
-    auto wait_stage = [&](int n) {
-      bounded_wait(&full[n % a.S], (uint32_t)((n / a.S) & 1), abort_flag, a.status, a.spin_limit);
+    // Stage access.  Every stage row is NVT * NT vectors long and the parts
+    // the producer never writes are zero, so the reads need no masks.
+    auto wait_stage = [&](const Ring& g) {
+      bounded_wait(&full[g.s], g.ph, abort_flag, a.status, a.spin_limit);
     };
-    auto from_stage = [&](int n) {
-      const T* st = stages + (n % a.S) * stage_elems;
-      return [=](int r, int u) {
-        const int v = tid + u * NT;
-        return (r < a.RB && v < nvs) ? Vec<T>::load_raw(st + (size_t)r * a.ld_s + v * V)
-                                     : make_uint4(0u, 0u, 0u, 0u);
-      };
+    auto from_stage = [&](const Ring& g) {
+      const T* st = stages + (size_t)g.s * stage_elems + tid * V;
+      const int ld = a.ld_s;
+      return [=](int r, int u) { return Vec<T>::load_raw(st + r * ld + u * NT * V); };
     };
-    // ... or copied to registers once (kept from the dot products to pass 2)
-    auto load_x = [&](int n, uint4 (&xr)[RBM][NVT]) {
-      auto src = from_stage(n);
+    // x of a batch copied to registers once (kept from the dot products to pass 2)
+    auto load_x = [&](const Ring& g, uint4 (&xr)[RBM][NVT]) {
+      auto src = from_stage(g);
 #pragma unroll
       for (int r = 0; r < RBM; ++r)
 #pragma unroll
         for (int u = 0; u < NVT; ++u) xr[r][u] = src(r, u);
     };
-    // hand stage n back to the producer (every lane of the warp is done reading it)
-    auto release = [&](int n) {
+    // hand a stage back to the producer (every lane of the warp is done reading it)
+    auto release = [&](const Ring& g) {
       __syncwarp();
-      if (lane == 0) mbar_arrive_local(&empty[n % a.S]);
+      if (lane == 0) mbar_arrive_local(&empty[g.s]);
     };
     // Dot products of batch n, reduced over the CTA (warp butterfly, then
     // lane-parallel over (warp, row) pairs) and, with clusters, sent to every
@@ -413,6 +436,18 @@ __global__ void __launch_bounds__(NT + 32, 1) k_chunkgrad(CGArgs a) {
         mbar_arrive_remote(&zfull[n % kZSlots], peer);
       }
     };
+    // Cluster sums of batch n once every peer's CTA sums have arrived: lane
+    // p * RBM + r reads peer p's sum of row r, a xor tree adds the peers.
+    auto cluster_sums = [&](int n, float (&z)[RBM]) {
+      bounded_wait(&zfull[n % kZSlots], (uint32_t)((n / kZSlots) & 1), abort_flag, a.status,
+                   a.spin_limit, true);
+      const float* zc = zcl + (n % kZSlots) * CL * RBM;
+      float t = lane < CL * RBM ? zc[lane] : 0.f;
+#pragma unroll
+      for (int o = RBM; o < CL * RBM; o <<= 1) t += __shfl_xor_sync(0xffffffffu, t, o);
+#pragma unroll
+      for (int r = 0; r < RBM; ++r) z[r] = __shfl_sync(0xffffffffu, t, r);
+    };
 
     // y of batch n for lane r < RB, loaded two batches ahead (off the
     // critical path between the dot products and the residuals)
@@ -422,49 +457,43 @@ __global__ void __launch_bounds__(NT + 32, 1) k_chunkgrad(CGArgs a) {
     float y0 = load_y(0), y1 = load_y(1);
     // Residuals, loss and pass 2 (acc += r * x) of batch n from its row sums z.
     auto finish = [&](int n, const float (&z)[RBM], auto&& xget) {
-      const long long chunk = (r0 + (long long)n * a.RB) / a.n_c;
-      if (chunk != cur) {
+      const long long row = r0 + (long long)n * a.RB;
+      if (row >= next_row) {
         if (cur >= 0) flush(cur);
 #pragma unroll
         for (int u = 0; u < NVT; ++u)
 #pragma unroll
           for (int e = 0; e < V; ++e) acc[u][e] = 0.f;
-        cur = chunk;
+        cur = cur < 0 ? first_chunk : cur + 1;
+        next_row = (cur + 1) * a.n_c;
       }
       const float yv = y0;
       y0 = y1;
       y1 = load_y(n + 2);
-      // ---- residuals: lane r takes row r, then broadcast
+      // ---- residuals: lane r < RBM takes row r (rows past RB are zero
+      // padding whose residual multiplies zeros), then a broadcast
+      float zr = z[0];
+#pragma unroll
+      for (int r = 1; r < RBM; ++r) zr = lane == r ? z[r] : zr;
+      const float mine =
+          a.loss == GC_LSQ ? zr - yv : 1.f / (1.f + __expf(-zr)) - 0.5f * (yv + 1.f);
       float res[RBM];
-      {
-        float mine = 0.f;
 #pragma unroll
-        for (int r = 0; r < RBM; ++r) {
-          if (lane == r && r < a.RB) {
-            if (a.loss == GC_LSQ) {
-              mine = z[r] - yv;
-            } else {
-              const float sg = 1.f / (1.f + __expf(-z[r]));
-              mine = sg - 0.5f * (yv + 1.f);
-            }
-          }
-        }
-#pragma unroll
-        for (int r = 0; r < RBM; ++r) res[r] = __shfl_sync(0xffffffffu, mine, r);
-      }
-      // ---- the loss: lane r of warp 0 takes row r (fp32), one fp64 add per batch
+      for (int r = 0; r < RBM; ++r) res[r] = __shfl_sync(0xffffffffu, mine, r);
+      // ---- the loss: lane r < RB of warp 0 takes row r (fp32), one fp64 add per batch
       if (a.want_loss && rank == 0 && warp == 0) {
         float lr = 0.f;
-#pragma unroll
-        for (int r = 0; r < RBM; ++r) {
-          if (r < a.RB && lane == r) {
-            if (a.loss == GC_LSQ) {
-              const float e = z[r] - yv;
-              lr = 0.5f * e * e;
-            } else {
-              const float t = -yv * z[r];  // log(1 + e^t), stable
-              lr = fmaxf(t, 0.f) + log1pf(expf(-fabsf(t)));
-            }
+        if (lane < a.RB) {
+          if (a.loss == GC_LSQ) {
+            const float e = zr - yv;
+            lr = 0.5f * e * e;
+          } else {
+            // log(1 + e^t) = max(t, 0) + log(1 + e^-|t|); the fast intrinsics
+            // are accurate to ~1e-6 absolute per row here (1 + e^-|t| lies in
+            // [1, 2]), far below the loss's 1e-5 relative tolerance, and keep
+            // warp 0 from lagging behind the others at every batch
+            const float t = -yv * zr;
+            lr = fmaxf(t, 0.f) + __logf(1.f + __expf(-fabsf(t)));
           }
         }
 #pragma unroll
@@ -487,55 +516,48 @@ __global__ void __launch_bounds__(NT + 32, 1) k_chunkgrad(CGArgs a) {
     // x in registers when they fit beside acc and w (fp32 rows; not bf16,
     // whose unpacked vectors would spill)
     constexpr bool kXRegs = NVT * RBM * V <= 32;
+    Ring g{0, 0u};
     if (CL == 1 && kXRegs) {
       // One pass over the stage: x stays in registers from the dot products to
       // pass 2, so the stage goes back to the producer as soon as it is read.
-      for (int n = 0; n < nb; ++n) {
+      for (int n = 0; n < nb; ++n, g.next(a.S)) {
         uint4 xr[RBM][NVT];
         float z[RBM];
-        wait_stage(n);
-        load_x(n, xr);
-        release(n);
+        wait_stage(g);
+        load_x(g, xr);
+        release(g);
         auto xget = [&](int r, int u) { return xr[r][u]; };
         dots(n, xget, z);
         finish(n, z, xget);
       }
     } else if (CL == 1) {
-      for (int n = 0; n < nb; ++n) {
+      for (int n = 0; n < nb; ++n, g.next(a.S)) {
         float z[RBM];
-        wait_stage(n);
-        dots(n, from_stage(n), z);
-        finish(n, z, from_stage(n));
-        release(n);
+        wait_stage(g);
+        dots(n, from_stage(g), z);
+        finish(n, z, from_stage(g));
+        release(g);
       }
     } else {
       // Clusters: batch n + 1's dot products and send run before the wait for
       // batch n's cluster sums (software pipelining); pass 2 re-reads the
       // stage, which is handed back afterwards.
       float znext[RBM];
+      Ring g1 = g;
       if (nb > 0) {
-        wait_stage(0);
-        dots(0, from_stage(0), znext);
+        wait_stage(g1);
+        dots(0, from_stage(g1), znext);
+        g1.next(a.S);
       }
-      for (int n = 0; n < nb; ++n) {
-        float z[RBM];
-#pragma unroll
-        for (int r = 0; r < RBM; ++r) z[r] = znext[r];
+      for (int n = 0; n < nb; ++n, g.next(a.S), g1.next(a.S)) {
         if (n + 1 < nb) {
-          wait_stage(n + 1);
-          dots(n + 1, from_stage(n + 1), znext);
+          wait_stage(g1);
+          dots(n + 1, from_stage(g1), znext);
         }
-        bounded_wait(&zfull[n % kZSlots], (uint32_t)((n / kZSlots) & 1), abort_flag, a.status,
-                     a.spin_limit, true);
-        const float* zc = zcl + (n % kZSlots) * CL * RBM;
-#pragma unroll
-        for (int r = 0; r < RBM; ++r) {
-          float t = 0.f;
-          for (int p = 0; p < CL; ++p) t += zc[p * RBM + r];
-          z[r] = t;
-        }
-        finish(n, z, from_stage(n));
-        release(n);
+        float z[RBM];
+        cluster_sums(n, z);
+        finish(n, z, from_stage(g));
+        release(g);
       }
     }
     // the reduction kernel may be scheduled now (it waits for this grid to
@@ -630,13 +652,16 @@ Plan make_plan(int N, int n_c, int d, int x_dtype, bool tma_ok) {
   while (p.CL < 8 && row_bytes / p.CL > max_slice) p.CL *= 2;
   p.use_tma = tma_ok && (row_bytes % 16 == 0) && (d % (p.CL * p.V) == 0);
   p.Wc = p.use_tma ? d / p.CL : (int)align_up((size_t)((d + p.CL - 1) / p.CL), (size_t)p.V);
-  p.ld_s = p.Wc;  // stage row stride (elements)
   const int nv = p.Wc / p.V;  // 16-byte vectors per row slice (<= 2048 by the slice caps)
   p.NT = nv >= 1024 ? 512 : (nv >= 256 ? 256 : 128);
   if (cps == 2 && p.NT == 512) p.NT = 256;  // only when nv <= 1024 (16 KB slices)
   const int need = (nv + p.NT - 1) / p.NT;
   p.NVT = need <= 1 ? 1 : (need <= 2 ? 2 : 4);
-  p.valid = (long long)p.NVT * p.NT >= nv;  // every vector of the slice has a thread
+  // every vector of the slice has a thread, and (NT, NVT) is an instantiated shape:
+  // NT = 128 with NVT <= 2, NT = 256 or 512 with NVT <= 4
+  p.valid = (long long)p.NVT * p.NT >= nv && (p.NT > 128 || p.NVT <= 2);
+  // stage row stride: one vector per (thread, u), so reads need no bounds
+  p.ld_s = p.NVT * p.NT * p.V;
   p.RBM = p.NVT >= 4 ? 2 : 4;
   p.RB = p.RBM;
   while (p.RB > 1 && n_c % p.RB != 0) p.RB /= 2;
@@ -696,8 +721,10 @@ int dispatch_nt(const Plan& p, const CGArgs& a, cudaStream_t s) {
   }
   if (p.NT == 256) {
     if (p.NVT == 4) return launch_one<T, CL, 256, 4, 2>(p, a, s);
+    if (p.NVT == 2) return launch_one<T, CL, 256, 2, 4>(p, a, s);
     return launch_one<T, CL, 256, 1, 4>(p, a, s);
   }
+  if (p.NVT == 2) return launch_one<T, CL, 128, 2, 4>(p, a, s);
   return launch_one<T, CL, 128, 1, 4>(p, a, s);
 }
 
@@ -744,8 +771,10 @@ int occ_nt(const Plan& p) {
   }
   if (p.NT == 256) {
     if (p.NVT == 4) return occ_one<T, CL, 256, 4, 2>(p);
+    if (p.NVT == 2) return occ_one<T, CL, 256, 2, 4>(p);
     return occ_one<T, CL, 256, 1, 4>(p);
   }
+  if (p.NVT == 2) return occ_one<T, CL, 128, 2, 4>(p);
   return occ_one<T, CL, 128, 1, 4>(p);
 }
 template <typename T>
