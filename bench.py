@@ -64,7 +64,8 @@ def parse():
     ap.add_argument("--small", action="store_true",
                     help="with --workload batched: a 134 MB case (N=64, n_c=1024, d=1024: the "
                          "same tile counts, short K for GEMM 1) for profiler captures instead of "
-                         "the 8.6 GB one")
+                         "the 8.6 GB one; with --workload sweep: given chunk gradients instead of "
+                         "X (the decode-combine alone, for profiler captures)")
     ap.add_argument("--shape", default=None,
                     help="with --workload chunkgrad: one case 'dtype,N,n_c,d' (dtype f32 or bf16) "
                          "timed over --steps calls after --warmup calls, instead of the table of "
@@ -620,13 +621,18 @@ def extra_workload(args):
     elif args.workload == "sweep":
         cfg = get("mse_sweep")
         N, m, delta, d, npat = cfg.N, cfg.m, cfg.delta, cfg.d, cfg.npat
-        data = make_data(cfg, dev)
-        G = torch.empty(N, d, device=dev)
-        wsA = gc.Workspace(dev)
-        t_cg = _time_ms(torch, lambda: gc.gc_chunk_grads(data["X"], data["y"], data["w"], N, cfg.n_c,
-                                                         gc.GC_LSQ, G=G, ws=wsA), 5)
-        del data
-        torch.cuda.empty_cache()
+        if args.small:
+            # profiler captures of the decode-combine: given chunk gradients, no X
+            G = make_chunk_grads(cfg, dev)
+            t_cg = float("nan")
+        else:
+            data = make_data(cfg, dev)
+            G = torch.empty(N, d, device=dev)
+            wsA = gc.Workspace(dev)
+            t_cg = _time_ms(torch, lambda: gc.gc_chunk_grads(data["X"], data["y"], data["w"], N, cfg.n_c,
+                                                             gc.GC_LSQ, G=G, ws=wsA), 5)
+            del data
+            torch.cuda.empty_cache()
         _, order, _ = gc.gc_make_assignment(N, m, delta)
         Rd = torch.from_numpy(make_R(cfg, ell)).to(dev)
         od = torch.from_numpy(order).to(dev)

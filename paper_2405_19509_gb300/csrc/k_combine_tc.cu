@@ -60,11 +60,14 @@ constexpr int OUT_BUF = 32 * 32 * 4;                 // one 32 x 32 fp32 store b
 constexpr int A_STAGE = 2 * A_PLANE;  // 32 KB
 constexpr int kBresStages = 2;        // A ring stages of the BRES shape
 constexpr int B_TILE = 2 * B_PLANE;   // 64 KB
-template <int STAGES, int EPI, bool BRES>
+// NKBR > 0: B resident (NKBR k-blocks of the current n-tile), A streamed.
+// OUT: output staging boxes for TMA stores of Ghat (none in MSE-only shapes).
+template <int STAGES, int EPI, int NKBR, bool OUT>
 struct Shape {
+  static constexpr bool BRES = NKBR > 0;
   static constexpr int THREADS = 64 + 32 * EPI;
-  static constexpr int OUT_BYTES = EPI * 2 * OUT_BUF;  // 2 staging boxes per epilogue warp
-  static constexpr int RING = BRES ? STAGES * A_STAGE + B_TILE : STAGES * STAGE_BYTES;
+  static constexpr int OUT_BYTES = OUT ? EPI * 2 * OUT_BUF : 0;  // 2 staging boxes per epilogue warp
+  static constexpr int RING = BRES ? STAGES * A_STAGE + NKBR * B_TILE : STAGES * STAGE_BYTES;
   static constexpr size_t SMEM = (size_t)RING + OUT_BYTES + 1024 + 256;
   static_assert(SMEM <= 232448, "shared memory per CTA");
 };
@@ -200,15 +203,16 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
   for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(r[j]);
 }
 
-template <int STAGES, int EPI, bool BRES>
+template <int STAGES, int EPI, int NKBR, bool OUT>
 __global__ void __launch_bounds__(64 + 32 * EPI, 1)
     k_combine_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                  const __grid_constant__ CUtensorMap tmC, Params p) {
-  using Sh = Shape<STAGES, EPI, BRES>;
+  using Sh = Shape<STAGES, EPI, NKBR, OUT>;
+  constexpr bool BRES = Sh::BRES;
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
-  uint8_t* bres = smem + STAGES * A_STAGE;                       // BRES: resident B tile
+  uint8_t* bres = smem + STAGES * A_STAGE;                       // BRES: resident B k-blocks
   float* outbuf = reinterpret_cast<float*>(smem + Sh::RING);     // 1024-aligned
   uint64_t* full = reinterpret_cast<uint64_t*>(smem + Sh::RING + Sh::OUT_BYTES);
   uint64_t* empty = full + STAGES;
@@ -275,18 +279,23 @@ __global__ void __launch_bounds__(64 + 32 * EPI, 1)
           if (nb_loads > 0 &&
               !mbar_wait(bempty, (nb_loads - 1) & 1, abort_flag, p.status, p.spin_limit))
             break;
-          mbar_expect_tx(bfull, B_TILE);
-          tma_load_3d(bres, &tmB, 0, nt * BN, 0, bfull);
+          mbar_expect_tx(bfull, NKBR * B_TILE);
+          for (int kb = 0; kb < NKBR; ++kb)
+            tma_load_3d(bres + kb * B_TILE, &tmB, kb * BK, nt * BN, 0, bfull);
           cur_nt = nt;
           ++nb_loads;
         }
-        const int s = it % STAGES;
-        const uint32_t ph = (it / STAGES) & 1;
-        if (!mbar_wait(&empty[s], ph ^ 1, abort_flag, p.status, p.spin_limit)) break;
-        uint8_t* st = smem + s * A_STAGE;
-        mbar_expect_tx(&full[s], A_STAGE);
-        tma_load_3d(st, &tmA, 0, mt * BM, 0, &full[s]);
-        ++it;
+        for (int kb = 0; kb < NKBR && ok; ++kb, ++it) {
+          const int s = it % STAGES;
+          const uint32_t ph = (it / STAGES) & 1;
+          if (!mbar_wait(&empty[s], ph ^ 1, abort_flag, p.status, p.spin_limit)) {
+            ok = false;
+            break;
+          }
+          uint8_t* st = smem + s * A_STAGE;
+          mbar_expect_tx(&full[s], A_STAGE);
+          tma_load_3d(st, &tmA, kb * BK, mt * BM, 0, &full[s]);
+        }
       }
       // drain: every issued copy has landed before the CTA may exit
       volatile int no_abort = 0;
@@ -333,21 +342,29 @@ __global__ void __launch_bounds__(64 + 32 * EPI, 1)
         const int ab = tile_it & 1;
         if (!mbar_wait(&tempty[ab], ((tile_it >> 1) & 1) ^ 1, abort_flag, p.status, p.spin_limit))
           break;
-        const int s = it % STAGES;
-        if (!mbar_wait(&full[s], (it / STAGES) & 1, abort_flag, p.status, p.spin_limit)) break;
-        fence_after();
         const uint32_t d_tmem = tmem_base + (uint32_t)(ab * BN);
-        const uint32_t a_hi = smem_u32(smem + s * A_STAGE), a_lo = a_hi + A_PLANE;
-        const uint32_t b_hi = smem_u32(bres), b_lo = b_hi + B_PLANE;
-        const int nks = p.K >= BK ? BK / 16 : (p.K + 15) / 16;
-        for (int ks = 0; ks < nks; ++ks) {
-          const uint32_t off = ks * 32;
-          mma_bf16(d_tmem, sdesc(a_hi + off), sdesc(b_hi + off), ks > 0 ? 1u : 0u);
-          mma_bf16(d_tmem, sdesc(a_hi + off), sdesc(b_lo + off), 1u);
-          mma_bf16(d_tmem, sdesc(a_lo + off), sdesc(b_hi + off), 1u);
+        bool ok = true;
+        for (int kb = 0; kb < NKBR; ++kb, ++it) {
+          const int s = it % STAGES;
+          if (!mbar_wait(&full[s], (it / STAGES) & 1, abort_flag, p.status, p.spin_limit)) {
+            ok = false;
+            break;
+          }
+          fence_after();
+          const uint32_t a_hi = smem_u32(smem + s * A_STAGE), a_lo = a_hi + A_PLANE;
+          const uint32_t b_hi = smem_u32(bres + kb * B_TILE), b_lo = b_hi + B_PLANE;
+          const int rem = p.K - kb * BK;
+          const int nks = rem >= BK ? BK / 16 : (rem + 15) / 16;
+          for (int ks = 0; ks < nks; ++ks) {
+            const uint32_t off = ks * 32;
+            const uint32_t acc = (kb > 0 || ks > 0) ? 1u : 0u;
+            mma_bf16(d_tmem, sdesc(a_hi + off), sdesc(b_hi + off), acc);
+            mma_bf16(d_tmem, sdesc(a_hi + off), sdesc(b_lo + off), 1u);
+            mma_bf16(d_tmem, sdesc(a_lo + off), sdesc(b_hi + off), 1u);
+          }
+          mma_commit(&empty[s]);
         }
-        mma_commit(&empty[s]);
-        ++it;
+        if (!ok) break;
         mma_commit(&tfull[ab]);
         // last tile on this B tile: hand it back once these MMAs complete
         const bool last_on_b = t + t_step >= t_last || (int)((t + t_step) / p.num_m_tiles) != nt;
@@ -442,7 +459,7 @@ __global__ void __launch_bounds__(64 + 32 * EPI, 1)
         __syncwarp();
         tmem_ld32(taddr + cc, v);  // warp-collective: every lane, every chunk
         const int c0 = n0 + cc;
-        if (p.tma_store && c0 < p.L) {
+        if (OUT && p.tma_store && c0 < p.L) {
           // stage the 32 x 32 box (row = lane) with the 128-byte swizzle, then one TMA store
           float* buf = wbuf + (chunk_it & 1) * (OUT_BUF / 4);
           if (lane == 0) bulk_wait_read1();  // the store that used this buffer has read it
@@ -679,13 +696,13 @@ int make_map(CUtensorMap* map, const void* base, int rows, int Kp, int box_rows)
 
 }  // namespace tc
 
-template <int STAGES, int EPI, bool BRES>
+template <int STAGES, int EPI, int NKBR, bool OUT>
 int launch_tc(int grid, const CUtensorMap& mA, const CUtensorMap& mB, const CUtensorMap& mC,
               const tc::Params& p, cudaStream_t s) {
-  using Sh = tc::Shape<STAGES, EPI, BRES>;
+  using Sh = tc::Shape<STAGES, EPI, NKBR, OUT>;
   static bool attr_set = false;
   if (!attr_set) {
-    cudaError_t e = cudaFuncSetAttribute(tc::k_combine_tc<STAGES, EPI, BRES>,
+    cudaError_t e = cudaFuncSetAttribute(tc::k_combine_tc<STAGES, EPI, NKBR, OUT>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, (int)Sh::SMEM);
     if (e != cudaSuccess) return cuda_check(e, "cudaFuncSetAttribute(k_combine_tc)");
     attr_set = true;
@@ -700,7 +717,7 @@ int launch_tc(int grid, const CUtensorMap& mA, const CUtensorMap& mB, const CUte
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  cudaError_t e = cudaLaunchKernelEx(&cfg, tc::k_combine_tc<STAGES, EPI, BRES>, mA, mB, mC, p);
+  cudaError_t e = cudaLaunchKernelEx(&cfg, tc::k_combine_tc<STAGES, EPI, NKBR, OUT>, mA, mB, mC, p);
   if (e != cudaSuccess) return cuda_check(e, "cudaLaunchKernelEx(k_combine_tc)");
   count_launches(1);
   return cuda_check(cudaGetLastError(), "k_combine_tc");
@@ -780,12 +797,18 @@ int launch_apply(const __nv_bfloat16* Cs, const float* G, int N, int ell, int np
   p.status = status;
   p.spin_limit = wait_limit(kSpin);
   p.stall = take_stall(GC_STALL_COMBINE) ? 1 : 0;
+  // shapes: one K block -> B resident, A streamed, output staged (write-bound);
+  // two K blocks and no output (the MSE sweep) -> B resident over a 3-stage
+  // A ring, so the next A tiles load while the MMAs run; else the 2-stage
+  // ring of A and B tiles
   const bool one_block = p.nkb == 1;
-  p.parts_per_row = nnt * (one_block ? 2 : 1);
+  const bool two_res = p.nkb == 2 && !Ghat;
+  p.parts_per_row = nnt * ((one_block || two_res) ? 2 : 1);
   const int sms = device_sm_count();
   const int grid = (int)std::min<long long>(p.num_tiles, sms);
-  rc = one_block ? launch_tc<kBresStages, 8, true>(grid, mA, mB, mC, p, s)
-                 : launch_tc<2, 4, false>(grid, mA, mB, mC, p, s);
+  rc = one_block ? launch_tc<kBresStages, 8, 1, true>(grid, mA, mB, mC, p, s)
+       : two_res ? launch_tc<3, 8, 2, false>(grid, mA, mB, mC, p, s)
+                 : launch_tc<2, 4, 0, true>(grid, mA, mB, mC, p, s);
   if (rc) return rc;
   if (grad_mse) {
     cudaLaunchConfig_t cfg{};
