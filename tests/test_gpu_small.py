@@ -189,7 +189,8 @@ def test_large_ell_and_explicit_uneven(gc):
     (16384, 8, 3, torch.float32, 0),     # cluster of 2
     (32768, 4, 2, torch.float32, 1),     # cluster of 4
     (65536, 4, 2, torch.float32, 0),     # cluster of 8
-    (65536, 8, 2, torch.bfloat16, 0),    # bf16, cluster of 8
+    (65536, 8, 2, torch.bfloat16, 0),    # bf16, cluster of 4 with 32 KB slices
+    (131072, 2, 2, torch.bfloat16, 1),   # bf16, cluster of 8 with 32 KB slices
     (16384, 3, 3, torch.float32, 1),     # cluster of 2, one row per stage (3 rows a chunk)
     (32768, 6, 2, torch.bfloat16, 1),    # bf16 cluster of 4, two rows per stage
     (4000, 5, 3, torch.bfloat16, 0),     # bf16, 256 threads x 2 vectors, slice shorter than the stage row
