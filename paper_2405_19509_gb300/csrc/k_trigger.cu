@@ -33,6 +33,11 @@ namespace gc {
 namespace {
 
 constexpr int kWarpsPerBlock = 4;
+// Resident blocks per SM the kernel is compiled for and the grid is sized
+// to: 12 (at most 40 registers a thread) while the 2 x ELL running minima
+// fit, else 8 (64 registers).  Many warps per SM keep the fp64 products and
+// the tau loads of many realizations in flight.
+constexpr int blocks_per_sm(int ell) { return ell <= 3 ? 12 : 8; }
 
 // k-th smallest (1-based, 1 <= k <= n) of n keys in shared memory, by warp.
 __device__ unsigned long long warp_select(const unsigned long long* keys, int n, int k, int lane) {
@@ -67,27 +72,43 @@ __device__ unsigned long long warp_select(const unsigned long long* keys, int n,
 // Keep the ELL smallest keys seen so far (ascending).  Keys are the bit
 // patterns of non-negative doubles, which order like the values, so the
 // comparisons are integer ones (GB300's fp64 pipe is 1/64 of fp32; only the
-// multiplies that define the times stay in fp64).
+// multiplies that define the times stay in fp64).  Branch-free with static
+// indices, so the array stays in registers: position k of the result is
+// b[k-1] when v goes before it, else min(v, b[k]).
 template <int ELL>
 __device__ __forceinline__ void insert_smallest(unsigned long long (&b)[ELL], unsigned long long v) {
-  if (!(v < b[ELL - 1])) return;
-  int q = ELL - 1;
-  while (q > 0 && b[q - 1] > v) {
-    b[q] = b[q - 1];
-    --q;
-  }
-  b[q] = v;
+#pragma unroll
+  for (int k = ELL - 1; k > 0; --k) b[k] = v < b[k - 1] ? b[k - 1] : (v < b[k] ? v : b[k]);
+  b[0] = v < b[0] ? v : b[0];
 }
 __device__ __forceinline__ unsigned long long dbits(double x) {
   return (unsigned long long)__double_as_longlong(x);
 }
+// isfinite on the bit pattern (integer ops; a double compare would use the fp64 pipe)
+__device__ __forceinline__ bool finite_bits(double x) {
+  return (dbits(x) & 0x7ff0000000000000ull) != 0x7ff0000000000000ull;
+}
+// A float near a finite non-negative double, from its bits (integer ops; the
+// mantissa is truncated, magnitudes outside the float range are clamped).
+// Only a starting point for an exact search, so its accuracy is not critical.
+__device__ __forceinline__ float approx_float(double x) {
+  const unsigned long long b = dbits(x);
+  const int e = (int)((b >> 52) & 0x7ff) - 1023 + 127;
+  if (e <= 0) return 0.f;
+  if (e >= 255) return 3.0e38f;
+  return __uint_as_float(((unsigned)e << 23) | (unsigned)((b >> 29) & 0x7fffffu));
+}
 
 template <int ELL>
-__global__ void __launch_bounds__(32 * kWarpsPerBlock)
+__global__ void __launch_bounds__(32 * kWarpsPerBlock, blocks_per_sm(ELL))
     k_trigger(const int32_t* __restrict__ order, Holders h, int N, int m, int delta,
               const double* __restrict__ tau, long long nsim, int theta, double* __restrict__ T_out,
               int32_t* __restrict__ psi_out, double* __restrict__ Tfull_out) {
   extern __shared__ unsigned long long s_dyn[];
+  // the integers 0..GC_MAX_REPL as doubles: the slot factors (p + 1) of the
+  // completion times are read here rather than converted per product (an
+  // int -> double conversion runs on the fp64 pipe, 1/64 of fp32 on GB300)
+  __shared__ double s_kd[GC_MAX_REPL + 1];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   // per block: delta_j of every worker; per warp: the finishing time of every
   // worker (m keys) and, for theta > 0, 2 N ELL completion keys
@@ -102,6 +123,7 @@ __global__ void __launch_bounds__(32 * kWarpsPerBlock)
     for (int p = 0; p < delta; ++p) c += order[(size_t)j * delta + p] >= 0;
     s_dj[j] = (int8_t)c;
   }
+  for (int c = threadIdx.x; c <= GC_MAX_REPL; c += blockDim.x) s_kd[c] = (double)c;
   __syncthreads();
   const int n = N * ELL;
   const int kth = n - theta;
@@ -112,7 +134,7 @@ __global__ void __launch_bounds__(32 * kWarpsPerBlock)
     // each worker's finishing time delta_j tau_j (+inf for a failed worker)
     for (int j = lane; j < m; j += 32) {
       const double tj = tr[j];
-      fin[j] = isfinite(tj) ? dbits((double)s_dj[j] * tj) : kInf;
+      fin[j] = finite_bits(tj) ? dbits(s_kd[s_dj[j]] * tj) : kInf;
     }
     __syncwarp();
     // theta = 0: the order statistic is the largest of the N ell values, i.e.
@@ -127,8 +149,8 @@ __global__ void __launch_bounds__(32 * kWarpsPerBlock)
         const int j = h.w[(size_t)i * GC_MAX_REPL + q];
         const int p = h.p[(size_t)i * GC_MAX_REPL + q];
         const double tj = tr[j];
-        if (isfinite(tj)) {
-          insert_smallest<ELL>(b, dbits((double)(p + 1) * tj));
+        if (finite_bits(tj)) {
+          insert_smallest<ELL>(b, dbits(s_kd[p + 1] * tj));
           insert_smallest<ELL>(bf, fin[j]);
         }
       }
@@ -165,11 +187,19 @@ __global__ void __launch_bounds__(32 * kWarpsPerBlock)
     }
     if (psi_out)
       for (int j = lane; j < m; j += 32) {
-        // slots finish in order: count p while p tau_j <= T
+        // slots finish in order: psi_j is the largest c <= delta_j with
+        // c tau_j <= T (the products are monotone in c).  An fp32 estimate of
+        // T / tau_j is corrected with the exact double products, so that
+        // typically two of them are formed instead of one per slot.
         const double tj = tr[j];
+        const int dj = s_dj[j];
         int c = 0;
-        if (isfinite(tj))
-          while (c < s_dj[j] && dbits((double)(c + 1) * tj) <= Tb) ++c;
+        if (finite_bits(tj) && dj > 0) {
+          const float q = __fdividef(approx_float(T), approx_float(tj));
+          c = q >= (float)dj ? dj : (q > 0.f ? (int)q : 0);
+          while (c > 0 && dbits(s_kd[c] * tj) > Tb) --c;
+          while (c < dj && dbits(s_kd[c + 1] * tj) <= Tb) ++c;
+        }
         psi_out[r * m + j] = c;
       }
     __syncwarp();
@@ -187,7 +217,8 @@ int launch_one(const int32_t* order, Holders h, int N, int m, int delta, const d
     if (e != cudaSuccess) return cuda_check(e, "cudaFuncSetAttribute(k_trigger)");
   }
   const long long blocks_needed = (nsim + kWarpsPerBlock - 1) / kWarpsPerBlock;
-  const int blocks = (int)std::min<long long>(blocks_needed, (long long)device_sm_count() * 16);
+  const int blocks =
+      (int)std::min<long long>(blocks_needed, (long long)device_sm_count() * blocks_per_sm(ELL));
   k_trigger<ELL><<<blocks, 32 * kWarpsPerBlock, smem, s>>>(order, h, N, m, delta, tau, nsim, theta,
                                                            T, psi, TF);
   count_launches(1);
