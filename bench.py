@@ -645,6 +645,21 @@ def extra_workload(args):
         Kp = -(-N * ell // 64) * 64
         useful = 2.0 * npat * ell * (N * ell) * L
         issued = 3 * 2.0 * npat * ell * Kp * L
+        # eq. (2) encode on the same G for 8 patterns (A4 alone, from Algorithm
+        # 1's worker coefficients): per pattern G read once and T written once
+        del Gh
+        torch.cuda.empty_cache()
+        ne = 8
+        pe = pd[:ne].contiguous()
+        E = gc.gc_find_encoding_coeff(Rd, ell, od, N, m, delta, pe, E=True, C=False, delta_out=False,
+                                      coef_err=False, est=False)["E"]
+        T = torch.empty(ne, m, L, device=dev)
+        t_enc = _time_ms(torch, lambda: gc.gc_encode_with_coeffs(E, ell, od, N, m, delta, pe, G, T=T), 3)
+        enc_bytes = ne * (N * d * 4 + m * L * 4)
+        line["encode"] = {"patterns": ne, "ms": t_enc, "GB/s": enc_bytes / (t_enc / 1e3) / 1e9,
+                          "frac_of_hbm": enc_bytes / (t_enc / 1e3) / 1e9 / hbm,
+                          "note": "algorithmic bytes per pattern: G read (N d 4) + T written (m L 4)"}
+        del T
         line.update({
             "metric": f"decoded gradients/sec (m=N=256, delta=16, d=2^20, 4096 patterns, l={ell})",
             "value": npat / ((t_plan + t_apply) / 1e3), "unit": "decoded gradients/s",

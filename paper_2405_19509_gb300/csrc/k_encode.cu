@@ -3,54 +3,119 @@
 //
 // All three are HBM-bound streaming kernels with coalesced accesses along the
 // block coordinate c (consecutive threads, consecutive columns).
+#include <algorithm>
+
 #include "gc_internal.cuh"
 
 namespace gc {
 
 // T[b][j][c] = sum_{p < psi[b][j]} sum_k E[b][j][p][k] * g_{order[j][p]}[k*L + c]
-// (g zero past d).  Block = (column tile, worker j, pattern b); worker j's
-// coefficients and chunk list are staged in shared memory (fp32) once per
-// block -- delta * (ell + 1) words of dynamic shared memory, so the kernel
-// still fits beside a resident kernel that holds nearly all of an SM's.
-__global__ void k_encode(const double* __restrict__ E, const int32_t* __restrict__ order,
-                         const int32_t* __restrict__ psi, int N, int m, int delta, int ell,
-                         int npat, const float* __restrict__ G, int d, int L,
-                         float* __restrict__ T) {
+// (g zero past d).  Block = (column stripe, worker j, group of up to
+// kEncPats patterns).  The patterns share worker j's chunk list, so each
+// thread loads g_{order[j][p]}[k*L + c] once per slot p and feeds it to
+// every pattern of the group that processed slot p (kEncPats accumulators)
+// instead of once per pattern; threads take V consecutive columns (16-byte
+// loads when rows are 16-byte aligned) and stride over the block's columns,
+// so the staging of the group's coefficients (fp32) and processed counts in
+// shared memory -- kEncPats * (delta * ell + 1) + delta words, small enough to
+// fit beside a resident kernel that holds nearly all of an SM's -- is paid
+// once per block, not once per 256 columns.
+constexpr int kEncPats = 8;
+constexpr int kEncThreads = 256;
+template <int V>
+__global__ void __launch_bounds__(kEncThreads)
+    k_encode(const double* __restrict__ E, const int32_t* __restrict__ order,
+             const int32_t* __restrict__ psi, int N, int m, int delta, int ell, int npat,
+             const float* __restrict__ G, int d, int L, float* __restrict__ T) {
   extern __shared__ float s_dyn[];
-  float* s_e = s_dyn;                                          // [delta * ell]
-  int* s_chunk = reinterpret_cast<int*>(s_dyn + delta * ell);  // [delta]
-  const int j = blockIdx.y, b = blockIdx.z;
-  int np = psi[(size_t)b * m + j];
-  np = np < 0 ? 0 : (np > delta ? delta : np);  // bad values are flagged by the solve
-  const double* Ej = E + ((size_t)b * m + j) * delta * ell;
-  for (int t = threadIdx.x; t < np * ell; t += blockDim.x) s_e[t] = (float)Ej[t];
-  for (int t = threadIdx.x; t < np; t += blockDim.x) s_chunk[t] = order[(size_t)j * delta + t];
+  const int j = blockIdx.y, b0 = blockIdx.z * kEncPats;
+  const int nb = min(kEncPats, npat - b0);
+  const int de = delta * ell;
+  float* s_e = s_dyn;                                                // [nb][delta * ell]
+  int* s_np = reinterpret_cast<int*>(s_dyn + kEncPats * de);         // [kEncPats]
+  int* s_chunk = s_np + kEncPats;                                    // [delta]
+  if (threadIdx.x < kEncPats) {
+    int np = 0;
+    if ((int)threadIdx.x < nb) {
+      np = psi[(size_t)(b0 + threadIdx.x) * m + j];
+      np = np < 0 ? 0 : (np > delta ? delta : np);  // bad values are flagged by the solve
+    }
+    s_np[threadIdx.x] = np;
+  }
+  for (int t = threadIdx.x; t < nb * de; t += blockDim.x) {
+    const int bb = t / de, r = t - bb * de;
+    s_e[t] = (float)E[((size_t)(b0 + bb) * m + j) * de + r];
+  }
+  for (int t = threadIdx.x; t < delta; t += blockDim.x) s_chunk[t] = order[(size_t)j * delta + t];
   __syncthreads();
-  const int c = blockIdx.x * blockDim.x + threadIdx.x;
-  if (c >= L) return;
-  float acc = 0.f;
-#pragma unroll 4
-  for (int p = 0; p < np; ++p) {
-    const int i = s_chunk[p];
-    if (i < 0 || i >= N) continue;
-    const float* gi = G + (size_t)i * d;
-    for (int k = 0; k < ell; ++k) {
-      const int col = k * L + c;
-      if (col < d) acc = fmaf(s_e[p * ell + k], __ldg(gi + col), acc);
+  int pmax = 0;
+#pragma unroll
+  for (int bb = 0; bb < kEncPats; ++bb) pmax = max(pmax, s_np[bb]);
+  for (int c = (blockIdx.x * kEncThreads + threadIdx.x) * V; c < L; c += gridDim.x * kEncThreads * V) {
+    float acc[kEncPats][V];
+#pragma unroll
+    for (int bb = 0; bb < kEncPats; ++bb)
+#pragma unroll
+      for (int v = 0; v < V; ++v) acc[bb][v] = 0.f;
+    for (int p = 0; p < pmax; ++p) {
+      const int i = s_chunk[p];
+      if (i < 0 || i >= N) continue;
+      const float* gi = G + (size_t)i * d;
+      for (int k = 0; k < ell; ++k) {
+        const int col = k * L + c;
+        float g[V];
+        if (V == 4 && col + 3 < d) {
+          const float4 q = __ldg(reinterpret_cast<const float4*>(gi + col));
+          g[0] = q.x; g[V > 1 ? 1 : 0] = q.y; g[V > 2 ? 2 : 0] = q.z; g[V > 3 ? 3 : 0] = q.w;
+        } else {
+#pragma unroll
+          for (int v = 0; v < V; ++v) g[v] = (c + v < L && col + v < d) ? __ldg(gi + col + v) : 0.f;
+        }
+#pragma unroll
+        for (int bb = 0; bb < kEncPats; ++bb)
+          if (p < s_np[bb]) {
+            const float e = s_e[bb * de + p * ell + k];
+#pragma unroll
+            for (int v = 0; v < V; ++v) acc[bb][v] = fmaf(e, g[v], acc[bb][v]);
+          }
+      }
+    }
+#pragma unroll
+    for (int bb = 0; bb < kEncPats; ++bb) {
+      if (bb >= nb) break;
+      float* Tr = T + ((size_t)(b0 + bb) * m + j) * L + c;
+      if (V == 4 && c + 3 < L) {
+        *reinterpret_cast<float4*>(Tr) = make_float4(acc[bb][0], acc[bb][V > 1 ? 1 : 0],
+                                                     acc[bb][V > 2 ? 2 : 0], acc[bb][V > 3 ? 3 : 0]);
+      } else {
+#pragma unroll
+        for (int v = 0; v < V; ++v)
+          if (c + v < L) Tr[v] = acc[bb][v];
+      }
     }
   }
-  T[((size_t)b * m + j) * L + c] = acc;
 }
 
 int launch_encode(const double* E, const int32_t* order, const int32_t* psi, int N, int m,
                   int delta, int ell, int npat, const float* G, int d, float* T, cudaStream_t s) {
   const int L = (d + ell - 1) / ell;
   if ((long long)npat * m * L == 0) return GC_OK;
-  if (npat > 65535 || m > 65535) return fail(GC_ERR_UNSUPPORTED, "encode grid: npat and m <= 65535");
-  const int threads = 256;
-  dim3 grid((L + threads - 1) / threads, m, npat);
-  const size_t smem = (size_t)delta * (ell + 1) * sizeof(float);
-  k_encode<<<grid, threads, smem, s>>>(E, order, psi, N, m, delta, ell, npat, G, d, L, T);
+  const int groups = (npat + kEncPats - 1) / kEncPats;
+  if (groups > 65535 || m > 65535) return fail(GC_ERR_UNSUPPORTED, "encode grid: npat / 8 and m <= 65535");
+  // 16-byte column vectors when every row start is 16-byte aligned
+  const bool vec = d % 4 == 0 && L % 4 == 0 && reinterpret_cast<uintptr_t>(G) % 16 == 0 &&
+                   reinterpret_cast<uintptr_t>(T) % 16 == 0;
+  const int V = vec ? 4 : 1;
+  const long long stripes = ((long long)L + (long long)kEncThreads * V - 1) / ((long long)kEncThreads * V);
+  // enough blocks for a few waves; each block strides over the rest of its row
+  const long long want = std::max<long long>(1, (long long)device_sm_count() * 32 / ((long long)m * groups));
+  const int gx = (int)std::max<long long>(1, std::min<long long>(stripes, want));
+  dim3 grid(gx, m, groups);
+  const size_t smem = ((size_t)kEncPats * delta * ell + kEncPats + delta) * sizeof(float);
+  if (vec)
+    k_encode<4><<<grid, kEncThreads, smem, s>>>(E, order, psi, N, m, delta, ell, npat, G, d, L, T);
+  else
+    k_encode<1><<<grid, kEncThreads, smem, s>>>(E, order, psi, N, m, delta, ell, npat, G, d, L, T);
   count_launches(1);
   return cuda_check(cudaGetLastError(), "k_encode");
 }
