@@ -299,6 +299,37 @@ def test_encode_with_coeffs_matches_encode(gc):
             assert rel_inf(to_np(T2[b]), r.T) <= 1e-4
 
 
+@pytest.mark.parametrize("explicit", [False, True])
+@pytest.mark.parametrize("npat", [1, 3])
+def test_encode_long_rows(gc, explicit, npat):
+    """Eq. (2) on long rows (L = 2^18, 16-byte column vectors, blocks striding
+    over many column stripes) for one pattern and for a group of three, with
+    the cyclic order and with an explicit order of disjoint chunk lists (64
+    chunks, one copy each): the transmissions equal the oracle's."""
+    ell, d, delta = 2, 1 << 19, 4
+    rng = np.random.default_rng(31 + 2 * npat + explicit)
+    if explicit:
+        N, m = 64, 16
+        order = np.arange(N, dtype=np.int32).reshape(m, delta)
+    else:
+        N = m = 16
+        order = O.cyclic_order(N, m, delta)
+    R = rng.standard_normal((ell, m))
+    psi = rng.integers(0, delta + 1, size=(npat, m)).astype(np.int32)
+    G = rng.standard_normal((N, d)).astype(np.float32)
+    Rd, od, pd = dev_tensors(R, order, psi)
+    Gd = torch.from_numpy(G).cuda()
+    T = gc.gc_encode(Rd, ell, od, N, m, delta, pd, Gd)
+    torch.cuda.synchronize()
+    G64 = G.astype(np.float64)
+    for b in range(npat):
+        r = O.run_pattern(R, order, psi[b], N, G64)
+        if np.max(np.abs(r.T)) > 0:
+            assert rel_inf(to_np(T[b]), r.T) <= 1e-4, f"pattern {b}"
+        else:
+            assert float(T[b].abs().max()) == 0.0
+
+
 @pytest.mark.parametrize("ell", [1, 3])
 def test_decode_plan_then_apply(gc, ell):
     """gc_decode_plan (psi side) then gc_decode_apply (data side) equals
