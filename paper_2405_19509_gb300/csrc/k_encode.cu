@@ -28,7 +28,11 @@ __global__ void __launch_bounds__(kEncThreads)
              const int32_t* __restrict__ psi, int N, int m, int delta, int ell, int npat,
              const float* __restrict__ G, int d, int L, float* __restrict__ T) {
   extern __shared__ float s_dyn[];
-  const int j = blockIdx.y, b0 = blockIdx.z * kEncPats;
+  // worker j varies fastest across the grid, so the blocks resident at one
+  // time cover all workers on a few column stripes: the chunk-gradient
+  // columns they read (each used by every holder of the chunk) stay in L2,
+  // where worker-major order swept whole rows of many chunks and re-read them
+  const int j = blockIdx.x, b0 = blockIdx.z * kEncPats;
   const int nb = min(kEncPats, npat - b0);
   const int de = delta * ell;
   float* s_e = s_dyn;                                                // [nb][delta * ell]
@@ -51,7 +55,7 @@ __global__ void __launch_bounds__(kEncThreads)
   int pmax = 0;
 #pragma unroll
   for (int bb = 0; bb < kEncPats; ++bb) pmax = max(pmax, s_np[bb]);
-  for (int c = (blockIdx.x * kEncThreads + threadIdx.x) * V; c < L; c += gridDim.x * kEncThreads * V) {
+  for (int c = (blockIdx.y * kEncThreads + threadIdx.x) * V; c < L; c += gridDim.y * kEncThreads * V) {
     float acc[kEncPats][V];
 #pragma unroll
     for (int bb = 0; bb < kEncPats; ++bb)
@@ -110,7 +114,7 @@ int launch_encode(const double* E, const int32_t* order, const int32_t* psi, int
   // enough blocks for a few waves; each block strides over the rest of its row
   const long long want = std::max<long long>(1, (long long)device_sm_count() * 32 / ((long long)m * groups));
   const int gx = (int)std::max<long long>(1, std::min<long long>(stripes, want));
-  dim3 grid(gx, m, groups);
+  dim3 grid(m, gx, groups);
   const size_t smem = ((size_t)kEncPats * delta * ell + kEncPats + delta) * sizeof(float);
   if (vec)
     k_encode<4><<<grid, kEncThreads, smem, s>>>(E, order, psi, N, m, delta, ell, npat, G, d, L, T);
