@@ -466,14 +466,27 @@ __global__ void __launch_bounds__(kPatThreads) k_patterns(const double* __restri
       const int cnt = hd.cnt[i];
       const int16_t* hw = hd.w + (size_t)i * GC_MAX_REPL;
       const int8_t* hp = hd.p + (size_t)i * GC_MAX_REPL;
+      // holders eight at a time with one 16-byte (workers) and one 8-byte
+      // (slots) load: lanes take consecutive chunks whose rows lie 64 and 32
+      // bytes apart, so per-entry loads cost a cache wavefront each
       uint32_t mask = 0;
-      for (int h = 0; h < cnt; ++h) {
-        int v = ps[hw[h]];
-        if (v < 0 || v > delta) {
-          atomicOr(status, ST_BAD_PSI);
-          v = 0;
+      for (int h0 = 0; h0 < cnt; h0 += 8) {
+        const uint4 w8 = *reinterpret_cast<const uint4*>(hw + h0);
+        const uint2 p8 = *reinterpret_cast<const uint2*>(hp + h0);
+        const uint32_t ww[4] = {w8.x, w8.y, w8.z, w8.w};
+#pragma unroll
+        for (int q = 0; q < 8; ++q) {
+          if (h0 + q < cnt) {
+            const int wq = (int)(int16_t)(ww[q >> 1] >> (16 * (q & 1)));
+            const int pq = (int)(int8_t)(((q < 4 ? p8.x : p8.y) >> (8 * (q & 3))) & 0xffu);
+            int v = ps[wq];
+            if (v < 0 || v > delta) {
+              atomicOr(status, ST_BAD_PSI);
+              v = 0;
+            }
+            if (pq < v) mask |= 1u << (h0 + q);
+          }
         }
-        if (hp[h] < v) mask |= 1u << h;
       }
       float Pf[ELL][ELL];
       double err;
@@ -485,10 +498,18 @@ __global__ void __launch_bounds__(kPatThreads) k_patterns(const double* __restri
       if (TABLE && cnt <= tb.bits) {
         const size_t e = ((size_t)i << tb.bits) | mask;
         const float* pi = tb.pi + e * ELL * ELL;
+        if (ELL == 2) {  // one 16-byte load for the 2 x 2 block
+          const float4 q = *reinterpret_cast<const float4*>(pi);
+          Pf[0][0] = q.x;
+          Pf[0][ELL - 1] = q.y;
+          Pf[ELL - 1][0] = q.z;
+          Pf[ELL - 1][ELL - 1] = q.w;
+        } else {
 #pragma unroll
-        for (int a = 0; a < ELL; ++a)
+          for (int a = 0; a < ELL; ++a)
 #pragma unroll
-          for (int k = 0; k < ELL; ++k) Pf[a][k] = pi[a * ELL + k];
+            for (int k = 0; k < ELL; ++k) Pf[a][k] = pi[a * ELL + k];
+        }
         err = tb.err[e];
         D = __popc(mask);
         if (E) {
