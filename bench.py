@@ -1,31 +1,28 @@
 #!/usr/bin/env python3
 """Benchmark of the gradient-coding hot path on one GB300 (or N replicas).
 
-Workload: logistic regression, m = N = 20 workers/chunks, cyclic assignment
-with delta = 4 chunks per worker, d = 4096, 512 points per chunk (X is 168 MB,
-larger than L2), 10^4 shifted-exponential straggler realizations per step,
-communication factor l = 2.
+Default workload (the headline): the decode-dominated batch -- m = N = 256
+workers/chunks, cyclic assignment with delta = 16 chunks per worker, given
+chunk gradients of length d = 2^20 (fp32 ~ N(0,1), 1.07 GB), 4096 straggler
+patterns per step (per pattern a completion fraction f ~ U[0.2, 1], psi_j ~
+Binomial(16, f)), communication factor l = 2.
 
-One step (every row of the hot path once):
-  1. chunk gradients g_{D_i} at the current w            (gc_chunk_grads)
-  2. Algorithm 1 for all 10^4 patterns -> decode plan,
-     coefficient error and estimate, by lookup in the
-     per-(chunk, holder subset) solutions prepared once   (gc_decode_plan_prepared)
-  3. batched decode-combine Ghat = C . G (10^4 decoded
-     gradients written) with the fused gradient MSE       (gc_decode_apply)
-  4. the live realization: worker encoding (eq. 2), PS
-     decode of the transmissions, and the SGD update      (gc_encode, gc_decode_tx, gc_sgd_step)
-Each stage is captured once in a CUDA graph.  Stages that do not depend on
-each other run concurrently on two streams (Algorithm 1 beside the chunk
-gradients; the live encode / decode / update beside the batched combine);
-CUDA events around every graph replay time each stage live inside the timed
-region.
+One step (every row of the PS's decode path once, on a fresh pattern batch):
+  1. Algorithm 1 for all 4096 patterns -> decode plan,
+     coefficient error and estimate                      (gc_decode_plan)
+  2. the batched decode: 4096 decoded gradients (17.2 GB)
+     written, with each pattern's gradient MSE            (gc_decode_apply)
+Both are captured once in a CUDA graph per double buffer; event-record nodes
+in instrumented copies time each call inside the timed region.  Step inputs
+(the pattern batch) and results (the decoded gradients and per-pattern errors)
+are double-buffered so that copies overlap the next step.
 
 Metric: decoded gradients per second (whole job).  `e2e` repeats the timed
-loop through the same C-ABI calls with the step's inputs (the pattern batch
-and the live pattern) copied from pinned host memory and the per-pattern
-results (coefficient error, estimate, gradient MSE, loss) copied back every
-step.  `--impl reference` times the fp64 CPU oracle on the host cores instead.
+loop through the same C-ABI calls with each step's pattern batch copied from
+pinned host memory and its 4096 decoded gradients (16 GiB) and per-pattern
+errors copied back to pinned host memory.  `--workload` selects the other
+configurations (one JSON line each); `--impl reference` times the fp64 CPU
+oracle on the host cores instead.
 """
 from __future__ import annotations
 
@@ -45,7 +42,9 @@ ROOT = os.path.dirname(os.path.abspath(__file__))
 if ROOT not in sys.path:
     sys.path.insert(0, ROOT)
 
-METRIC = "decoded gradients/sec (logistic m=N=20, delta=4, d=4096, 10^4 realizations, l=2)"
+METRIC = ("decoded gradients/sec (decode-dominated batch: m=N=256, delta=16, d=2^20, "
+          "4096 straggler patterns per step, l=2)")
+METRIC_LOGISTIC = "decoded gradients/sec (logistic m=N=20, delta=4, d=4096, 10^4 realizations, l=2)"
 UNIT = "decoded gradients/s"
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 
@@ -53,27 +52,40 @@ FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustain
 def parse():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=200)
-    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--steps", type=int, default=None,
+                    help="timed steps (default 60 for the decode batch, 200 for logistic)")
+    ap.add_argument("--warmup", type=int, default=None,
+                    help="untimed warm-up steps (default 10 for the decode batch, 20 for logistic)")
     ap.add_argument("--impl", choices=["gc", "reference"], default="gc")
     ap.add_argument("--ell", type=int, default=2)
-    ap.add_argument("--workload", default="logistic",
-                    choices=["logistic", "decode", "sweep", "sgd", "trigger", "batched", "chunkgrad"],
-                    help="logistic: the headline step (default).  The others measure the "
-                         "remaining configurations, one JSON line each (1 GPU)")
+    ap.add_argument("--workload", default="decode",
+                    choices=["decode", "logistic", "sweep", "sgd", "trigger", "batched", "chunkgrad",
+                             "encode"],
+                    help="decode: the headline step (default); logistic: the logistic-regression "
+                         "step (N replicas like the headline).  The others measure the remaining "
+                         "configurations, one JSON line each (1 GPU)")
     ap.add_argument("--small", action="store_true",
                     help="with --workload batched: a 134 MB case (N=64, n_c=1024, d=1024: the "
                          "same tile counts, short K for GEMM 1) for profiler captures instead of "
                          "the 8.6 GB one; with --workload sweep: given chunk gradients instead of "
-                         "X (the decode-combine alone, for profiler captures)")
+                         "X (the decode-combine alone, for profiler captures); with --workload "
+                         "decode: 256 patterns per step (profiler captures)")
     ap.add_argument("--shape", default=None,
                     help="with --workload chunkgrad: one case 'dtype,N,n_c,d' (dtype f32 or bf16) "
                          "timed over --steps calls after --warmup calls, instead of the table of "
                          "8.6 GB cases")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-extras", action="store_true",
+                    help="decode: skip the tensor-GEMM and chunk-gradient side measurements")
     ap.add_argument("--min-warm-seconds", type=float, default=1.5,
                     help="keep warming up at least this long (steady clocks, clock samples)")
-    return ap.parse_args()
+    a = ap.parse_args()
+    dflt = {"decode": (60, 10), "logistic": (200, 20)}.get(a.workload, (10, 3))
+    if a.steps is None:
+        a.steps = dflt[0]
+    if a.warmup is None:
+        a.warmup = dflt[1]
+    return a
 
 
 def peaks():
@@ -185,6 +197,14 @@ def reference_arm(args, rank, world):
 
     if rank != 0:
         return
+    if args.workload == "decode":
+        reference_decode(args, world)
+        return
+    if args.workload != "logistic":
+        print(json.dumps({"impl": "reference", "unavailable": "the reference arm times the decode "
+                          "and logistic workloads; the other workload lines carry the oracle as "
+                          "cpu_baseline"}), flush=True)
+        return
     cfg = get("logistic")
     data = make_data(cfg, "cpu")
     n_sample = 64
@@ -198,7 +218,7 @@ def reference_arm(args, rank, world):
     value = statistics.median(rates)
     cores = os.cpu_count()
     line = {
-        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
+        "impl": "reference", "metric": METRIC_LOGISTIC, "value": value, "unit": UNIT, "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * cfg.npat / value,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
         "data": "synthetic",
@@ -237,7 +257,387 @@ def _traffic(kernel, src_files):
     return e.get("dram_bytes_per_launch")
 
 
-def gpu_arm(args, rank, world, local_rank):
+def oracle_decode_sample(cfg, ell, G32, psi, cols, min_patterns, max_seconds):
+    """Time the fp64 oracle on a bounded sample of the decode workload.
+
+    For each pattern (at least `min_patterns`, more while under `max_seconds`):
+    Algorithm 1 in full (every worker's least-squares problem), then the
+    eq. (2) encode and the Sec. II-B decode on the first `cols` columns of
+    every block (the same block structure on a d' = l * cols problem), the
+    latter scaled to the full block length.  Returns seconds per decoded
+    gradient and the split."""
+    import oracle as O
+    from workloads import make_R
+
+    N, m, delta, d = cfg.N, cfg.m, cfg.delta, cfg.d
+    L = -(-d // ell)
+    S = min(cols, L)
+    idx = np.concatenate([k * L + np.arange(S) for k in range(ell)])
+    idx = idx[idx < d]
+    Gs = G32[:, idx].astype(np.float64)
+    order = O.cyclic_order(N, m, delta)
+    R = make_R(cfg, ell)
+    t_alg = t_cod = 0.0
+    n = 0
+    t0 = time.perf_counter()
+    for b in range(psi.shape[0]):
+        if n >= min_patterns and time.perf_counter() - t0 > max_seconds:
+            break
+        ta = time.perf_counter()
+        B = O.encoding_matrix(R, order, psi[b], N)
+        tb = time.perf_counter()
+        T = O.encode(B, Gs, order, psi[b], ell)
+        O.decode(R, T, Gs.shape[1])
+        tc = time.perf_counter()
+        t_alg += tb - ta
+        t_cod += tc - tb
+        n += 1
+    per = (t_alg + t_cod * (L / S)) / n
+    return {"s_per_gradient": per, "patterns": n, "seconds": time.perf_counter() - t0,
+            "alg1_s": t_alg / n, "codec_s_sample": t_cod / n, "cols": S}
+
+
+def reference_decode(args, world):
+    """--impl reference for the decode batch: the fp64 oracle on the host
+    cores, each step one pattern (Algorithm 1 in full, encode + decode on a
+    2^14-column sample of each block, scaled to d = 2^20)."""
+    from workloads import get, make_chunk_grads, make_patterns
+
+    cfg = get("decode")
+    ell = args.ell
+    G32 = make_chunk_grads(cfg, "cpu").numpy()
+    psi = make_patterns(cfg, stream=900_000)
+    for t in range(args.warmup):
+        oracle_decode_sample(cfg, ell, G32, psi[t:t + 1], 1 << 14, 1, 0.0)
+    per, t_all = [], time.perf_counter()
+    for t in range(args.steps):
+        r = oracle_decode_sample(cfg, ell, G32, psi[args.warmup + t:args.warmup + t + 1], 1 << 14, 1, 0.0)
+        per.append(r["s_per_gradient"])
+    wall = time.perf_counter() - t_all
+    value = 1.0 / statistics.median(per)
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * cfg.npat / value,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic",
+        "config": {"workload": f"decode m=N=256 delta=16 d=2^20 npat=4096 ell={ell}",
+                   "l2": "host run"},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": os.cpu_count(), "kind": "oracle",
+                         "sample": "each step one pattern: Algorithm 1 in full (per-worker "
+                                   "least squares), eq. (2) encode + Sec. II-B decode on 2^14 "
+                                   "columns of each block, scaled to d = 2^20; median over steps"},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+        "wall_s": wall,
+    }
+    print(json.dumps(line), flush=True)
+
+
+def decode_arm(args, rank, world, local_rank):
+    """The headline: Algorithm 1 + the batched decode of 4096 patterns per step."""
+    import dataclasses
+
+    import torch
+
+    import paper_2405_19509_gb300 as gc
+    from workloads import get, make_chunk_grads, make_patterns, make_R
+
+    dev = torch.device("cuda", local_rank)
+    torch.cuda.set_device(dev)
+    cfg = get("decode")
+    if args.small:
+        cfg = dataclasses.replace(cfg, npat=256)
+    N, m, delta, d, npat, ell = cfg.N, cfg.m, cfg.delta, cfg.d, cfg.npat, args.ell
+    G = make_chunk_grads(cfg, dev)
+    _, order, _ = gc.gc_make_assignment(N, m, delta, gc.GC_CYCLIC)
+    Rd = torch.from_numpy(make_R(cfg, ell)).to(dev)
+    od = torch.from_numpy(order).to(dev)
+    S = args.warmup + args.steps
+    nbatch = min(S, 16)   # distinct pattern batches, cycled
+    base = 1_000_000 * rank
+    psi_host = np.stack([make_patterns(cfg, stream=base + t) for t in range(nbatch)])
+    psi_all = torch.from_numpy(psi_host).to(dev)
+    # step inputs and results double-buffered (index k % 2)
+    psi_b = [torch.empty(npat, m, dtype=torch.int32, device=dev) for _ in range(2)]
+    Gh_b = [torch.empty(npat, d, dtype=torch.float32, device=dev) for _ in range(2)]
+    ce_b = [torch.empty(npat, dtype=torch.float64, device=dev) for _ in range(2)]
+    est_b = [torch.empty(npat, dtype=torch.float64, device=dev) for _ in range(2)]
+    mse_b = [torch.empty(npat, dtype=torch.float64, device=dev) for _ in range(2)]
+    plan_s = torch.empty(int(gc.lib.gc_decode_plan_bytes(N, ell, npat)), dtype=torch.uint8, device=dev)
+    wsP, wsA = gc.Workspace(dev), gc.Workspace(dev)
+    bi = [0]
+
+    def stage_plan():   # psi -> Algorithm 1 -> decode plan, coefficient error, estimate
+        gc.gc_decode_plan(Rd, ell, od, N, m, delta, psi_b[bi[0]], plan=plan_s, coef_err=ce_b[bi[0]],
+                          est=est_b[bi[0]], ws=wsP)
+
+    def stage_apply():  # the batched decode: decoded gradients and their MSE
+        gc.gc_decode_apply(plan_s, ell, N, npat, G, Ghat=Gh_b[bi[0]], grad_mse=mse_b[bi[0]], ws=wsA)
+
+    for b in range(2):
+        bi[0] = b
+        psi_b[b].copy_(psi_all[b % nbatch])
+        stage_plan()
+        stage_apply()
+    gc.gc_status(wsP)
+    gc.gc_status(wsA)
+    torch.cuda.synchronize()
+    ser_ev = [torch.cuda.Event(enable_timing=True) for _ in range(4)]
+    for rep in range(3):
+        bi[0] = rep % 2
+        ser_ev[0].record()
+        stage_plan()
+        ser_ev[1].record()
+        ser_ev[2].record()
+        stage_apply()
+        ser_ev[3].record()
+    torch.cuda.synchronize()
+    serial_ms = [ser_ev[0].elapsed_time(ser_ev[1]), ser_ev[2].elapsed_time(ser_ev[3])]
+
+    n0 = gc.gc_kernel_launches()
+    cap_stream = torch.cuda.Stream(dev)
+    graphs = []
+    for b in range(2):
+        bi[0] = b
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=cap_stream):
+            stage_plan()
+            stage_apply()
+        graphs.append(g)
+        if b == 0:
+            launches_per_step = gc.gc_kernel_launches() - n0
+    # instrumented copies (buffer 0): event-record nodes around each call
+    EVERY, NE = 4, 6
+    kev = [[[torch.cuda.Event(enable_timing=True, external=True) for _ in range(2)] for _ in range(2)]
+           for _ in range(NE)]
+    gi = []
+    bi[0] = 0
+    for j in range(NE):
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=cap_stream):
+            kev[j][0][0].record(cap_stream)
+            stage_plan()
+            kev[j][0][1].record(cap_stream)
+            kev[j][1][0].record(cap_stream)
+            stage_apply()
+            kev[j][1][1].record(cap_stream)
+        gi.append(g)
+    torch.cuda.synchronize()
+
+    stream = torch.cuda.current_stream(dev)
+    copy_stream = torch.cuda.Stream(dev)
+    ev_ready = [torch.cuda.Event() for _ in range(2)]
+    ev_done = [torch.cuda.Event() for _ in range(2)]
+    ev_out = [torch.cuda.Event() for _ in range(2)]
+
+    def put_inputs(t, b, src):
+        with torch.cuda.stream(copy_stream):
+            copy_stream.wait_event(ev_done[b])
+            psi_b[b].copy_(src[t % nbatch], non_blocking=True)
+            ev_ready[b].record(copy_stream)
+
+    def run_step(k, t_next, src, instrumented=False, outs=None):
+        b = k % 2
+        g = graphs[b]
+        if instrumented:
+            assert b == 0
+            g = gi[(k // EVERY) % NE]
+        if t_next is not None:
+            put_inputs(t_next, 1 - b, src)
+        stream.wait_event(ev_ready[b])
+        stream.wait_event(ev_out[b])  # results of step k - 2 have been read out
+        g.replay()
+        ev_done[b].record(stream)
+        if outs is not None:
+            with torch.cuda.stream(copy_stream):
+                copy_stream.wait_event(ev_done[b])
+                outs["Ghat"].copy_(Gh_b[b], non_blocking=True)
+                outs["ce"][k].copy_(ce_b[b], non_blocking=True)
+                outs["est"][k].copy_(est_b[b], non_blocking=True)
+                outs["mse"][k].copy_(mse_b[b], non_blocking=True)
+                ev_out[b].record(copy_stream)
+
+    import torch.distributed as tdist
+
+    def barrier():
+        if world > 1:
+            tdist.barrier()
+
+    props = torch.cuda.get_device_properties(dev)
+    uuid = getattr(props, "uuid", None)
+    clocks = Clocks(f"GPU-{uuid}" if uuid is not None else None)
+    clocks.start()
+    t_w = time.perf_counter()
+    put_inputs(0, 0, psi_all)
+    k = 0
+    while k < args.warmup or time.perf_counter() - t_w < args.min_warm_seconds:
+        run_step(k, k + 1, psi_all)
+        k += 1
+        if k % 32 == 0:
+            torch.cuda.synchronize()
+    torch.cuda.synchronize()
+    K = args.steps
+    barrier()
+    torch.cuda.synchronize()
+    t_start = torch.cuda.Event(enable_timing=True)
+    t_end = torch.cuda.Event(enable_timing=True)
+    wall0 = time.perf_counter()
+    t_start.record(stream)
+    copy_stream.wait_stream(stream)
+    put_inputs(args.warmup, 0, psi_all)
+    n_inst = 0
+    for k in range(K):
+        inst = k % EVERY == 0 and k % 2 == 0
+        n_inst += inst
+        run_step(k, args.warmup + k + 1 if k + 1 < K else None, psi_all, instrumented=inst)
+    t_end.record(stream)
+    torch.cuda.synchronize()
+    barrier()
+    wall = time.perf_counter() - wall0
+    clk = clocks.stop()
+    total_ms = t_start.elapsed_time(t_end)
+    n_used = min(NE, n_inst)
+    call_ms = np.array([[kev[j][si][0].elapsed_time(kev[j][si][1]) for si in range(2)]
+                        for j in range(n_used)]).mean(axis=0)
+    gc.gc_status(wsP)
+    gc.gc_status(wsA)
+    mse_dev = mse_b[(K - 1) % 2].clone()
+
+    # ---- end to end: pattern batches from pinned host memory, decoded
+    # gradients and errors back to pinned host memory, every step
+    pin_psi = torch.from_numpy(psi_host).pin_memory()
+    outs = {"Ghat": torch.empty(npat, d, dtype=torch.float32).pin_memory(),
+            "ce": torch.empty(K, npat, dtype=torch.float64).pin_memory(),
+            "est": torch.empty(K, npat, dtype=torch.float64).pin_memory(),
+            "mse": torch.empty(K, npat, dtype=torch.float64).pin_memory()}
+    barrier()
+    torch.cuda.synchronize()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    copy_stream.wait_stream(stream)
+    put_inputs(args.warmup, 0, pin_psi)
+    for k in range(K):
+        run_step(k, args.warmup + k + 1 if k + 1 < K else None, pin_psi, outs=outs)
+    stream.wait_stream(copy_stream)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    barrier()
+    e2e_ms = e0.elapsed_time(e1)
+    assert np.all(np.isfinite(outs["mse"].numpy())) and np.all(outs["est"].numpy() >= 0)
+    assert torch.isfinite(outs["Ghat"][:4]).all()
+    total_ms, e2e_ms = max_over_ranks([total_ms, e2e_ms], world, dev)
+    value = job_rate(npat * K, world, total_ms)
+    e2e_value = job_rate(npat * K, world, e2e_ms)
+
+    # ---- roofline of the dominant call (the decode; Algorithm 1 is the other)
+    pk, pk_src = peaks()
+    hbm = float(pk["hbm_gbs"])
+    Kp = -(-N * ell // 64) * 64
+    plan_b = 2 * npat * ell * Kp * 2
+    apply_bytes = npat * d * 4 + N * d * 4 + plan_b + npat * 8          # Ghat written; G, plan read
+    plan_bytes_alg = npat * m * 4 + plan_b + 2 * npat * 8                 # psi read; plan, errors written
+    achieved = apply_bytes / (call_ms[1] / 1e3) / 1e9
+    roofline = {"kernel": "gc_decode_apply (k_decode_resid + helpers)", "bound": "hbm",
+                "achieved": achieved, "peak": hbm, "unit": "GB/s", "frac": achieved / hbm,
+                "peak_source": f"{pk_src} hbm_gbs",
+                "traffic": _traffic("k_decode_resid", ["k_decode_resid.cu"]),
+                "algorithmic_bytes_per_call": apply_bytes,
+                "timing": "CUDA events recorded by event nodes inside the step's graph around the "
+                          f"gc_decode_apply call (every {EVERY}th timed step, the last {n_used} "
+                          "averaged); the call is the plan scan, the residual decode (which also "
+                          "forms sum_i g), the operand split and GEMM when a tile needs them, and "
+                          "the MSE reduction",
+                "call_ms": {"gc_decode_plan (Algorithm 1)": float(call_ms[0]),
+                            "gc_decode_apply": float(call_ms[1])},
+                "call_GBps": {"gc_decode_plan": plan_bytes_alg / (call_ms[0] / 1e3) / 1e9,
+                              "gc_decode_apply": achieved},
+                "serial_ms": {"gc_decode_plan": serial_ms[0], "gc_decode_apply": serial_ms[1]}}
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K,
+        "warmup": args.warmup, "ms_per_step": total_ms / K, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f32 (Algorithm 1 in f64)",
+        "data": "synthetic",
+        "config": {"workload": f"decode m=N=256 delta=16 d=2^20 npat={npat} ell={ell}",
+                   "l2": "inputs larger than L2 (G 1.07 GB read, Ghat 17.2 GB written per step)",
+                   "parallelism": f"replicas x{world} (independent pattern batches)"},
+        "roofline": roofline,
+        "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": int(npat * m * 4),
+                "d2h_bytes_per_step": int(npat * d * 4 + 3 * npat * 8),
+                "returns": "the step's decoded gradients (npat x d fp32) and per-pattern "
+                           "coefficient error, estimate and gradient MSE"},
+        "gpu_launches": int(launches_per_step * K),
+        "clocks": clk,
+        "wall_s_timed": wall,
+        "exact_patterns_frac": float((mse_dev == 0).double().mean()),
+    }
+    if rank == 0 and world == 1 and not args.no_extras:
+        line["extras"] = decode_extras(gc, torch, dev, cfg, ell, G, Rd, od, psi_all[0], plan_s,
+                                       wsP, wsA, Gh_b[0], mse_b[0], call_ms, pk, pk_src)
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        G32 = G.cpu().numpy()
+        r = oracle_decode_sample(cfg, ell, G32, psi_host[0], 1 << 14, 16, 20.0)
+        line["cpu_baseline"] = {
+            "value": 1.0 / r["s_per_gradient"], "unit": UNIT, "cores": os.cpu_count(), "kind": "oracle",
+            "sample": f"{r['patterns']} patterns of the first batch: Algorithm 1 in full "
+                      f"({r['alg1_s']:.2f} s per pattern), eq. (2) encode + Sec. II-B decode on "
+                      f"{r['cols']} columns of each block ({r['codec_s_sample']:.2f} s) scaled to "
+                      f"d = 2^20; {r['seconds']:.1f} s of CPU work, NumPy with its BLAS threads"}
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+
+
+def decode_extras(gc, torch, dev, cfg, ell, G, Rd, od, pd, plan, wsP, wsA, Gh, mse, call_ms, pk, pk_src):
+    """Side measurements on the headline workload (not part of the step):
+    the same decode forced onto the tensor-core GEMM, and the chunk-gradient
+    pass of the coded-SGD workload (8.6 GB fp32 X)."""
+    from workloads import make_data
+    from workloads import get as get_cfg
+
+    N, m, delta, d, npat = cfg.N, cfg.m, cfg.delta, cfg.d, cfg.npat
+    out = {}
+    bf16s = float(pk.get("bf16_tflops_sustained", pk["bf16_tflops"]))
+    gc.gc_decode_plan(Rd, ell, od, N, m, delta, pd, plan=plan, coef_err=False, est=False, ws=wsP)
+    gc.gc_set_decode_policy(gc.GC_DECODE_DENSE)
+    try:
+        t_dense = _time_ms(torch, lambda: gc.gc_decode_apply(plan, ell, N, npat, G, Ghat=Gh,
+                                                             grad_mse=mse, ws=wsA), 3)
+    finally:
+        gc.gc_set_decode_policy(gc.GC_DECODE_AUTO)
+    gc.gc_status(wsA)
+    L = -(-d // ell)
+    Kp = -(-N * ell // 64) * 64
+    useful = 2.0 * npat * ell * (N * ell) * L
+    issued = 3 * 2.0 * npat * ell * Kp * L
+    out["decode_on_tensor_cores"] = {
+        "ms_apply": t_dense, "decoded_gradients_per_s_apply_only": npat / (t_dense / 1e3),
+        "useful_tflops": useful / (t_dense / 1e3) / 1e12, "issued_tflops": issued / (t_dense / 1e3) / 1e12,
+        "frac_useful_of_bf16_sustained": useful / (t_dense / 1e3) / 1e12 / bf16s,
+        "frac_issued_of_bf16_sustained": issued / (t_dense / 1e3) / 1e12 / bf16s,
+        "note": "gc_decode_apply with every tile on the bf16x3 tcgen05 GEMM (gc_set_decode_policy "
+                "DENSE), operand split included; useful = 2 npat N l^2 L, issued = 3 MMAs per K "
+                "step over the padded K; peak = measured bf16 sustained",
+        "residual_path_speedup": t_dense / float(call_ms[1])}
+    sg = get_cfg("sgd")
+    data = make_data(sg, dev)
+    Gc = torch.empty(sg.N, sg.d, device=dev)
+    lo = torch.zeros(1, dtype=torch.float64, device=dev)
+    ws = gc.Workspace(dev)
+    t_cg = _time_ms(torch, lambda: gc.gc_chunk_grads(data["X"], data["y"], data["w"], sg.N, sg.n_c,
+                                                     gc.GC_LOGISTIC, G=Gc, loss_out=lo, ws=ws), 5)
+    gc.gc_status(ws)
+    nbytes = sg.Ntil * sg.d * 4 + sg.Ntil * 4 + sg.N * sg.d * 4
+    out["chunk_grads"] = {
+        "workload": "sgd m=N=128 n_c=2048 d=8192 fp32 X (8.6 GB), logistic, with the loss",
+        "ms": t_cg, "GB/s": nbytes / (t_cg / 1e3) / 1e9,
+        "frac_of_hbm": nbytes / (t_cg / 1e3) / 1e9 / float(pk["hbm_gbs"]),
+        "TFLOP/s": 4.0 * sg.Ntil * sg.d / (t_cg / 1e3) / 1e12,
+        "note": "two matrix-vector products per chunk (HBM-bound); TFLOP/s = 4 N~ d / t"}
+    del data, Gc
+    torch.cuda.empty_cache()
+    return out
+
+
+def logistic_arm(args, rank, world, local_rank):
     import torch
 
     import paper_2405_19509_gb300 as gc
@@ -563,7 +963,7 @@ def gpu_arm(args, rank, world, local_rank):
                 "serial_stage_ms": {n: float(v) for n, v in zip(names, serial_ms)}}
 
     line = {
-        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K,
+        "metric": METRIC_LOGISTIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K,
         "warmup": args.warmup, "ms_per_step": total_ms / K, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
         "config": {"workload": "logistic m=N=20 delta=4 d=4096 n_c=512 npat=10000 ell=%d" % ell,
@@ -622,57 +1022,41 @@ def extra_workload(args):
     n0 = gc.gc_kernel_launches()
     ell = args.ell
     line = {"workload": args.workload, "n_gpus": 1, "data": "synthetic", "dtype": "f32"}
-    if args.workload == "decode":
+    if args.workload == "encode":
+        # eq. (2) on the decode workload's chunk gradients (A4 alone, from
+        # Algorithm 1's worker coefficients): per pattern G is read and T written
         cfg = get("decode")
-        N, m, delta, d, npat = cfg.N, cfg.m, cfg.delta, cfg.d, cfg.npat
+        N, m, delta, d = cfg.N, cfg.m, cfg.delta, cfg.d
         G = make_chunk_grads(cfg, dev)
         _, order, _ = gc.gc_make_assignment(N, m, delta)
         Rd = torch.from_numpy(make_R(cfg, ell)).to(dev)
         od = torch.from_numpy(order).to(dev)
-        pd = torch.from_numpy(make_patterns(cfg)).to(dev)
-        plan = torch.empty(int(gc.lib.gc_decode_plan_bytes(N, ell, npat)), dtype=torch.uint8, device=dev)
-        Gh = torch.empty(npat, d, device=dev)
-        ce = torch.empty(npat, dtype=torch.float64, device=dev)
-        es = torch.empty_like(ce)
-        wsB, wsC = gc.Workspace(dev), gc.Workspace(dev)
-        t_plan = _time_ms(torch, lambda: gc.gc_decode_plan(Rd, ell, od, N, m, delta, pd, plan=plan,
-                                                           coef_err=ce, est=es, ws=wsB), 5)
-        t_apply = _time_ms(torch, lambda: gc.gc_decode_apply(plan, ell, N, npat, G, Ghat=Gh,
-                                                             grad_mse=False, ws=wsC), 5)
-        gc.gc_status(wsB)
-        gc.gc_status(wsC)
+        psi_all = make_patterns(cfg)
         L = -(-d // ell)
-        Kp = -(-N * ell // 64) * 64
-        useful = 2.0 * npat * ell * (N * ell) * L
-        issued = 3 * 2.0 * npat * ell * Kp * L
-        # eq. (2) encode on the same G for 8 patterns (A4 alone, from Algorithm
-        # 1's worker coefficients): per pattern G read once and T written once
-        del Gh
-        torch.cuda.empty_cache()
-        ne = 8
-        pe = pd[:ne].contiguous()
-        E = gc.gc_find_encoding_coeff(Rd, ell, od, N, m, delta, pe, E=True, C=False, delta_out=False,
-                                      coef_err=False, est=False)["E"]
-        T = torch.empty(ne, m, L, device=dev)
-        t_enc = _time_ms(torch, lambda: gc.gc_encode_with_coeffs(E, ell, od, N, m, delta, pe, G, T=T), 3)
-        enc_bytes = ne * (N * d * 4 + m * L * 4)
-        line["encode"] = {"patterns": ne, "ms": t_enc, "GB/s": enc_bytes / (t_enc / 1e3) / 1e9,
-                          "frac_of_hbm": enc_bytes / (t_enc / 1e3) / 1e9 / hbm,
-                          "note": "algorithmic bytes per pattern: G read (N d 4) + T written (m L 4)"}
-        del T
+        rows = {}
+        for ne in (1, 8):
+            pe = torch.from_numpy(psi_all[:ne]).to(dev)
+            E = gc.gc_find_encoding_coeff(Rd, ell, od, N, m, delta, pe, E=True, C=False, delta_out=False,
+                                          coef_err=False, est=False)["E"]
+            T = torch.empty(ne, m, L, device=dev)
+            t = _time_ms(torch, lambda: gc.gc_encode_with_coeffs(E, ell, od, N, m, delta, pe, G, T=T),
+                         max(3, args.steps), warm=max(2, args.warmup), flush=flush)
+            alg = ne * (N * d * 4 + m * L * 4)
+            dram = N * d * 4 + ne * m * L * 4
+            rows[ne] = {"patterns": ne, "ms": t, "GB/s": alg / (t / 1e3) / 1e9,
+                        "frac_of_hbm": alg / (t / 1e3) / 1e9 / hbm,
+                        "GB/s_G_once": dram / (t / 1e3) / 1e9}
+            del T, E
         line.update({
-            "metric": f"decoded gradients/sec (m=N=256, delta=16, d=2^20, 4096 patterns, l={ell})",
-            "value": npat / ((t_plan + t_apply) / 1e3), "unit": "decoded gradients/s",
-            "ms_plan": t_plan, "ms_apply": t_apply,
-            "roofline": {"kernel": "k_combine_tc", "bound": "tensor", "unit": "TFLOP/s",
-                         "achieved": issued / (t_apply / 1e3) / 1e12, "peak": bf16,
-                         "frac": issued / (t_apply / 1e3) / 1e12 / bf16,
-                         "useful_tflops": useful / (t_apply / 1e3) / 1e12,
-                         "note": "issued = three bf16 MMAs per K step (hi/lo split) over the padded K; "
-                                 "timed gc_decode_apply includes the operand split",
-                         "peak_source": f"{pk_src} bf16_tflops"},
-            "config": {"workload": f"decode m=N=256 delta=16 d=2^20 npat=4096 ell={ell}",
-                       "l2": "inputs larger than L2 (G 1.07 GB, Ghat 17.2 GB)"}})
+            "metric": f"encode GB/s (eq. 2; m=N=256, delta=16, d=2^20, l={ell}, 1 pattern)",
+            "value": rows[1]["GB/s"], "unit": "GB/s", "per_patterns": rows,
+            "roofline": {"kernel": "k_encode", "bound": "hbm", "unit": "GB/s",
+                         "achieved": rows[1]["GB/s"], "peak": hbm, "frac": rows[1]["frac_of_hbm"],
+                         "note": "algorithmic bytes per pattern: G read once (N d 4) + T written "
+                                 "(m L 4); GB/s_G_once counts G once for the whole call",
+                         "peak_source": f"{pk_src} hbm_gbs"},
+            "config": {"workload": f"encode m=N=256 delta=16 d=2^20 ell={ell}, 1 and 8 patterns",
+                       "l2": "L2 flushed before each timed call (G 1.07 GB)"}})
     elif args.workload == "sweep":
         cfg = get("mse_sweep")
         N, m, delta, d, npat = cfg.N, cfg.m, cfg.delta, cfg.d, cfg.npat
@@ -893,7 +1277,7 @@ def extra_workload(args):
 
 def main():
     args = parse()
-    if args.workload != "logistic" and args.impl == "gc":
+    if args.workload not in ("decode", "logistic") and args.impl == "gc":
         extra_workload(args)
         return
     world = int(os.environ.get("WORLD_SIZE", "1"))
@@ -907,7 +1291,10 @@ def main():
         import torch.distributed as tdist
         torch.cuda.set_device(local_rank)
         tdist.init_process_group("nccl", device_id=torch.device("cuda", local_rank))
-    gpu_arm(args, rank, world, local_rank)
+    if args.workload == "decode":
+        decode_arm(args, rank, world, local_rank)
+    else:
+        logistic_arm(args, rank, world, local_rank)
     if world > 1:
         import torch.distributed as tdist
         tdist.destroy_process_group()

@@ -97,9 +97,38 @@ int gc_set_wait_limit(int64_t cycles);
  * bit is consumed by the launch it affects.  Do not arm it while capturing a
  * CUDA graph (the capture would keep the withheld copy).  Process-wide. */
 #define GC_STALL_CHUNK_GRADS 1 /* the chunk-gradient kernel (gc_chunk_grads)  */
-#define GC_STALL_COMBINE 2     /* the tensor-core combine (decode apply, MSE) */
+#define GC_STALL_COMBINE 2     /* the tensor-core combine (decode apply, MSE;
+                                  it waits only on tiles it computes, see
+                                  gc_set_decode_policy) */
 #define GC_STALL_BATCHED 4     /* the batched chunk-gradient GEMMs (first one) */
 int gc_inject_stall(int kernels);
+
+/* Path of the batched decode (gc_decode_batch, gc_decode_apply,
+ * gc_decode_combine, gc_mse).  Every decode block Pi_i = R_{S_i} X^+ is the
+ * identity I_ell when Delta_i >= ell (Sec. II-A), so the decoded gradient is
+ *   ghat_b = sum_i g_{D_i} + sum_{i : Pi_{b,i} != I} (Pi_{b,i} - I) g_{D_i}   (blockwise),
+ * which costs the write of ghat_b plus one chunk-gradient read per
+ * non-identity block.  Each 128-row tile of the decode (128 / ell patterns)
+ * is computed either that way (the residual path) or by the bf16x3
+ * tensor-core GEMM Ghat = C . G; the choice is made on the device from the
+ * decode matrix:
+ *   GC_DECODE_AUTO      a tile takes the residual path when its patterns
+ *                       average at most ceil(N*ell/64) non-identity blocks
+ *                       (what the GEMM spends per pattern, in chunk-gradient
+ *                       reads) and none has more than the list capacity
+ *                       (16 blocks for ell <= 2, 8 for ell <= 4, else 4).
+ *   GC_DECODE_DENSE     every tile on the GEMM.
+ *   GC_DECODE_RESIDUAL  every tile whose patterns fit the list capacity on
+ *                       the residual path.
+ * Both paths give the same values up to fp32 rounding (the tests compare them
+ * with each other and with the fp64 oracle); a pattern whose blocks are all
+ * I_ell has grad_mse exactly 0 on the residual path.  Process-wide setting
+ * (default GC_DECODE_AUTO) read at each launch; meant for tests and
+ * measurements. */
+#define GC_DECODE_AUTO 0
+#define GC_DECODE_DENSE 1
+#define GC_DECODE_RESIDUAL 2
+int gc_set_decode_policy(int policy);
 
 /* Zero the status header of a workspace (asynchronous on `stream`). */
 int gc_workspace_init(void* ws, size_t ws_bytes, void* stream);
@@ -295,11 +324,16 @@ int gc_encode_with_coeffs(const double* E, int ell, const int32_t* order, int N,
 int gc_decode_tx(const double* R, int ell, int m, const float* T, int npat, int d, float* ghat,
                  void* stream);
 
-/* ---- batched decode-combine -------------------------------------------
- * The composition of encode and decode for many patterns at once, using the
- * identity sum_j R[k][j] T[b][j] = sum_i sum_k' (R B_b)[k][i*ell+k'] g_{D_i}[k']:
+/* ---- batched decode-combine (Sec. II-B decode of the eq. (2) transmissions) --
+ * The PS decode of Sec. II-B, sum_j R[k][j] T[b][j], applied to the
+ * transmissions of eq. (2) for many patterns at once, through the identity
+ * sum_j R[k][j] T[b][j] = sum_i sum_k' (R B_b)[k][i*ell+k'] g_{D_i}[k']:
  *   Ghat (npat*ell x L) = C (npat*ell x N*ell) . G (N*ell x L),
- * with C from Algorithm 1 (above) and G viewed as N*ell blocks of length L.
+ * with C from Algorithm 1 (above) and G viewed as N*ell blocks of length L;
+ * each 128-row tile is computed by the residual path or the tensor-core
+ * GEMM (gc_set_decode_policy).  The supports (masks), Delta_i, the worker
+ * coefficients E and C itself are outputs of gc_find_encoding_coeff on the
+ * same psi; this call returns only the decoded gradients and errors.
  * G     N x d float32 chunk gradients.
  * Ghat  NULL or npat x d float32 decoded gradients.
  * coef_err, est   NULL or npat float64 (as gc_find_encoding_coeff).

@@ -41,6 +41,7 @@ _sig("gc_version", _i)
 _sig("gc_kernel_launches", ctypes.c_uint64)
 _sig("gc_set_wait_limit", _i, _i64)
 _sig("gc_inject_stall", _i, _i)
+_sig("gc_set_decode_policy", _i, _i)
 _sig("gc_workspace_init", _i, _p, _sz, _p)
 _sig("gc_status", _i, _p, _p)
 _sig("gc_make_assignment", _i, _i, _i, _i, _i, _p, _p, _p, _p)
@@ -454,6 +455,18 @@ GC_STALL_BATCHED = 4
 def gc_inject_stall(kernels: int) -> None:
     """Testing aid: the next launch of each selected kernel withholds its copies."""
     _check(lib.gc_inject_stall(int(kernels)))
+
+
+GC_DECODE_AUTO = 0
+GC_DECODE_DENSE = 1
+GC_DECODE_RESIDUAL = 2
+
+
+def gc_set_decode_policy(policy: int) -> None:
+    """Path of the batched decode per 128-row tile: GC_DECODE_AUTO (default),
+    GC_DECODE_DENSE (tensor-core GEMM) or GC_DECODE_RESIDUAL (sum of the
+    chunk gradients plus the non-identity blocks).  Process-wide."""
+    _check(lib.gc_set_decode_policy(int(policy)))
 
 
 def gc_kernel_launches() -> int:

@@ -38,6 +38,8 @@ long long wait_limit(long long dflt) {
 }
 static std::atomic<int> g_stall{0};
 bool take_stall(int bit) { return (g_stall.fetch_and(~bit) & bit) != 0; }
+static std::atomic<int> g_policy{GC_DECODE_AUTO};
+int decode_policy() { return g_policy.load(std::memory_order_relaxed); }
 
 int device_sm_count() {
   int dev = 0, n = 0;
@@ -99,7 +101,7 @@ extern "C" {
 
 const char* gc_last_error(void) { return g_err; }
 
-int gc_version(void) { return 100; }
+int gc_version(void) { return 200; }
 
 uint64_t gc_kernel_launches(void) { return g_launches.load(); }
 
@@ -159,6 +161,13 @@ int gc_trigger_times(const int32_t* order, int N, int m, int delta, const double
   Holders h = carve_holders(c, N);
   launch_holders(order, N, m, delta, h, status_of(ws), s);
   return launch_trigger(order, h, N, m, delta, tau, nsim, ell, theta, T, psi, T_full, s);
+}
+
+int gc_set_decode_policy(int policy) {
+  if (policy != GC_DECODE_AUTO && policy != GC_DECODE_DENSE && policy != GC_DECODE_RESIDUAL)
+    return fail(GC_ERR_ARG, "unknown decode policy %d", policy);
+  g_policy.store(policy, std::memory_order_relaxed);
+  return GC_OK;
 }
 
 int gc_set_wait_limit(int64_t cycles) {

@@ -113,6 +113,41 @@ int launch_decode_tx(const double* R, int ell, int m, const float* T, int npat, 
                      cudaStream_t s);
 int launch_sgd(float* w, const float* ghat, int d, float lr, int64_t Ntil, cudaStream_t s);
 
+// ---- batched decode in residual form (k_decode_resid.cu) -----------------
+// Per pattern the ordered list of decode blocks that differ from I_ell (chunk
+// index and D = Pi - I); per 128-row tile of the decode the path that
+// produces its rows (tflag = 1: the tensor-core GEMM; 0: the residual kernel)
+// and, for a residual tile, the ordered list of its rows that need
+// corrections, each with a slot of squared-error partials.
+constexpr int kResidThreads = 256;
+constexpr int kResidW = 32;          // columns of one block per stripe (one per lane)
+constexpr int kResidRcap = 32;       // corrected rows a residual tile may hold
+constexpr int kResidMaxRows = 1280;  // N*ell staged per stripe (160 KB of shared memory)
+struct ResidLists {
+  int32_t* nnz;        // [npat] non-identity blocks (may exceed ksp)
+  int32_t* idx;        // [npat][ksp] their chunks, ascending
+  float* D;            // [npat][ksp][ell][ell] Pi - I
+  int32_t* tflag;      // [ntiles]
+  int32_t* any_dense;  // one word: some tile is on the GEMM
+  int32_t* rslot;      // [npat*ell] slot of a corrected row of a residual tile, else -1
+  int32_t* rowlist;    // [ntiles][kResidRcap] corrected rows of each tile, ascending
+  int32_t* tcount;     // [ntiles] entries of rowlist
+  float* msp;          // [ntiles*kResidRcap][parts] squared-error partials, or null
+  int ksp;             // list capacity per pattern
+  int parts;           // partials per corrected row (column stripes)
+};
+int resid_ksp(int ell);
+bool resid_fits(int N, int ell);
+size_t resid_ws_bytes(int N, int ell, int npat, int d);
+ResidLists carve_resid(Carve& c, int N, int ell, int npat, int d, bool want_mse);
+int launch_plan_scan(const __nv_bfloat16* Cs, int Kp, int N, int ell, int npat, int budget,
+                     int policy, const ResidLists& rl, unsigned int* done_counter, cudaStream_t s);
+int launch_gsum(const float* G, int N, int d, float* gsum, cudaStream_t s);
+int launch_decode_resid(const float* G, const ResidLists& rl, int N, int ell, int npat, int d,
+                        float* gsum, float* Ghat, cudaStream_t s);
+// Process-wide path policy of the batched decode (gc_set_decode_policy).
+int decode_policy();
+
 // ---- batched decode-combine on the tensor cores (k_combine_tc.cu) --------
 // K = N*ell padded to whole 64-element blocks (the GEMM's K extent).
 inline int combine_kp(int N, int ell) { return (N * ell + 63) / 64 * 64; }

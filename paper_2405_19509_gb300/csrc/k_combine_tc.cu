@@ -39,7 +39,7 @@
 
 #include <algorithm>
 
-#include "gc_internal.cuh"
+#include "tc_ptx.cuh"
 
 namespace gc {
 namespace tc {
@@ -85,137 +85,29 @@ struct Params {
   int parts_per_row;    // num_n_tiles * (epilogue warps per TMEM lane quarter)
   long long spin_limit; // clock cycles a wait may take before the kernel gives up
   int stall;            // failure-path test: the TMA producer issues nothing
+  const int32_t* tflag; // per m-tile: nonzero = this kernel computes the tile's rows (null = all)
   uint32_t* status;
 };
 
-__device__ __forceinline__ uint32_t smem_u32(const void* p) {
-  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+// The tiles a CTA computes: t, t + step, ... below t_last whose m-tile is
+// flagged for the GEMM (the other rows come from the residual decode).  Every
+// role walks the same sequence.
+__device__ __forceinline__ long long active_tile(const Params& p, long long t, long long t_last,
+                                                 long long step) {
+  if (p.tflag)
+    while (t < t_last && __ldg(p.tflag + (int)(t % p.num_m_tiles)) == 0) t += step;
+  return t;
 }
-__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
-  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count) : "memory");
-}
-__device__ __forceinline__ void mbar_expect_tx(uint64_t* bar, uint32_t bytes) {
-  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)),
-               "r"(bytes)
-               : "memory");
-}
-__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
-  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
-}
-__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
-  uint32_t ok;
-  asm volatile(
-      "{\n\t.reg .pred p;\n\t"
-      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
-      "selp.u32 %0, 1, 0, p;\n\t}"
-      : "=r"(ok)
-      : "r"(smem_u32(bar)), "r"(parity)
-      : "memory");
-  return ok != 0;
-}
-// Bounded wait; gives up when the limit passes or another role aborted.
-__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag,
-                                          uint32_t* status, long long limit) {
-  if (mbar_try_wait(bar, parity)) return true;
-  const long long t0 = clock64();
-  while (!mbar_try_wait(bar, parity)) {
-    if (*abort_flag) return false;
-    if (clock64() - t0 > limit) {
-      atomicOr(status, ST_TIMEOUT);
-      *abort_flag = 1;
-      return false;
-    }
-  }
-  return true;
-}
-__device__ __forceinline__ void tma_load_3d(void* dst, const CUtensorMap* map, int x, int y, int z,
-                                            uint64_t* bar) {
-  asm volatile(
-      "cp.async.bulk.tensor.3d.shared::cluster.global.mbarrier::complete_tx::bytes "
-      "[%0], [%1, {%2, %3, %4}], [%5];" ::"r"(smem_u32(dst)),
-      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(z), "r"(smem_u32(bar))
-      : "memory");
-}
-__device__ __forceinline__ void tma_store_2d(const CUtensorMap* map, const void* src, int x, int y) {
-  asm volatile(
-      "cp.async.bulk.tensor.2d.global.shared::cta.bulk_group [%0, {%1, %2}], [%3];" ::"l"(
-          reinterpret_cast<uint64_t>(map)),
-      "r"(x), "r"(y), "r"(smem_u32(src))
-      : "memory");
-}
-// The same store with an L2 cache policy operand (createpolicy).
-__device__ __forceinline__ void tma_store_2d_hint(const CUtensorMap* map, const void* src, int x, int y,
-                                                  uint64_t policy) {
-  asm volatile(
-      "cp.async.bulk.tensor.2d.global.shared::cta.bulk_group.L2::cache_hint [%0, {%1, %2}], [%3], %4;" ::"l"(
-          reinterpret_cast<uint64_t>(map)),
-      "r"(x), "r"(y), "r"(smem_u32(src)), "l"(policy)
-      : "memory");
-}
-__device__ __forceinline__ uint64_t policy_evict_first() {
-  uint64_t pol;
-  asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(pol));
-  return pol;
-}
-__device__ __forceinline__ void bulk_commit() {
-  asm volatile("cp.async.bulk.commit_group;" ::: "memory");
-}
-__device__ __forceinline__ void bulk_wait_read1() {
-  asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory");
-}
-__device__ __forceinline__ void bulk_wait_all() {
-  asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
-}
-// Shared-memory matrix descriptor: K-major, 128-byte swizzle, 8-row groups
-// 1024 bytes apart (stride byte offset), descriptor version 1.
-__device__ __forceinline__ uint64_t sdesc(uint32_t saddr) {
-  uint64_t d = 0;
-  d |= (uint64_t)((saddr >> 4) & 0x3FFFu);
-  d |= (uint64_t)1u << 16;             // leading byte offset (unused for swizzled K-major)
-  d |= (uint64_t)(1024u >> 4) << 32;   // stride byte offset
-  d |= (uint64_t)1u << 46;             // version
-  d |= (uint64_t)2u << 61;             // SWIZZLE_128B
-  return d;
-}
-// Instruction descriptor, kind::f16: D fp32, A and B bf16, both K-major.
+
+using namespace tcw;
+
+// Descriptor of a K-major operand tile (128-byte swizzle, 8-row groups 1 KB apart).
+__device__ __forceinline__ uint64_t sdesc(uint32_t saddr) { return tcw::sdesc(saddr, 16, 1024); }
+// Instruction descriptor, kind::f16: D fp32, A and B bf16, both K-major, M = BM, N = BN.
 constexpr uint32_t kIdesc = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(BN >> 3) << 17) |
                             ((uint32_t)(BM >> 4) << 24);
-
 __device__ __forceinline__ void mma_bf16(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t accum) {
-  asm volatile(
-      "{\n\t.reg .pred p;\n\t"
-      "setp.ne.b32 p, %4, 0;\n\t"
-      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
-      "l"(a), "l"(b), "r"(kIdesc), "r"(accum)
-      : "memory");
-}
-__device__ __forceinline__ void mma_commit(uint64_t* bar) {
-  asm volatile(
-      "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
-          smem_u32(bar))
-      : "memory");
-}
-__device__ __forceinline__ void fence_before() {
-  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
-}
-__device__ __forceinline__ void fence_after() {
-  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-}
-__device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
-  uint32_t r[32];
-  asm volatile(
-      "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
-      "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, "
-      "%16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31}, [%32];"
-      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
-        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
-        "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]),
-        "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]),
-        "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
-      : "r"(taddr));
-  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
-#pragma unroll
-  for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(r[j]);
+  tcw::mma_bf16(d_tmem, a, b, kIdesc, accum);
 }
 
 template <int STAGES, int EPI, int NKBR, bool OUT>
@@ -287,7 +179,8 @@ __global__ void __launch_bounds__(64 + 32 * EPI, 1)
       uint32_t it = 0, nb_loads = 0;
       int cur_nt = -1;
       bool ok = !p.stall;
-      for (long long t = t_first; t < t_last && ok; t += t_step) {
+      for (long long t = active_tile(p, t_first, t_last, t_step); t < t_last && ok;
+           t = active_tile(p, t + t_step, t_last, t_step)) {
         const int nt = (int)(t / p.num_m_tiles), mt = (int)(t % p.num_m_tiles);
         if (nt != cur_nt) {
           // the MMAs on the previous B tile have finished before it is replaced
@@ -320,7 +213,8 @@ __global__ void __launch_bounds__(64 + 32 * EPI, 1)
     } else if (lane == 0) {
       uint32_t it = 0;
       bool ok = !p.stall;
-      for (long long t = t_first; t < t_last && ok; t += t_step) {
+      for (long long t = active_tile(p, t_first, t_last, t_step); t < t_last && ok;
+           t = active_tile(p, t + t_step, t_last, t_step)) {
         const int nt = (int)(t / p.num_m_tiles), mt = (int)(t % p.num_m_tiles);
         for (int kb = 0; kb < p.nkb; ++kb, ++it) {
           const int s = it % STAGES;
@@ -347,7 +241,8 @@ __global__ void __launch_bounds__(64 + 32 * EPI, 1)
     if (lane == 0 && BRES) {
       uint32_t it = 0, tile_it = 0, nb_used = 0;
       int cur_nt = -1;
-      for (long long t = t_first; t < t_last; t += t_step, ++tile_it) {
+      for (long long t = active_tile(p, t_first, t_last, t_step); t < t_last;
+           t = active_tile(p, t + t_step, t_last, t_step), ++tile_it) {
         const int nt = (int)(t / p.num_m_tiles);
         if (nt != cur_nt) {
           if (!mbar_wait(bfull, nb_used & 1, abort_flag, p.status, p.spin_limit)) break;
@@ -382,7 +277,8 @@ __global__ void __launch_bounds__(64 + 32 * EPI, 1)
         if (!ok) break;
         mma_commit(&tfull[ab]);
         // last tile on this B tile: hand it back once these MMAs complete
-        const bool last_on_b = t + t_step >= t_last || (int)((t + t_step) / p.num_m_tiles) != nt;
+        const long long tn = active_tile(p, t + t_step, t_last, t_step);
+        const bool last_on_b = tn >= t_last || (int)(tn / p.num_m_tiles) != nt;
         if (last_on_b) mma_commit(bempty);
       }
       mma_commit(done);
@@ -391,7 +287,8 @@ __global__ void __launch_bounds__(64 + 32 * EPI, 1)
     } else if (lane == 0) {
       uint32_t it = 0, tile_it = 0;
       bool ok = true;
-      for (long long t = t_first; t < t_last && ok; t += t_step, ++tile_it) {
+      for (long long t = active_tile(p, t_first, t_last, t_step); t < t_last && ok;
+           t = active_tile(p, t + t_step, t_last, t_step), ++tile_it) {
         const int ab = tile_it & 1;
         if (!mbar_wait(&tempty[ab], ((tile_it >> 1) & 1) ^ 1, abort_flag, p.status, p.spin_limit))
           break;
@@ -436,7 +333,8 @@ __global__ void __launch_bounds__(64 + 32 * EPI, 1)
     const int cbeg = (e / 4) * SPAN;
     float* wbuf = outbuf + e * 2 * (OUT_BUF / 4);
     uint32_t tile_it = 0, chunk_it = 0;
-    for (long long t = t_first; t < t_last; t += t_step, ++tile_it) {
+    for (long long t = active_tile(p, t_first, t_last, t_step); t < t_last;
+         t = active_tile(p, t + t_step, t_last, t_step), ++tile_it) {
       const int ab = tile_it & 1;
       const int nt = (int)(t / p.num_m_tiles), mt = (int)(t % p.num_m_tiles);
       // warp-uniform: the TMEM loads below are warp-collective
@@ -571,18 +469,19 @@ __global__ void k_split_c(const float* __restrict__ C, int M, int K, int Kp,
 // transposes the tile of 32 K-rows (kk = 32 y ..) by COLS columns
 // (c = COLS x ..) through shared memory: 16-byte loads along c, 16-byte
 // stores along kk (COLS = 128 for long rows, 32 when L is short and more
-// blocks are wanted).  Blocks with y == 0 also write
-// gsum[k'*L + c] = sum_i g_{D_i}[k'*L + c] (chunks in order) when gsum != 0.
+// blocks are wanted).  Nothing is done when *any_dense is zero: no row tile
+// of the batch is on the GEMM.
 template <int COLS>
 __global__ void __launch_bounds__(256) k_split_gt(const float* __restrict__ G, int N, int d,
                                                   int ell, int L, int Kp,
                                                   __nv_bfloat16* __restrict__ out,
-                                                  float* __restrict__ gsum) {
+                                                  const int32_t* __restrict__ any_dense) {
   constexpr int kSplitCols = COLS;
   constexpr int TPR = COLS / 4;            // threads per row of the load phase
   constexpr int RPP = 256 / TPR;           // rows per pass
   // the combine kernel may be scheduled now; it waits for this grid to finish
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+  if (__ldg(any_dense) == 0) return;
   __shared__ float tile[32][kSplitCols + 1];
   const int c0 = blockIdx.x * kSplitCols, k0 = blockIdx.y * 32;
   const int t = threadIdx.x;
@@ -636,37 +535,45 @@ __global__ void __launch_bounds__(256) k_split_gt(const float* __restrict__ G, i
       }
     }
   }
-  if (gsum && blockIdx.y == 0) {
-    for (int it = t; it < kSplitCols * ell; it += blockDim.x) {
-      const int cc = it % kSplitCols, kp = it / kSplitCols, c = c0 + cc;
-      const int col = kp * L + c;
-      if (c < L && col < d) {
-        float acc = 0.f;
-        for (int i = 0; i < N; ++i) acc += __ldg(G + (size_t)i * d + col);
-        gsum[col] = acc;
-      }
-    }
-  }
 }
 
-// grad_mse[b] = (sum of the partial squared errors of rows b*ell .. b*ell+ell-1) / d:
-// one warp per pattern (its ell * parts partials are contiguous), lanes
-// stride over them, then a fixed xor tree (fp32: the partials are fp32 sums
-// already; the result is scaled in fp64).  Launched as a programmatic
-// dependent of the combine kernel.
-__global__ void k_mse_reduce_tiles(const float* __restrict__ msep, int npat, int ell,
-                                   int parts, double inv_d, double* __restrict__ grad_mse) {
+// grad_mse[b] = (sum over the rows b*ell .. b*ell+ell-1 of their partial
+// squared errors) / d: one warp per pattern; a row of a GEMM tile sums the
+// combine's partials, a row of a residual tile the residual kernel's (none
+// for a pattern whose blocks are all I_ell: its error is exactly zero).
+// Lanes stride over a row's partials, then a fixed xor tree; rows are added
+// in order (fp32 partial sums, the result scaled in fp64).  Launched as a
+// programmatic dependent of the combine kernel.
+__global__ void k_mse_reduce_tiles(const float* __restrict__ msep, int parts,
+                                   const float* __restrict__ msp, int parts_r,
+                                   const int32_t* __restrict__ tflag, const int32_t* __restrict__ rslot,
+                                   int npat, int ell, double inv_d, double* __restrict__ grad_mse) {
   asm volatile("griddepcontrol.wait;" ::: "memory");
   const long long b = ((long long)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
   const int lane = threadIdx.x & 31;
   if (b >= npat) return;
-  const float* r = msep + (size_t)b * ell * parts;
-  const int n = ell * parts;
-  float s = 0.f;
-  for (int t = lane; t < n; t += 32) s += __ldg(r + t);
+  float tot = 0.f;
+  for (int k = 0; k < ell; ++k) {
+    const long long row = b * ell + k;
+    const float* r = nullptr;
+    int n = 0;
+    if (__ldg(tflag + (row >> 7))) {
+      r = msep + (size_t)row * parts;
+      n = parts;
+    } else {
+      const int slot = __ldg(rslot + row);
+      if (slot >= 0) {
+        r = msp + (size_t)slot * parts_r;
+        n = parts_r;
+      }
+    }
+    float s = 0.f;
+    for (int t = lane; t < n; t += 32) s += __ldg(r + t);
 #pragma unroll
-  for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
-  if (lane == 0) grad_mse[b] = (double)s * inv_d;
+    for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+    tot += s;
+  }
+  if (lane == 0) grad_mse[b] = (double)tot * inv_d;
 }
 
 PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
@@ -748,7 +655,7 @@ size_t apply_ws_bytes(int N, int ell, int npat, int d) {
   const int Kp = combine_kp(N, ell);
   const int nnt = (L + tc::BN - 1) / tc::BN;
   return align_up((size_t)2 * L * Kp * 2, 256) + align_up((size_t)d * sizeof(float), 256) +
-         align_up((size_t)M * nnt * 2 * sizeof(float), 256);
+         align_up((size_t)M * nnt * 2 * sizeof(float), 256) + resid_ws_bytes(N, ell, npat, d);
 }
 
 int launch_split_c(const float* C, int N, int ell, int npat, __nv_bfloat16* Cs, cudaStream_t s) {
@@ -761,6 +668,10 @@ int launch_split_c(const float* C, int N, int ell, int npat, __nv_bfloat16* Cs, 
   return cuda_check(cudaGetLastError(), "k_split_c");
 }
 
+// The decode of a batch: the plan scan picks the path of every 128-row tile
+// (k_decode_resid.cu); residual tiles are written by the residual kernel, the
+// others by the tensor-core GEMM (whose operand split runs only when some
+// tile needs it), then the per-pattern errors are reduced.
 int launch_apply(const __nv_bfloat16* Cs, const float* G, int N, int ell, int npat, int d,
                  float* Ghat, double* grad_mse, Carve& ws, uint32_t* status, cudaStream_t s) {
   using namespace tc;
@@ -772,21 +683,38 @@ int launch_apply(const __nv_bfloat16* Cs, const float* G, int N, int ell, int np
   const int nmt = (int)((M + BM - 1) / BM), nnt = (L + BN - 1) / BN;
   __nv_bfloat16* Gs = ws.take<__nv_bfloat16>((size_t)2 * L * Kp);
   float* gsum = ws.take<float>((size_t)d);
-  float* msep = grad_mse ? ws.take<float>((size_t)M * nnt * 2) : nullptr;
+  float* msep_mem = ws.take<float>((size_t)M * nnt * 2);
+  float* msep = grad_mse ? msep_mem : nullptr;
+  const ResidLists rl = carve_resid(ws, N, ell, npat, d, grad_mse != nullptr);
+  // batches too wide for a staged stripe of every chunk gradient go to the GEMM
+  const bool resid_ok = resid_fits(N, ell);
+  const int policy = resid_ok ? decode_policy() : GC_DECODE_DENSE;
+  // a residual tile may spend up to Kp / 64 corrections per pattern: about
+  // what the three MMAs per 64-wide K block cost against reading the ell
+  // blocks of one chunk gradient
+  const int budget = std::max(1, Kp / 64);
+  // header word 4: completion counter of the plan scan (zeroed with the header)
+  unsigned int* counter = reinterpret_cast<unsigned int*>(status) + 4;
+  int rc = launch_plan_scan(Cs, Kp, N, ell, npat, budget, policy, rl, counter, s);
+  if (rc) return rc;
+  // the residual kernel also forms s = sum_i g_{D_i} (the GEMM's MSE needs it)
+  rc = resid_ok ? launch_decode_resid(G, rl, N, ell, npat, d, gsum, Ghat, s)
+                : launch_gsum(G, N, d, gsum, s);
+  if (rc) return rc;
   {
     if (L >= 16384) {
       dim3 grid((L + 127) / 128, Kp / 32);
-      k_split_gt<128><<<grid, 256, 0, s>>>(G, N, d, ell, L, Kp, Gs, grad_mse ? gsum : nullptr);
+      k_split_gt<128><<<grid, 256, 0, s>>>(G, N, d, ell, L, Kp, Gs, rl.any_dense);
     } else {
       dim3 grid((L + 31) / 32, Kp / 32);
-      k_split_gt<32><<<grid, 256, 0, s>>>(G, N, d, ell, L, Kp, Gs, grad_mse ? gsum : nullptr);
+      k_split_gt<32><<<grid, 256, 0, s>>>(G, N, d, ell, L, Kp, Gs, rl.any_dense);
     }
     count_launches(1);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return cuda_check(e, "k_split_gt");
   }
   CUtensorMap mA, mB, mC;
-  int rc = make_map(&mA, Cs, (int)M, Kp, BM);
+  rc = make_map(&mA, Cs, (int)M, Kp, BM);
   if (rc) return rc;
   rc = make_map(&mB, Gs, L, Kp, BN);
   if (rc) return rc;
@@ -816,6 +744,7 @@ int launch_apply(const __nv_bfloat16* Cs, const float* G, int N, int ell, int np
   p.Ghat = Ghat;
   p.gsum = grad_mse ? gsum : nullptr;
   p.msep = msep;
+  p.tflag = rl.tflag;
   p.status = status;
   p.spin_limit = wait_limit(kSpin);
   p.stall = take_stall(GC_STALL_COMBINE) ? 1 : 0;
@@ -842,8 +771,9 @@ int launch_apply(const __nv_bfloat16* Cs, const float* G, int N, int ell, int np
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    cudaError_t e = cudaLaunchKernelEx(&cfg, k_mse_reduce_tiles, (const float*)msep, npat, ell,
-                                       p.parts_per_row, 1.0 / (double)d, grad_mse);
+    cudaError_t e = cudaLaunchKernelEx(&cfg, k_mse_reduce_tiles, (const float*)msep, p.parts_per_row,
+                                       (const float*)rl.msp, rl.parts, (const int32_t*)rl.tflag,
+                                       (const int32_t*)rl.rslot, npat, ell, 1.0 / (double)d, grad_mse);
     if (e != cudaSuccess) return cuda_check(e, "cudaLaunchKernelEx(k_mse_reduce_tiles)");
     count_launches(1);
   }

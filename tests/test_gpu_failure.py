@@ -70,6 +70,8 @@ def test_combine_stall_times_out_then_recovers(gc):
     pd, Gd = torch.from_numpy(psi).to(dev), torch.from_numpy(G).to(dev)
     ws = gc.Workspace()
     gc.gc_set_wait_limit(SHORT)
+    # every row tile on the tensor-core GEMM, so the withheld copy is waited on
+    gc.gc_set_decode_policy(gc.GC_DECODE_DENSE)
     try:
         gc.gc_inject_stall(gc.GC_STALL_COMBINE)
         gc.gc_decode_batch(Rd, ell, od, N, m, delta, pd, Gd, ws=ws)
@@ -78,6 +80,7 @@ def test_combine_stall_times_out_then_recovers(gc):
     finally:
         gc.gc_inject_stall(0)
         gc.gc_set_wait_limit(0)
+        gc.gc_set_decode_policy(gc.GC_DECODE_AUTO)
     res = gc.gc_decode_batch(Rd, ell, od, N, m, delta, pd, Gd, ws=ws)
     gc.gc_status(ws)
     Gh = to_np(res["Ghat"])

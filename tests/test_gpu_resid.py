@@ -1,0 +1,207 @@
+"""The two paths of the batched decode against the oracle and each other.
+
+Every decode block Pi_{b,i} is I_ell when Delta_i >= ell (Sec. II-A), so the
+library writes the rows of a 128-row tile either as sum_i g_{D_i} plus the
+non-identity blocks (residual path) or by the tensor-core GEMM C . G; the
+choice is made per tile on the device (gc_set_decode_policy).  These tests
+force each policy and let the automatic one mix them: tiles of exact and of
+approximate patterns side by side, patterns straddling two tiles (ell = 3),
+lists longer than the residual path holds, ragged block lengths, and a
+decode matrix that is not a projector (gc_decode_combine)."""
+import numpy as np
+import pytest
+import torch
+
+import oracle as O
+from _parity import assert_grad_close, assert_mse_close, dev_tensors, to_np
+from workloads import all_patterns, get, make_data, make_patterns, make_R
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def gc():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    import paper_2405_19509_gb300 as m
+    yield m
+    m.gc_set_decode_policy(m.GC_DECODE_AUTO)
+
+
+def _policies(gc):
+    return {"auto": gc.GC_DECODE_AUTO, "dense": gc.GC_DECODE_DENSE, "residual": gc.GC_DECODE_RESIDUAL}
+
+
+def _decode(gc, policy, *args, **kw):
+    gc.gc_set_decode_policy(policy)
+    try:
+        res = gc.gc_decode_batch(*args, **kw)
+        torch.cuda.synchronize()
+    finally:
+        gc.gc_set_decode_policy(gc.GC_DECODE_AUTO)
+    return res
+
+
+def _copies(order, psi, N):
+    """Delta per (pattern, chunk) for an order given as m x delta."""
+    m, delta = order.shape
+    D = np.zeros((psi.shape[0], N), dtype=np.int64)
+    for j in range(m):
+        for p in range(delta):
+            i = order[j, p]
+            if i >= 0:
+                D[:, i] += psi[:, j] > p
+    return D
+
+
+def _tiny_G():
+    cfg = get("tiny")
+    data = make_data(cfg)
+    G64 = O.chunk_gradients(data["X"].numpy(), data["y"].numpy(), data["w"].numpy(), cfg.N, cfg.n_c,
+                            O.LSQ)
+    return G64.astype(np.float32)
+
+
+@pytest.mark.parametrize("ell", [1, 2, 3])
+def test_policies_every_tiny_pattern(gc, ell):
+    """All 4,096 patterns of the 6-worker workload plus 256 seeded ones under
+    each policy: decoded gradients and errors against the oracle; on the
+    residual path an exact pattern's error is exactly zero."""
+    cfg = get("tiny")
+    N, m, delta, d = cfg.N, cfg.m, cfg.delta, cfg.d
+    order = O.cyclic_order(N, m, delta)
+    R = make_R(cfg, ell)
+    psi = np.concatenate([all_patterns(m, delta), make_patterns(cfg)])
+    G32 = _tiny_G()
+    Gref = G32.astype(np.float64)
+    gsum = Gref.sum(axis=0)
+    floor = 1e-8 * float(gsum @ gsum) / d
+    Rd, od, pd = dev_tensors(R, order, psi)
+    Gd = torch.from_numpy(G32).cuda()
+    out = {k: _decode(gc, v, Rd, ell, od, N, m, delta, pd, Gd) for k, v in _policies(gc).items()}
+    exact = _copies(order, psi, N).min(axis=1) >= ell
+    assert np.array_equal(to_np(out["residual"]["grad_mse"])[exact], np.zeros(int(exact.sum())))
+    Gh = {k: to_np(v["Ghat"]) for k, v in out.items()}
+    ms = {k: to_np(v["grad_mse"]) for k, v in out.items()}
+    for b in range(psi.shape[0]):
+        r = O.run_pattern(R, order, psi[b], N, Gref, want_transmit=False)
+        for k in Gh:
+            assert_grad_close(Gh[k][b], r.ghat, f"{k} b={b}")
+            assert_mse_close(ms[k][b], r.grad_mse, floor, f"{k} mse b={b}")
+
+
+@pytest.mark.parametrize("ell", [2, 3])
+def test_mixed_and_straddling_tiles(gc, ell):
+    """Runs of 64 exact patterns (all workers finished) alternate with runs of
+    uniformly random ones, so the automatic policy sends some tiles to each
+    path; with ell = 3 patterns straddle tile boundaries."""
+    cfg = get("tiny")
+    N, m, delta, d = cfg.N, cfg.m, cfg.delta, cfg.d
+    order = O.cyclic_order(N, m, delta)
+    R = make_R(cfg, ell)
+    rnd = make_patterns(cfg, npat=512, stream=7)
+    runs = []
+    for r in range(8):
+        runs.append(np.full((64, m), delta, dtype=np.int32) if r % 2 == 0 else rnd[64 * r:64 * r + 64])
+    psi = np.concatenate(runs + [rnd[:5]])   # a ragged last tile
+    G32 = _tiny_G()
+    Gref = G32.astype(np.float64)
+    gsum = Gref.sum(axis=0)
+    floor = 1e-8 * float(gsum @ gsum) / d
+    Rd, od, pd = dev_tensors(R, order, psi)
+    res = _decode(gc, gc.GC_DECODE_AUTO, Rd, ell, od, N, m, delta, pd, torch.from_numpy(G32).cuda())
+    dense = _decode(gc, gc.GC_DECODE_DENSE, Rd, ell, od, N, m, delta, pd, torch.from_numpy(G32).cuda())
+    Gh, ms = to_np(res["Ghat"]), to_np(res["grad_mse"])
+    for b in range(psi.shape[0]):
+        r = O.run_pattern(R, order, psi[b], N, Gref, want_transmit=False)
+        assert_grad_close(Gh[b], r.ghat, f"auto b={b}")
+        assert_mse_close(ms[b], r.grad_mse, floor, f"auto mse b={b}")
+    assert np.max(np.abs(Gh - to_np(dense["Ghat"]))) <= 1e-5 * np.max(np.abs(Gh))
+
+
+def test_list_overflow_goes_to_the_gemm(gc):
+    """m = N = 64, delta = 8, l = 2 with Binomial(8, 0.3) patterns: many have
+    more non-identity blocks than the residual list holds (16), so even the
+    residual policy must decode their tiles on the GEMM; sampled patterns,
+    the heaviest included, against the oracle."""
+    cfg = get("mse_sweep")
+    N, m, delta, ell, d = cfg.N, cfg.m, cfg.delta, 2, 2048
+    order = O.cyclic_order(N, m, delta)
+    R = make_R(cfg, ell)
+    psi = make_patterns(cfg, npat=384, p=0.3)
+    nnz = (_copies(order, psi, N) < ell).sum(axis=1)
+    assert nnz.max() > 16
+    rng = np.random.default_rng(3)
+    G32 = rng.standard_normal((N, d)).astype(np.float32)
+    Gref = G32.astype(np.float64)
+    gsum = Gref.sum(axis=0)
+    floor = 1e-8 * float(gsum @ gsum) / d
+    Rd, od, pd = dev_tensors(R, order, psi)
+    Gd = torch.from_numpy(G32).cuda()
+    outs = [_decode(gc, v, Rd, ell, od, N, m, delta, pd, Gd) for v in _policies(gc).values()]
+    picks = sorted(set([int(np.argmax(nnz)), int(np.argmin(nnz))] + list(range(0, 384, 29))))
+    for b in picks:
+        r = O.run_pattern(R, order, psi[b], N, Gref, want_transmit=False)
+        for res in outs:
+            assert_grad_close(to_np(res["Ghat"][b]), r.ghat, f"b={b} nnz={nnz[b]}")
+            assert_mse_close(float(res["grad_mse"][b]), r.grad_mse, floor, f"b={b}")
+
+
+@pytest.mark.parametrize("d,ell,npat", [(67, 2, 1), (5, 4, 3), (64, 3, 129), (1, 1, 130), (1030, 2, 200)])
+def test_ragged_shapes_both_paths(gc, d, ell, npat):
+    """Block lengths that are not multiples of 4 (scalar loads and stores),
+    zero padding past d, a single pattern, a last tile of one row."""
+    N = m = 6
+    delta = 3
+    order = O.cyclic_order(N, m, delta)
+    rng = np.random.default_rng(d * 100 + ell)
+    R = rng.standard_normal((ell, m))
+    psi = rng.integers(0, delta + 1, size=(npat, m)).astype(np.int32)
+    psi[0] = delta
+    G32 = rng.standard_normal((N, d)).astype(np.float32)
+    Gref = G32.astype(np.float64)
+    gsum = Gref.sum(axis=0)
+    floor = 1e-8 * float(gsum @ gsum) / d
+    Rd, od, pd = dev_tensors(R, order, psi)
+    Gd = torch.from_numpy(G32).cuda()
+    for pol in (gc.GC_DECODE_DENSE, gc.GC_DECODE_RESIDUAL):
+        res = _decode(gc, pol, Rd, ell, od, N, m, delta, pd, Gd)
+        for b in range(npat):
+            r = O.run_pattern(R, order, psi[b], N, Gref, want_transmit=False)
+            assert_grad_close(to_np(res["Ghat"][b]), r.ghat, f"policy {pol} b={b}")
+            assert_mse_close(float(res["grad_mse"][b]), r.grad_mse, floor, f"policy {pol} b={b}")
+
+
+def test_combine_non_projector_matrix(gc):
+    """gc_decode_combine with a decode matrix that is near, but not exactly,
+    the identity blocks (every block differs from I): both paths against the
+    plain product C . G in fp64 and against each other; MSE-only as well."""
+    N, ell, npat, d = 6, 2, 300, 1024
+    rng = np.random.default_rng(17)
+    C = np.tile(np.kron(np.ones((1, N)), np.eye(ell)), (npat, 1, 1))
+    C += 1e-3 * rng.standard_normal(C.shape)
+    C[::5] = np.kron(np.ones((1, N)), np.eye(ell))  # every fifth pattern exact
+    C = C.astype(np.float32)
+    G32 = rng.standard_normal((N, d)).astype(np.float32)
+    L = d // ell
+    Gv = G32.astype(np.float64).reshape(N, ell, L).reshape(N * ell, L)
+    ref = np.einsum("bkj,jc->bkc", C.astype(np.float64), Gv).reshape(npat, d)
+    gsum = G32.astype(np.float64).sum(axis=0)
+    mref = ((ref - gsum) ** 2).sum(axis=1) / d
+    floor = 1e-8 * float(gsum @ gsum) / d
+    Cd, Gd = torch.from_numpy(C).cuda(), torch.from_numpy(G32).cuda()
+    got = {}
+    for name, pol in (("dense", gc.GC_DECODE_DENSE), ("residual", gc.GC_DECODE_RESIDUAL)):
+        gc.gc_set_decode_policy(pol)
+        try:
+            res = gc.gc_decode_combine(Cd, ell, N, Gd)
+            mo = gc.gc_decode_combine(Cd, ell, N, Gd, Ghat=False)["grad_mse"]
+            torch.cuda.synchronize()
+        finally:
+            gc.gc_set_decode_policy(gc.GC_DECODE_AUTO)
+        got[name] = to_np(res["Ghat"])
+        for b in range(npat):
+            assert_grad_close(got[name][b], ref[b], f"{name} b={b}")
+            assert_mse_close(float(res["grad_mse"][b]), mref[b], floor, f"{name} mse b={b}")
+            assert_mse_close(float(mo[b]), mref[b], floor, f"{name} mse-only b={b}")
+    assert np.max(np.abs(got["dense"] - got["residual"])) <= 1e-5 * np.max(np.abs(ref))
