@@ -10,91 +10,156 @@
 namespace gc {
 
 // T[b][j][c] = sum_{p < psi[b][j]} sum_k E[b][j][p][k] * g_{order[j][p]}[k*L + c]
-// (g zero past d).  Block = (column stripe, worker j, group of up to
-// kEncPats patterns).  The patterns share worker j's chunk list, so each
-// thread loads g_{order[j][p]}[k*L + c] once per slot p and feeds it to
-// every pattern of the group that processed slot p (kEncPats accumulators)
-// instead of once per pattern; threads take V consecutive columns (16-byte
-// loads when rows are 16-byte aligned) and stride over the block's columns,
-// so the staging of the group's coefficients (fp32) and processed counts in
-// shared memory -- kEncPats * (delta * ell + 1) + delta words, small enough to
-// fit beside a resident kernel that holds nearly all of an SM's -- is paid
-// once per block, not once per 256 columns.
-constexpr int kEncPats = 8;
-constexpr int kEncThreads = 256;
+// (g zero past d), eq. (2).
+//
+// Under the cyclic assignment (order[j][p] = (j + p) mod N, Sec. III) the
+// holders of chunk i are the workers i, i-1, ..., i-delta+1, so a block that
+// sweeps the chunks in order over one column stripe keeps a ring of
+// per-worker accumulators in registers: each loaded stripe of g_{D_i} feeds
+// every holder of D_i once, and a worker's transmission is stored when its
+// window of chunks has passed.  The chunk gradients are read once per
+// (pattern, worker group) instead of once per worker and slot.
+// Block = (pattern b, column stripe, worker group [j0, j1)).  The ring has DR
+// slots (DR = the power of two >= delta); the coefficients are staged
+// diagonally, s_d[k][w][p] = E[b][j0 + w - p][p][k] for the worker that holds
+// sweep position w in slot p (zero past its psi, for p >= delta and outside
+// the group), so every chunk step is DR/4 vector loads from shared memory and
+// DR*V FMAs with no branches; positions past the group's range add zeros.
+// A transmission is summed over slots p ascending, blocks k ascending within
+// a slot -- the same order in the direct form, which a block whose workers'
+// orders are not cyclic (an explicit order) uses instead.
+constexpr int kEncThreads = 128;
+constexpr int kEncSmemFloats = 12288;  // staged coefficients (48 KB)
+
+__device__ __forceinline__ void enc_load(const float* __restrict__ gi, long long col, int c, int L,
+                                         int d, bool vec, float* g, int V) {
+  if (vec && V == 4 && c + 3 < L && col + 3 < d) {
+    const float4 q = __ldg(reinterpret_cast<const float4*>(gi + col));
+    g[0] = q.x; g[1] = q.y; g[2] = q.z; g[3] = q.w;
+  } else if (vec && V == 2 && c + 1 < L && col + 1 < d) {
+    const float2 q = __ldg(reinterpret_cast<const float2*>(gi + col));
+    g[0] = q.x; g[1] = q.y;
+  } else {
+    for (int v = 0; v < V; ++v) g[v] = (c + v < L && col + v < d) ? __ldg(gi + col + v) : 0.f;
+  }
+}
+
 template <int V>
+__device__ __forceinline__ void enc_store(float* __restrict__ Tr, int c, int L, bool vec, const float* a) {
+  if (vec && V == 4 && c + 3 < L) {
+    *reinterpret_cast<float4*>(Tr) = make_float4(a[0], a[V > 1 ? 1 : 0], a[V > 2 ? 2 : 0], a[V > 3 ? 3 : 0]);
+  } else if (vec && V == 2 && c + 1 < L) {
+    *reinterpret_cast<float2*>(Tr) = make_float2(a[0], a[V > 1 ? 1 : 0]);
+  } else {
+#pragma unroll
+    for (int v = 0; v < V; ++v)
+      if (c + v < L) Tr[v] = a[v];
+  }
+}
+
+// Workers per group so that the diagonal staging fits (and at most 256).
+__host__ __device__ inline int enc_group_max(int DR, int ell) {
+  const int j = kEncSmemFloats / (ell * DR) - DR;
+  return j < 1 ? 1 : (j > 256 ? 256 : j);
+}
+
+template <int DR, int V>
 __global__ void __launch_bounds__(kEncThreads)
     k_encode(const double* __restrict__ E, const int32_t* __restrict__ order,
              const int32_t* __restrict__ psi, int N, int m, int delta, int ell, int npat,
-             const float* __restrict__ G, int d, int L, float* __restrict__ T) {
-  extern __shared__ float s_dyn[];
-  // worker j varies fastest across the grid, so the blocks resident at one
-  // time cover all workers on a few column stripes: the chunk-gradient
-  // columns they read (each used by every holder of the chunk) stay in L2,
-  // where worker-major order swept whole rows of many chunks and re-read them
-  const int j = blockIdx.x, b0 = blockIdx.z * kEncPats;
-  const int nb = min(kEncPats, npat - b0);
+             const float* __restrict__ G, int d, int L, int J, int vec, float* __restrict__ T) {
+  __shared__ __align__(16) float s_e[kEncSmemFloats];
+  __shared__ int s_np[256];               // processed counts of the group's workers (J <= 256)
+  const int b = blockIdx.x;               // pattern fastest: blocks on one stripe share G in L2
+  const int j0 = blockIdx.z * J, j1 = min(m, j0 + J);
+  const int nj = j1 - j0;
   const int de = delta * ell;
-  float* s_e = s_dyn;                                                // [nb][delta * ell]
-  int* s_np = reinterpret_cast<int*>(s_dyn + kEncPats * de);         // [kEncPats]
-  int* s_chunk = s_np + kEncPats;                                    // [delta]
-  if (threadIdx.x < kEncPats) {
-    int np = 0;
-    if ((int)threadIdx.x < nb) {
-      np = psi[(size_t)(b0 + threadIdx.x) * m + j];
-      np = np < 0 ? 0 : (np > delta ? delta : np);  // bad values are flagged by the solve
+  const int c = (blockIdx.y * kEncThreads + threadIdx.x) * V;
+  for (int t = threadIdx.x; t < nj; t += kEncThreads) {
+    int np = psi[(size_t)b * m + j0 + t];
+    s_np[t] = np < 0 ? 0 : (np > delta ? delta : np);  // bad values are flagged by the solve
+  }
+  int cyc = delta <= DR ? 1 : 0;
+  for (int t = threadIdx.x; t < nj * delta; t += kEncThreads) {
+    const int jj = t / delta, p = t - jj * delta;
+    if (order[(size_t)(j0 + jj) * delta + p] != (j0 + jj + p) % N) cyc = 0;
+  }
+  cyc = __syncthreads_and(cyc);
+  const double* Eb = E + ((size_t)b * m + j0) * de;
+  if (!cyc) {
+    // direct form: s_e[jj][p][k]
+    for (int t = threadIdx.x; t < nj * de; t += kEncThreads) s_e[t] = (float)Eb[t];
+    __syncthreads();
+    if (c >= L) return;
+    for (int jj = 0; jj < nj; ++jj) {
+      float acc[V];
+#pragma unroll
+      for (int v = 0; v < V; ++v) acc[v] = 0.f;
+      const int j = j0 + jj;
+      for (int p = 0; p < s_np[jj]; ++p) {
+        const int i = order[(size_t)j * delta + p];
+        if (i < 0 || i >= N) continue;
+        const float* gi = G + (size_t)i * d;
+        for (int k = 0; k < ell; ++k) {
+          float g[V];
+          enc_load(gi, (long long)k * L + c, c, L, d, vec != 0, g, V);
+          const float e = s_e[jj * de + p * ell + k];
+#pragma unroll
+          for (int v = 0; v < V; ++v) acc[v] = fmaf(e, g[v], acc[v]);
+        }
+      }
+      enc_store<V>(T + ((size_t)b * m + j) * L + c, c, L, vec != 0, acc);
     }
-    s_np[threadIdx.x] = np;
+    return;
   }
-  for (int t = threadIdx.x; t < nb * de; t += blockDim.x) {
-    const int bb = t / de, r = t - bb * de;
-    s_e[t] = (float)E[((size_t)(b0 + bb) * m + j) * de + r];
+  // diagonal staging: s_e[(k * W + w) * DR + p], w = 0 .. nj + DR - 2 sweep positions
+  const int W = nj + DR - 1;
+  for (int t = threadIdx.x; t < ell * W * DR; t += kEncThreads) {
+    const int p = t % DR, w = (t / DR) % W, k = t / (DR * W);
+    const int jj = w - p;
+    float e = 0.f;
+    if (jj >= 0 && jj < nj && p < s_np[jj]) e = (float)Eb[(size_t)jj * de + p * ell + k];
+    s_e[t] = e;
   }
-  for (int t = threadIdx.x; t < delta; t += blockDim.x) s_chunk[t] = order[(size_t)j * delta + t];
   __syncthreads();
-  int pmax = 0;
+  if (c >= L) return;  // no barrier below
+  float acc[DR][V];
 #pragma unroll
-  for (int bb = 0; bb < kEncPats; ++bb) pmax = max(pmax, s_np[bb]);
-  for (int c = (blockIdx.y * kEncThreads + threadIdx.x) * V; c < L; c += gridDim.y * kEncThreads * V) {
-    float acc[kEncPats][V];
+  for (int r = 0; r < DR; ++r)
 #pragma unroll
-    for (int bb = 0; bb < kEncPats; ++bb)
+    for (int v = 0; v < V; ++v) acc[r][v] = 0.f;
+  // sweep position w = vv - j0 holds chunk vv mod N; worker j0 + w - p takes it
+  // in slot p, ring slot (w - p) mod DR; worker j0 + w - DR + 1 is complete after it
+  for (int w0 = 0; w0 < W; w0 += DR) {
 #pragma unroll
-      for (int v = 0; v < V; ++v) acc[bb][v] = 0.f;
-    for (int p = 0; p < pmax; ++p) {
-      const int i = s_chunk[p];
-      if (i < 0 || i >= N) continue;
+    for (int u = 0; u < DR; ++u) {
+      const int w = w0 + u;
+      if (w >= W) break;
+      const int i = (j0 + w) % N;
       const float* gi = G + (size_t)i * d;
       for (int k = 0; k < ell; ++k) {
-        const int col = k * L + c;
         float g[V];
-        if (V == 4 && col + 3 < d) {
-          const float4 q = __ldg(reinterpret_cast<const float4*>(gi + col));
-          g[0] = q.x; g[V > 1 ? 1 : 0] = q.y; g[V > 2 ? 2 : 0] = q.z; g[V > 3 ? 3 : 0] = q.w;
-        } else {
+        enc_load(gi, (long long)k * L + c, c, L, d, vec != 0, g, V);
+        const float4* e4 = reinterpret_cast<const float4*>(s_e + ((size_t)k * W + w) * DR);
 #pragma unroll
-          for (int v = 0; v < V; ++v) g[v] = (c + v < L && col + v < d) ? __ldg(gi + col + v) : 0.f;
-        }
+        for (int q = 0; q < DR / 4; ++q) {
+          const float4 e = e4[q];
+          const float ev[4] = {e.x, e.y, e.z, e.w};
 #pragma unroll
-        for (int bb = 0; bb < kEncPats; ++bb)
-          if (p < s_np[bb]) {
-            const float e = s_e[bb * de + p * ell + k];
+          for (int h = 0; h < 4; ++h) {
+            const int p = 4 * q + h;
 #pragma unroll
-            for (int v = 0; v < V; ++v) acc[bb][v] = fmaf(e, g[v], acc[bb][v]);
+            for (int v = 0; v < V; ++v)
+              acc[(u - p) & (DR - 1)][v] = fmaf(ev[h], g[v], acc[(u - p) & (DR - 1)][v]);
           }
+        }
       }
-    }
+      const int jj = w - DR + 1;
+      if (jj >= 0) {  // jj < nj since w < nj + DR - 1
+        float* a = acc[(u + 1) & (DR - 1)];
+        enc_store<V>(T + ((size_t)b * m + j0 + jj) * L + c, c, L, vec != 0, a);
 #pragma unroll
-    for (int bb = 0; bb < kEncPats; ++bb) {
-      if (bb >= nb) break;
-      float* Tr = T + ((size_t)(b0 + bb) * m + j) * L + c;
-      if (V == 4 && c + 3 < L) {
-        *reinterpret_cast<float4*>(Tr) = make_float4(acc[bb][0], acc[bb][V > 1 ? 1 : 0],
-                                                     acc[bb][V > 2 ? 2 : 0], acc[bb][V > 3 ? 3 : 0]);
-      } else {
-#pragma unroll
-        for (int v = 0; v < V; ++v)
-          if (c + v < L) Tr[v] = acc[bb][v];
+        for (int v = 0; v < V; ++v) a[v] = 0.f;
       }
     }
   }
@@ -104,22 +169,34 @@ int launch_encode(const double* E, const int32_t* order, const int32_t* psi, int
                   int delta, int ell, int npat, const float* G, int d, float* T, cudaStream_t s) {
   const int L = (d + ell - 1) / ell;
   if ((long long)npat * m * L == 0) return GC_OK;
-  const int groups = (npat + kEncPats - 1) / kEncPats;
-  if (groups > 65535 || m > 65535) return fail(GC_ERR_UNSUPPORTED, "encode grid: npat / 8 and m <= 65535");
-  // 16-byte column vectors when every row start is 16-byte aligned
-  const bool vec = d % 4 == 0 && L % 4 == 0 && reinterpret_cast<uintptr_t>(G) % 16 == 0 &&
-                   reinterpret_cast<uintptr_t>(T) % 16 == 0;
-  const int V = vec ? 4 : 1;
+  // ring of the smallest power of two >= delta; 2 columns per thread with 32 slots
+  const int DR = delta <= 4 ? 4 : delta <= 8 ? 8 : delta <= 16 ? 16 : 32;
+  const int V = DR == 32 ? 2 : 4;
+  const bool vec = d % V == 0 && L % V == 0 && reinterpret_cast<uintptr_t>(G) % (4 * V) == 0 &&
+                   reinterpret_cast<uintptr_t>(T) % (4 * V) == 0;
   const long long stripes = ((long long)L + (long long)kEncThreads * V - 1) / ((long long)kEncThreads * V);
-  // enough blocks for a few waves; each block strides over the rest of its row
-  const long long want = std::max<long long>(1, (long long)device_sm_count() * 32 / ((long long)m * groups));
-  const int gx = (int)std::max<long long>(1, std::min<long long>(stripes, want));
-  dim3 grid(m, gx, groups);
-  const size_t smem = ((size_t)kEncPats * delta * ell + kEncPats + delta) * sizeof(float);
-  if (vec)
-    k_encode<4><<<grid, kEncThreads, smem, s>>>(E, order, psi, N, m, delta, ell, npat, G, d, L, T);
-  else
-    k_encode<1><<<grid, kEncThreads, smem, s>>>(E, order, psi, N, m, delta, ell, npat, G, d, L, T);
+  // worker groups: as few as the staging allows, more when the patterns and
+  // stripes alone give under about four blocks per SM
+  int J = std::min(m, enc_group_max(DR, ell));
+  const long long want = 4LL * device_sm_count();
+  const long long have = (long long)npat * stripes;
+  if (have < want) {
+    const long long groups = (want + have - 1) / have;
+    J = (int)std::min<long long>(J, std::max<long long>(std::min(delta, m), (m + groups - 1) / groups));
+  }
+  const int ngroups = (m + J - 1) / J;
+  if (npat > 2147483647 || stripes > 65535 || ngroups > 65535)
+    return fail(GC_ERR_UNSUPPORTED, "encode grid too large");
+#define GC_ENC(R, VV) \
+  k_encode<R, VV><<<dim3((unsigned)npat, (unsigned)stripes, (unsigned)ngroups), kEncThreads, 0, s>>>( \
+      E, order, psi, N, m, delta, ell, npat, G, d, L, J, vec ? 1 : 0, T)
+  switch (DR) {
+    case 4: GC_ENC(4, 4); break;
+    case 8: GC_ENC(8, 4); break;
+    case 16: GC_ENC(16, 4); break;
+    default: GC_ENC(32, 2); break;
+  }
+#undef GC_ENC
   count_launches(1);
   return cuda_check(cudaGetLastError(), "k_encode");
 }

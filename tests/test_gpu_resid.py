@@ -54,6 +54,22 @@ def _copies(order, psi, N):
     return D
 
 
+def _residual_rows(nnz, ell, ksp):
+    """Rows the residual policy leaves off the GEMM: a 128-row tile stays on
+    the residual path unless a pattern overlapping it has more than `ksp`
+    non-identity blocks or more than 32 of its rows need corrections."""
+    npat = nnz.shape[0]
+    M = npat * ell
+    row_pat = np.arange(M) // ell
+    res = np.zeros(M, dtype=bool)
+    for t0 in range(0, M, 128):
+        rows = np.arange(t0, min(M, t0 + 128))
+        pats = np.unique(row_pat[rows])
+        corrected = int((nnz[row_pat[rows]] > 0).sum())
+        res[rows] = not (np.any(nnz[pats] > ksp) or corrected > 32)
+    return res
+
+
 def _tiny_G():
     cfg = get("tiny")
     data = make_data(cfg)
@@ -65,8 +81,8 @@ def _tiny_G():
 @pytest.mark.parametrize("ell", [1, 2, 3])
 def test_policies_every_tiny_pattern(gc, ell):
     """All 4,096 patterns of the 6-worker workload plus 256 seeded ones under
-    each policy: decoded gradients and errors against the oracle; on the
-    residual path an exact pattern's error is exactly zero."""
+    each policy: decoded gradients and errors against the oracle (tiles with
+    more than 32 corrected rows stay on the GEMM under every policy)."""
     cfg = get("tiny")
     N, m, delta, d = cfg.N, cfg.m, cfg.delta, cfg.d
     order = O.cyclic_order(N, m, delta)
@@ -79,8 +95,6 @@ def test_policies_every_tiny_pattern(gc, ell):
     Rd, od, pd = dev_tensors(R, order, psi)
     Gd = torch.from_numpy(G32).cuda()
     out = {k: _decode(gc, v, Rd, ell, od, N, m, delta, pd, Gd) for k, v in _policies(gc).items()}
-    exact = _copies(order, psi, N).min(axis=1) >= ell
-    assert np.array_equal(to_np(out["residual"]["grad_mse"])[exact], np.zeros(int(exact.sum())))
     Gh = {k: to_np(v["Ghat"]) for k, v in out.items()}
     ms = {k: to_np(v["grad_mse"]) for k, v in out.items()}
     for b in range(psi.shape[0]):
@@ -112,6 +126,11 @@ def test_mixed_and_straddling_tiles(gc, ell):
     res = _decode(gc, gc.GC_DECODE_AUTO, Rd, ell, od, N, m, delta, pd, torch.from_numpy(G32).cuda())
     dense = _decode(gc, gc.GC_DECODE_DENSE, Rd, ell, od, N, m, delta, pd, torch.from_numpy(G32).cuda())
     Gh, ms = to_np(res["Ghat"]), to_np(res["grad_mse"])
+    if ell == 2:
+        # a run of 64 exact patterns is one whole tile: residual path, ghat = sum_i g, zero error
+        for r0 in (0, 128, 256, 384):
+            assert np.all(ms[r0:r0 + 64] == 0.0)
+            assert np.array_equal(Gh[r0], Gh[r0 + 63])
     for b in range(psi.shape[0]):
         r = O.run_pattern(R, order, psi[b], N, Gref, want_transmit=False)
         assert_grad_close(Gh[b], r.ghat, f"auto b={b}")
@@ -120,10 +139,10 @@ def test_mixed_and_straddling_tiles(gc, ell):
 
 
 def test_list_overflow_goes_to_the_gemm(gc):
-    """m = N = 64, delta = 8, l = 2 with Binomial(8, 0.3) patterns: many have
-    more non-identity blocks than the residual list holds (16), so even the
-    residual policy must decode their tiles on the GEMM; sampled patterns,
-    the heaviest included, against the oracle."""
+    """m = N = 64, delta = 8, l = 2 with Binomial(8, 0.3) patterns: nearly every
+    pattern needs corrections, more rows than a residual tile holds (32), so
+    even the residual policy must decode those tiles on the GEMM; sampled
+    patterns, the heaviest included, against the oracle."""
     cfg = get("mse_sweep")
     N, m, delta, ell, d = cfg.N, cfg.m, cfg.delta, 2, 2048
     order = O.cyclic_order(N, m, delta)
@@ -147,6 +166,48 @@ def test_list_overflow_goes_to_the_gemm(gc):
             assert_mse_close(float(res["grad_mse"][b]), r.grad_mse, floor, f"b={b}")
 
 
+def _sparse_stragglers(rng, npat, m, delta, every):
+    """Every worker finished, except in every `every`-th pattern (offset 1),
+    whose counts are uniform in 0..delta: residual tiles with corrected rows."""
+    psi = np.full((npat, m), delta, dtype=np.int32)
+    idx = np.arange(1, npat, every)
+    psi[idx] = rng.integers(0, delta + 1, size=(idx.size, m))
+    return psi
+
+
+@pytest.mark.parametrize("ell", [1, 2, 3])
+def test_sparse_stragglers_tiny(gc, ell):
+    """4096 patterns of the 6-worker workload, one in five with stragglers:
+    the residual tiles now hold corrected rows (the list and slot machinery);
+    every pattern against the oracle under each policy."""
+    cfg = get("tiny")
+    N, m, delta, d = cfg.N, cfg.m, cfg.delta, cfg.d
+    order = O.cyclic_order(N, m, delta)
+    R = make_R(cfg, ell)
+    psi = _sparse_stragglers(np.random.default_rng(40 + ell), 4096, m, delta, 5)
+    G32 = _tiny_G()
+    Gref = G32.astype(np.float64)
+    gsum = Gref.sum(axis=0)
+    floor = 1e-8 * float(gsum @ gsum) / d
+    Rd, od, pd = dev_tensors(R, order, psi)
+    Gd = torch.from_numpy(G32).cuda()
+    out = {k: _decode(gc, v, Rd, ell, od, N, m, delta, pd, Gd) for k, v in _policies(gc).items()}
+    nnz = (_copies(order, psi, N) < ell).sum(axis=1)
+    res_rows = _residual_rows(nnz, ell, N).reshape(-1, ell).all(axis=1)
+    assert res_rows.mean() > 0.5, "most tiles should stay on the residual path"
+    exact_res = (nnz == 0) & res_rows
+    assert np.all(to_np(out["residual"]["grad_mse"])[exact_res] == 0.0)
+    cache = {}
+    for b in range(psi.shape[0]):
+        key = psi[b].tobytes()
+        if key not in cache:
+            cache[key] = O.run_pattern(R, order, psi[b], N, Gref, want_transmit=False)
+        r = cache[key]
+        for k, res in out.items():
+            assert_grad_close(to_np(res["Ghat"][b]), r.ghat, f"{k} b={b}")
+            assert_mse_close(float(res["grad_mse"][b]), r.grad_mse, floor, f"{k} mse b={b}")
+
+
 @pytest.mark.parametrize("d,ell,npat", [(67, 2, 1), (5, 4, 3), (64, 3, 129), (1, 1, 130), (1030, 2, 200)])
 def test_ragged_shapes_both_paths(gc, d, ell, npat):
     """Block lengths that are not multiples of 4 (scalar loads and stores),
@@ -156,8 +217,9 @@ def test_ragged_shapes_both_paths(gc, d, ell, npat):
     order = O.cyclic_order(N, m, delta)
     rng = np.random.default_rng(d * 100 + ell)
     R = rng.standard_normal((ell, m))
-    psi = rng.integers(0, delta + 1, size=(npat, m)).astype(np.int32)
-    psi[0] = delta
+    psi = _sparse_stragglers(rng, npat, m, delta, 3)
+    if npat == 1:
+        psi[0] = rng.integers(0, delta + 1, size=m)
     G32 = rng.standard_normal((N, d)).astype(np.float32)
     Gref = G32.astype(np.float64)
     gsum = Gref.sum(axis=0)
@@ -173,14 +235,16 @@ def test_ragged_shapes_both_paths(gc, d, ell, npat):
 
 
 def test_combine_non_projector_matrix(gc):
-    """gc_decode_combine with a decode matrix that is near, but not exactly,
-    the identity blocks (every block differs from I): both paths against the
-    plain product C . G in fp64 and against each other; MSE-only as well."""
+    """gc_decode_combine with a decode matrix whose blocks, in one pattern in
+    four, are near but not exactly I (every block of such a pattern differs
+    from I): both paths against the plain product C . G in fp64 and against
+    each other; MSE-only as well."""
     N, ell, npat, d = 6, 2, 300, 1024
     rng = np.random.default_rng(17)
     C = np.tile(np.kron(np.ones((1, N)), np.eye(ell)), (npat, 1, 1))
     C += 1e-3 * rng.standard_normal(C.shape)
-    C[::5] = np.kron(np.ones((1, N)), np.eye(ell))  # every fifth pattern exact
+    keep = np.arange(npat) % 4 != 1
+    C[keep] = np.kron(np.ones((1, N)), np.eye(ell))  # three patterns in four exact
     C = C.astype(np.float32)
     G32 = rng.standard_normal((N, d)).astype(np.float32)
     L = d // ell
