@@ -334,12 +334,11 @@ __global__ void __launch_bounds__(kResidThreads) k_decode_resid(const float* __r
 #pragma unroll
         for (int kp = 0; kp < ELL; ++kp) corr = fmaf(__ldg(Dr + kp), sg[(i * ELL + kp) * W + lane], corr);
       }
-      if (Ghat) {
-        const long long col = (long long)k * L + c0 + lane;
-        if (c0 + lane < L && col < d) __stcs(Ghat + (size_t)b * d + col, ss[k * W + lane] + corr);
-      }
+      // output column k*L + c0 + lane exists (padding past L and past d does not)
+      const bool col_ok = c0 + lane < L && (long long)k * L + c0 + lane < d;
+      if (Ghat && col_ok) __stcs(Ghat + (size_t)b * d + (size_t)k * L + c0 + lane, ss[k * W + lane] + corr);
       if (rl.msp) {
-        float sq = corr * corr;  // zero on padding lanes: their staged values are zero
+        float sq = col_ok ? corr * corr : 0.f;
 #pragma unroll
         for (int o = 16; o > 0; o >>= 1) sq += __shfl_xor_sync(0xffffffffu, sq, o);
         if (lane == 0) rl.msp[((size_t)mt * kResidRcap + q) * rl.parts + stripe] = sq;
