@@ -1272,7 +1272,110 @@ def extra_workload(args):
             "config": {"workload": "chunk gradients 'dtype,N,n_c,d': " + ", ".join(shapes),
                        "l2": "inputs larger than L2 (8.6 GB per case), else flushed"}})
     line["gpu_launches_total"] = int(gc.gc_kernel_launches() - n0)
+    if not args.no_cpu_baseline:
+        torch.cuda.synchronize()
+        line["cpu_baseline"] = oracle_baseline(args, line)
     print(json.dumps(line), flush=True)
+
+
+def oracle_baseline(args, line):
+    """The fp64 oracle on the host cores, on a bounded sample of the same
+    workload (synthetic inputs of the same shapes; the timing does not depend
+    on the values), in the unit of the line's metric."""
+    import oracle as O
+    from workloads import (get, make_patterns, make_R, make_worker_times, random_regular_graph)
+
+    ell = args.ell
+    rng = np.random.default_rng(12345)
+    cores = os.cpu_count()
+    w = args.workload
+    t0 = time.perf_counter()
+
+    def chunk_rate(N, n_c, d, dtype, loss, k):
+        # k chunks through the oracle's chunk gradient (fp64), seconds per chunk
+        X = rng.standard_normal((k * n_c, d), dtype=np.float32)
+        if dtype == "bf16":
+            import torch
+            X = torch.from_numpy(X).to(torch.bfloat16)
+        y = np.sign(rng.standard_normal(k * n_c)).astype(np.float32)
+        wv = rng.standard_normal(d) / np.sqrt(d)
+        ta = time.perf_counter()
+        O.chunk_gradients(X, y, wv, k, n_c, loss)
+        return (time.perf_counter() - ta) / k
+
+    if w == "encode":
+        cfg = get("decode")
+        N, m, delta, d = cfg.N, cfg.m, cfg.delta, cfg.d
+        L = -(-d // ell)
+        S = 1 << 14
+        order = O.cyclic_order(N, m, delta)
+        psi = make_patterns(cfg, npat=1)[0]
+        B = O.encoding_matrix(make_R(cfg, ell), order, psi, N)
+        Gs = rng.standard_normal((N, ell * S))
+        ta = time.perf_counter()
+        O.encode(B, Gs, order, psi, ell)
+        t = (time.perf_counter() - ta) * (L / S)
+        v = (N * d * 4 + m * L * 4) / t / 1e9
+        sample = f"eq. (2) encode of one pattern on {S} columns of each block, scaled to d = 2^20"
+    elif w == "sweep":
+        cfg = get("mse_sweep")
+        N, m, delta, d = cfg.N, cfg.m, cfg.delta, cfg.d
+        order = O.cyclic_order(N, m, delta)
+        R = make_R(cfg, ell)
+        G = rng.standard_normal((N, d))
+        psi = make_patterns(cfg, npat=16, p=0.5)
+        ta = time.perf_counter()
+        for b in range(psi.shape[0]):
+            O.run_pattern(R, order, psi[b], N, G, want_transmit=False)
+        per = (time.perf_counter() - ta) / psi.shape[0]
+        v = 1.0 / per
+        cg = chunk_rate(N, cfg.n_c, d, "bf16", O.LSQ, 2)
+        sample = (f"16 patterns (p = 0.5): Algorithm 1, decode and errors over all of d "
+                  f"({per:.3f} s each); chunk gradients {cg:.2f} s per chunk "
+                  f"({N * cg:.1f} s per 8.6 GB pass, from 2 chunks)")
+    elif w == "sgd":
+        cfg = get("sgd")
+        N, m, delta, d = cfg.N, cfg.m, cfg.delta, cfg.d
+        cg = chunk_rate(N, cfg.n_c, d, "f32", O.LOGISTIC, 2)
+        order = O.cyclic_order(N, m, delta)
+        R = make_R(cfg, ell)
+        psi = make_patterns(cfg, npat=1)[0]
+        G = rng.standard_normal((N, d))
+        ta = time.perf_counter()
+        B = O.encoding_matrix(R, order, psi, N)
+        gh = O.decode(R, O.encode(B, G, order, psi, ell), d)
+        O.sgd_step(np.zeros(d), gh, cfg.lr, cfg.Ntil)
+        rest = time.perf_counter() - ta
+        it = 2 * N * cg + rest   # the loss is a second pass over X in the oracle
+        v = 1.0 / it
+        sample = (f"chunk gradients of 2 chunks ({cg:.2f} s each), scaled to 128 chunks and counted "
+                  f"twice (gradient pass and loss pass); Algorithm 1 + encode + decode + update of "
+                  f"one realization ({rest:.2f} s)")
+    elif w == "batched":
+        cfg = get("mse_sweep")
+        cg = chunk_rate(cfg.N, cfg.n_c, cfg.d, "bf16", O.LSQ, 2)
+        n_w = 256
+        t = cg * cfg.N * n_w
+        v = 4.0 * cfg.Ntil * cfg.d * n_w / t / 1e12
+        sample = f"one parameter vector, 2 chunks ({cg:.2f} s each), scaled to 64 chunks x 256 vectors"
+    elif w == "trigger":
+        N, delta = 200, 8
+        order = O.cyclic_order(N, N, delta)
+        tau = make_worker_times(N, 200, 22, alpha=delta - ell)
+        ta = time.perf_counter()
+        O.completion_times(order, tau, N, ell)
+        v = 200 / (time.perf_counter() - ta)
+        sample = "200 realizations, cyclic N=m=200, delta=8, alpha = delta - l"
+    elif w == "chunkgrad":
+        sh = (args.shape or "bf16,64,1024,65536").split(",")
+        dt, N, n_c, d = sh[0], int(sh[1]), int(sh[2]), int(sh[3])
+        cg = chunk_rate(N, n_c, d, dt, O.LOGISTIC, 2)
+        v = (n_c * d * (2 if dt == "bf16" else 4) + n_c * 4 + d * 4) / cg / 1e9
+        sample = f"2 chunks of shape {dt},{n_c}x{d} ({cg:.2f} s each)"
+    else:
+        return None
+    return {"value": v, "unit": line.get("unit"), "cores": cores, "kind": "oracle",
+            "sample": sample + f"; {time.perf_counter() - t0:.1f} s of CPU work, NumPy with its BLAS threads"}
 
 
 def main():

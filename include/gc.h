@@ -282,8 +282,11 @@ int gc_find_encoding_coeff(const double* R, int ell, const int32_t* order, int N
  *  - Sizes whose scratch (holder table, plus the memo table when it fits)
  *    exceeds GC_NOALLOC_SCRATCH_BYTES are rejected with GC_ERR_WORKSPACE.
  *  - The first call on each device looks up the array's device address
- *    (cudaGetSymbolAddress) with that device current; make that first call
- *    before any stream capture.
+ *    (cudaGetSymbolAddress) with that device current and caches it with the
+ *    current CUDA context; make that first call before any stream capture.
+ *    A device reset (cudaDeviceReset) destroys the context and the array's
+ *    memory: the next call, in the new context, looks the address up again
+ *    (that call, too, must come before any capture).
  *  - All calls share the array: two calls whose executions overlap on the
  *    GPU (other streams, other host threads) race and give wrong results.
  *  - Device-detected data errors (psi out of range, a singular R_S) are

@@ -13,13 +13,19 @@
 // Host code must not use the array's name as a device address (in host code
 // it names a host-side stand-in).  The first call on each device therefore
 // looks the device address up with cudaGetSymbolAddress while that device is
-// current, checks the result, and caches it; later calls on that device reuse
-// the cached address.  Make that first call before any stream capture.
+// current, checks the result, and caches it with the CUDA context that was
+// current; later calls in the same context reuse the cached address.  A
+// device reset destroys the context and the module's memory with it, so a
+// call made in a new context looks the address up again instead of using a
+// dead one.  Make the first call in each context before any stream capture.
 //
 // All calls share the array and leave their contents in it: each call clears
 // the status header it uses, and every other byte it reads is written earlier
 // in the same call.  Calls whose executions overlap on the GPU (different
 // streams, or different host threads on one device) race on the array.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+
 #include <mutex>
 
 #include "gc_internal.cuh"
@@ -31,25 +37,54 @@ __device__ __align__(256) unsigned char g_noalloc_scratch[GC_NOALLOC_SCRATCH_BYT
 
 constexpr int kMaxDevices = 64;
 std::mutex g_mu;
-void* g_addr[kMaxDevices] = {};
+struct Cached {
+  CUcontext ctx;  // context current when the address was looked up
+  void* addr;
+};
+Cached g_addr[kMaxDevices] = {};
+
+// The driver's cuCtxGetCurrent, through the runtime (no link to libcuda).
+PFN_cuCtxGetCurrent_v4000 ctx_current_fn() {
+  static PFN_cuCtxGetCurrent_v4000 fn = [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &p, 4000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      return reinterpret_cast<PFN_cuCtxGetCurrent_v4000>(p);
+    return static_cast<PFN_cuCtxGetCurrent_v4000>(nullptr);
+  }();
+  return fn;
+}
+
+CUcontext current_context() {
+  CUcontext c = nullptr;
+  auto fn = ctx_current_fn();
+  if (!fn || fn(&c) != CUDA_SUCCESS) return nullptr;
+  return c;
+}
 
 // Device address of the static scratch on the current device (set-up on the
-// first call per device).
+// first call per device and context).
 int scratch_address(void** out) {
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return cuda_check(e, "cudaGetDevice");
   if (dev < 0 || dev >= kMaxDevices)
     return fail(GC_ERR_UNSUPPORTED, "device ordinal %d beyond %d", dev, kMaxDevices);
+  CUcontext ctx = current_context();
   std::lock_guard<std::mutex> lock(g_mu);
-  if (!g_addr[dev]) {
+  Cached& c = g_addr[dev];
+  if (!c.addr || !ctx || c.ctx != ctx) {
     void* p = nullptr;
-    e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
+    e = cudaGetSymbolAddress(&p, g_noalloc_scratch);  // makes the device's context current
     if (e != cudaSuccess) return cuda_check(e, "cudaGetSymbolAddress(static scratch)");
     if (!p) return fail(GC_ERR_CUDA, "cudaGetSymbolAddress returned NULL");
-    g_addr[dev] = p;
+    if (!ctx) ctx = current_context();
+    c.ctx = ctx;
+    c.addr = p;
   }
-  *out = g_addr[dev];
+  *out = c.addr;
   return GC_OK;
 }
 
