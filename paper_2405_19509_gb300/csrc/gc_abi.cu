@@ -5,6 +5,8 @@
 #include <stdio.h>
 #include <string.h>
 
+#include <nvtx3/nvToolsExt.h>
+
 #include <algorithm>
 #include <atomic>
 #include <vector>
@@ -12,6 +14,9 @@
 #include "gc_internal.cuh"
 
 namespace gc {
+
+NvtxRange::NvtxRange(const char* name) { nvtxRangePushA(name); }
+NvtxRange::~NvtxRange() { nvtxRangePop(); }
 
 static thread_local char g_err[512] = "";
 
@@ -119,6 +124,7 @@ size_t gc_chunk_grads_batched_workspace(int N, int n_c, int d, int n_w) {
 
 int gc_chunk_grads_batched(const void* X, const float* y, const float* W, int N, int n_c, int d,
                            int n_w, int loss, float* G, void* ws, size_t ws_bytes, void* stream) {
+  NvtxRange nvtx_("gc_chunk_grads_batched");
   if (N < 1 || n_c < 1 || d < 1 || n_w < 1) return fail(GC_ERR_SHAPE, "N, n_c, d, n_w must be >= 1");
   if (n_w % 32 != 0 || n_w > 256)
     return fail(GC_ERR_UNSUPPORTED, "n_w=%d must be a multiple of 32 in [32, 256]", n_w);
@@ -146,6 +152,7 @@ size_t gc_trigger_workspace(int N) {
 int gc_trigger_times(const int32_t* order, int N, int m, int delta, const double* tau, int64_t nsim,
                      int ell, int theta, double* T, int32_t* psi, double* T_full, void* ws,
                      size_t ws_bytes, void* stream) {
+  NvtxRange nvtx_("gc_trigger_times");
   if (N < 1 || m < 1 || delta < 1 || nsim < 0) return fail(GC_ERR_SHAPE, "N, m, delta >= 1, nsim >= 0");
   if (ell < 1 || ell > GC_MAX_ELL) return fail(GC_ERR_UNSUPPORTED, "ell=%d outside [1, %d]", ell, GC_MAX_ELL);
   if (delta > GC_MAX_DELTA) return fail(GC_ERR_UNSUPPORTED, "delta=%d exceeds %d", delta, GC_MAX_DELTA);
@@ -255,6 +262,7 @@ size_t gc_chunk_grads_workspace(int N, int n_c, int d, int x_dtype) {
 int gc_chunk_grads(const void* X, int x_dtype, const float* y, const float* w, int N, int n_c,
                    int d, int loss, float* G, double* loss_out, void* ws, size_t ws_bytes,
                    void* stream) {
+  NvtxRange nvtx_("gc_chunk_grads");
   if (!X || !y || !w || !G) return fail(GC_ERR_ARG, "X, y, w and G must be non-NULL");
   if (x_dtype != GC_F32 && x_dtype != GC_BF16) return fail(GC_ERR_ARG, "x_dtype=%d", x_dtype);
   if (loss != GC_LSQ && loss != GC_LOGISTIC) return fail(GC_ERR_ARG, "loss=%d", loss);
@@ -279,6 +287,7 @@ int gc_find_encoding_coeff(const double* R, int ell, const int32_t* order, int N
                            const int32_t* psi, int npat, double* E, float* C, uint8_t* delta_out,
                            uint8_t* support, double* coef_err, double* est, void* ws,
                            size_t ws_bytes, void* stream) {
+  NvtxRange nvtx_("gc_find_encoding_coeff");
   int rc = check_dims(N, m, delta, ell, npat);
   if (rc) return rc;
   if (!R || !order || (!psi && npat > 0)) return fail(GC_ERR_ARG, "R, order and psi must be non-NULL");
@@ -306,6 +315,7 @@ size_t gc_encode_workspace(int N, int m, int delta, int ell, int npat, int d) {
 int gc_encode(const double* R, int ell, const int32_t* order, int N, int m, int delta,
               const int32_t* psi, int npat, const float* G, int d, float* T, void* ws,
               size_t ws_bytes, void* stream) {
+  NvtxRange nvtx_("gc_encode");
   int rc = check_dims(N, m, delta, ell, npat);
   if (rc) return rc;
   if (d < 1) return fail(GC_ERR_SHAPE, "d=%d must be >= 1", d);
@@ -329,6 +339,7 @@ int gc_encode(const double* R, int ell, const int32_t* order, int N, int m, int 
 int gc_encode_with_coeffs(const double* E, int ell, const int32_t* order, int N, int m, int delta,
                           const int32_t* psi, int npat, const float* G, int d, float* T,
                           void* stream) {
+  NvtxRange nvtx_("gc_encode_with_coeffs");
   int rc = check_dims(N, m, delta, ell, npat);
   if (rc) return rc;
   if (d < 1) return fail(GC_ERR_SHAPE, "d=%d must be >= 1", d);
@@ -340,6 +351,7 @@ int gc_encode_with_coeffs(const double* E, int ell, const int32_t* order, int N,
 
 int gc_decode_tx(const double* R, int ell, int m, const float* T, int npat, int d, float* ghat,
                  void* stream) {
+  NvtxRange nvtx_("gc_decode_tx");
   if (!R || !T || !ghat) return fail(GC_ERR_ARG, "R, T and ghat must be non-NULL");
   if (m < 1 || npat < 0 || d < 1) return fail(GC_ERR_SHAPE, "m, d >= 1 and npat >= 0 required");
   if (ell < 1) return fail(GC_ERR_SHAPE, "ell=%d must be >= 1", ell);
@@ -360,6 +372,7 @@ size_t gc_decode_plan_workspace(int N, int m, int delta, int ell, int npat) {
 int gc_decode_plan(const double* R, int ell, const int32_t* order, int N, int m, int delta,
                    const int32_t* psi, int npat, void* plan, size_t plan_bytes_, double* coef_err,
                    double* est, void* ws, size_t ws_bytes, void* stream) {
+  NvtxRange nvtx_("gc_decode_plan");
   int rc = check_dims(N, m, delta, ell, npat);
   if (rc) return rc;
   if (!R || !order || (!psi && npat > 0)) return fail(GC_ERR_ARG, "R, order and psi must be non-NULL");
@@ -395,6 +408,7 @@ size_t gc_decode_prepare_bytes(int N, int m, int delta, int ell) {
 
 int gc_decode_prepare(const double* R, int ell, const int32_t* order, int N, int m, int delta,
                       void* prep, size_t prep_bytes, void* stream) {
+  NvtxRange nvtx_("gc_decode_prepare");
   int rc = check_dims(N, m, delta, ell, 0);
   if (rc) return rc;
   if (!R || !order) return fail(GC_ERR_ARG, "R and order must be non-NULL");
@@ -422,6 +436,7 @@ int gc_decode_plan_prepared(const void* prep, const double* R, int ell, int N, i
                             const int32_t* psi, int npat, void* plan, size_t plan_bytes_,
                             double* coef_err, double* est, void* ws, size_t ws_bytes,
                             void* stream) {
+  NvtxRange nvtx_("gc_decode_plan_prepared");
   int rc = check_dims(N, m, delta, ell, npat);
   if (rc) return rc;
   if (!prep || !R || (!psi && npat > 0)) return fail(GC_ERR_ARG, "prep, R and psi must be non-NULL");
@@ -462,6 +477,7 @@ static int check_apply(int N, int ell, int npat, int d, const void* G, const flo
 
 int gc_decode_apply(const void* plan, int ell, int N, int npat, const float* G, int d, float* Ghat,
                     double* grad_mse, void* ws, size_t ws_bytes, void* stream) {
+  NvtxRange nvtx_("gc_decode_apply");
   int rc = check_apply(N, ell, npat, d, G, Ghat, grad_mse);
   if (rc) return rc;
   if (npat == 0) return GC_OK;
@@ -486,6 +502,7 @@ int gc_decode_batch(const double* R, int ell, const int32_t* order, int N, int m
                     const int32_t* psi, int npat, const float* G, int d, float* Ghat,
                     double* coef_err, double* est, double* grad_mse, void* ws, size_t ws_bytes,
                     void* stream) {
+  NvtxRange nvtx_("gc_decode_batch");
   int rc = check_dims(N, m, delta, ell, npat);
   if (rc) return rc;
   if (d < 1) return fail(GC_ERR_SHAPE, "d=%d must be >= 1", d);
@@ -517,6 +534,7 @@ size_t gc_decode_combine_workspace(int N, int ell, int npat, int d) {
 
 int gc_decode_combine(const float* C, int ell, int N, int npat, const float* G, int d,
                       float* Ghat, double* grad_mse, void* ws, size_t ws_bytes, void* stream) {
+  NvtxRange nvtx_("gc_decode_combine");
   int rc = check_apply(N, ell, npat, d, G, Ghat, grad_mse);
   if (rc) return rc;
   if (!C) return fail(GC_ERR_ARG, "C must be non-NULL");
@@ -538,12 +556,14 @@ size_t gc_mse_workspace(int N, int m, int delta, int ell, int npat, int d) {
 int gc_mse(const double* R, int ell, const int32_t* order, int N, int m, int delta,
            const int32_t* psi, int npat, const float* G, int d, double* coef_err, double* est,
            double* grad_mse, void* ws, size_t ws_bytes, void* stream) {
+  NvtxRange nvtx_("gc_mse");
   if (!grad_mse && npat > 0) return fail(GC_ERR_ARG, "grad_mse must be non-NULL");
   return gc_decode_batch(R, ell, order, N, m, delta, psi, npat, G, d, nullptr, coef_err, est,
                          grad_mse, ws, ws_bytes, stream);
 }
 
 int gc_sgd_step(float* w, const float* ghat, int d, float lr, int64_t Ntil, void* stream) {
+  NvtxRange nvtx_("gc_sgd_step");
   if (!w || !ghat) return fail(GC_ERR_ARG, "w and ghat must be non-NULL");
   if (d < 1 || Ntil < 1) return fail(GC_ERR_SHAPE, "d and Ntil must be >= 1");
   return launch_sgd(w, ghat, d, lr, Ntil, as_stream(stream));

@@ -23,6 +23,15 @@ struct WsHeader {
   uint32_t info;
 };
 
+// ---- NVTX range around a host entry point (a named range on the profiler's
+// timeline; no cost without a profiler attached) --------------------------
+struct NvtxRange {
+  explicit NvtxRange(const char* name);
+  ~NvtxRange();
+  NvtxRange(const NvtxRange&) = delete;
+  NvtxRange& operator=(const NvtxRange&) = delete;
+};
+
 // ---- error reporting (thread-local, host) --------------------------------
 int fail(int code, const char* fmt, ...);
 int cuda_check(cudaError_t e, const char* what);
