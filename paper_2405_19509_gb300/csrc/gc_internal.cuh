@@ -129,9 +129,8 @@ int launch_sgd(float* w, const float* ghat, int d, float lr, int64_t Ntil, cudaS
 // and, for a residual tile, the ordered list of its rows that need
 // corrections, each with a slot of squared-error partials.
 constexpr int kResidThreads = 256;
-constexpr int kResidW = 32;          // columns of one block per stripe (one per lane)
-constexpr int kResidRcap = 32;       // corrected rows a residual tile may hold
-constexpr int kResidMaxRows = 1280;  // N*ell staged per stripe (160 KB of shared memory)
+constexpr int kResidW = kResidThreads * 4;  // columns of one block per CTA (4 KB rows)
+constexpr int kResidRcap = 32;              // corrected rows a residual tile may hold
 struct ResidLists {
   int32_t* nnz;        // [npat] non-identity blocks (may exceed ksp)
   int32_t* idx;        // [npat][ksp] their chunks, ascending
@@ -143,17 +142,16 @@ struct ResidLists {
   int32_t* tcount;     // [ntiles] entries of rowlist
   float* msp;          // [ntiles*kResidRcap][parts] squared-error partials, or null
   int ksp;             // list capacity per pattern
-  int parts;           // partials per corrected row (column stripes)
+  int parts;           // partials per corrected row (column ranges x warps)
 };
 int resid_ksp(int ell);
-bool resid_fits(int N, int ell);
 size_t resid_ws_bytes(int N, int ell, int npat, int d);
 ResidLists carve_resid(Carve& c, int N, int ell, int npat, int d, bool want_mse);
 int launch_plan_scan(const __nv_bfloat16* Cs, int Kp, int N, int ell, int npat, int budget,
                      int policy, const ResidLists& rl, unsigned int* done_counter, cudaStream_t s);
 int launch_gsum(const float* G, int N, int d, float* gsum, cudaStream_t s);
-int launch_decode_resid(const float* G, const ResidLists& rl, int N, int ell, int npat, int d,
-                        float* gsum, float* Ghat, cudaStream_t s);
+int launch_decode_resid(const float* G, const float* gsum, const ResidLists& rl, int ell, int npat,
+                        int d, float* Ghat, cudaStream_t s);
 // Process-wide path policy of the batched decode (gc_set_decode_policy).
 int decode_policy();
 

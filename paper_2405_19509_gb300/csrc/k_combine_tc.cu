@@ -686,9 +686,7 @@ int launch_apply(const __nv_bfloat16* Cs, const float* G, int N, int ell, int np
   float* msep_mem = ws.take<float>((size_t)M * nnt * 2);
   float* msep = grad_mse ? msep_mem : nullptr;
   const ResidLists rl = carve_resid(ws, N, ell, npat, d, grad_mse != nullptr);
-  // batches too wide for a staged stripe of every chunk gradient go to the GEMM
-  const bool resid_ok = resid_fits(N, ell);
-  const int policy = resid_ok ? decode_policy() : GC_DECODE_DENSE;
+  const int policy = decode_policy();
   // a residual tile may spend up to Kp / 64 corrections per pattern: about
   // what the three MMAs per 64-wide K block cost against reading the ell
   // blocks of one chunk gradient
@@ -697,10 +695,13 @@ int launch_apply(const __nv_bfloat16* Cs, const float* G, int N, int ell, int np
   unsigned int* counter = reinterpret_cast<unsigned int*>(status) + 4;
   int rc = launch_plan_scan(Cs, Kp, N, ell, npat, budget, policy, rl, counter, s);
   if (rc) return rc;
-  // the residual kernel also forms s = sum_i g_{D_i} (the GEMM's MSE needs it)
-  rc = resid_ok ? launch_decode_resid(G, rl, N, ell, npat, d, gsum, Ghat, s)
-                : launch_gsum(G, N, d, gsum, s);
+  // s = sum_i g_{D_i}: the residual rows start from it, the GEMM's MSE uses it
+  rc = launch_gsum(G, N, d, gsum, s);
   if (rc) return rc;
+  if (policy != GC_DECODE_DENSE) {
+    rc = launch_decode_resid(G, gsum, rl, ell, npat, d, Ghat, s);
+    if (rc) return rc;
+  }
   {
     if (L >= 16384) {
       dim3 grid((L + 127) / 128, Kp / 32);

@@ -21,14 +21,16 @@
 //                   corrections (each gets a slot for its squared-error
 //                   partials) and the tile's path; the last CTA ORs the tile
 //                   flags into one "some tile is on the GEMM" word.
-//   k_decode_resid  one CTA per 32-column stripe of every block (and pattern
-//                   group): stages the stripe of all N*ell chunk-gradient
-//                   blocks in shared memory (G is read from HBM once in
-//                   all), forms s from it, writes s to the rows of exact
-//                   patterns and s + corrections to the listed rows, with
-//                   ||ghat_b - s||^2 = ||corrections||^2 per (row, stripe).
-//   k_gsum          s alone, for batches too wide for the stripe (N*ell >
-//                   kResidMaxRows), which go to the GEMM.
+//   k_gsum          s = sum_i g_{D_i} over all of d (one pass over G).
+//   k_decode_resid  one CTA per (residual tile, 1024-column range of each
+//                   block): every row of the tile gets one contiguous 4 KB
+//                   store -- s for exact patterns, s + corrections for the
+//                   listed rows, whose chunk gradients come through L2 (the
+//                   tiles of one column range run side by side, so each
+//                   range of g_{D_i} is read from HBM about once); the
+//                   squared error ||ghat_b - s||^2 = ||corrections||^2 is
+//                   left as one partial per (corrected row, range, warp).
+//                   CTAs of GEMM tiles return at once.
 #include <algorithm>
 
 #include "gc_internal.cuh"
@@ -37,18 +39,12 @@ namespace gc {
 
 int resid_ksp(int ell) { return ell <= 2 ? 32 : (ell <= 4 ? 16 : 8); }
 
-bool resid_fits(int N, int ell) { return (long long)N * ell <= kResidMaxRows; }
-
-static size_t resid_smem(int N, int ell) {
-  return ((size_t)N * ell + ell) * kResidW * sizeof(float);
-}
-
 size_t resid_ws_bytes(int N, int ell, int npat, int d) {
   const int L = (d + ell - 1) / ell;
   const long long M = (long long)npat * ell;
   const long long nmt = (M + 127) / 128;
   const int ksp = std::min(resid_ksp(ell), N);
-  const long long parts = (L + kResidW - 1) / kResidW;
+  const long long parts = (long long)((L + kResidW - 1) / kResidW) * (kResidThreads / 32);
   return align_up((size_t)npat * sizeof(int32_t), 256) +
          align_up((size_t)npat * ksp * sizeof(int32_t), 256) +
          align_up((size_t)npat * ksp * ell * ell * sizeof(float), 256) +
@@ -65,7 +61,7 @@ ResidLists carve_resid(Carve& c, int N, int ell, int npat, int d, bool want_mse)
   const long long nmt = (M + 127) / 128;
   ResidLists r{};
   r.ksp = std::min(resid_ksp(ell), N);
-  r.parts = (L + kResidW - 1) / kResidW;
+  r.parts = ((L + kResidW - 1) / kResidW) * (kResidThreads / 32);
   r.nnz = c.take<int32_t>(npat);
   r.idx = c.take<int32_t>((size_t)npat * r.ksp);
   r.D = c.take<float>((size_t)npat * r.ksp * ell * ell);
@@ -234,114 +230,94 @@ __global__ void __launch_bounds__(128) k_gsum(const float* __restrict__ G, int N
 }
 
 // ---------------------------------------------------------------------------
-// Residual decode.  Block (stripe, group): columns c0 .. c0+31 of every block
-// k (c0 = 32 * stripe; the same offsets in all ell blocks, so one staged row
-// of g_{D_i}[k'] serves every output block), patterns [b0, b1).
+// Residual decode.  Block (tile mt, range r): columns c = r*W + 4*t .. +3 of
+// every block k (the same offsets in all ell blocks, so one load of
+// g_{D_i}[k'] serves every output block) for the rows of tile mt.
 // ---------------------------------------------------------------------------
+__device__ __forceinline__ float4 ld4(const float* p, long long off, bool vec, int nvalid) {
+  if (vec && nvalid == 4) return __ldg(reinterpret_cast<const float4*>(p + off));
+  float v[4] = {0.f, 0.f, 0.f, 0.f};
+  for (int u = 0; u < nvalid; ++u) v[u] = __ldg(p + off + u);
+  return make_float4(v[0], v[1], v[2], v[3]);
+}
+__device__ __forceinline__ void st4(float* p, long long off, bool vec, int nvalid, float4 v) {
+  if (vec && nvalid == 4) {
+    __stcs(reinterpret_cast<float4*>(p + off), v);  // written once, never re-read here
+    return;
+  }
+  const float a[4] = {v.x, v.y, v.z, v.w};
+  for (int u = 0; u < nvalid; ++u) __stcs(p + off + u, a[u]);
+}
+
 template <int ELL>
-__global__ void __launch_bounds__(kResidThreads) k_decode_resid(const float* __restrict__ G,
-                                                                ResidLists rl, int N, int npat,
-                                                                int d, int L, int ppg, int vec,
-                                                                float* __restrict__ gsum,
+__global__ void __launch_bounds__(kResidThreads, 2) k_decode_resid(const float* __restrict__ G,
+                                                                const float* __restrict__ gsum,
+                                                                ResidLists rl, int npat, int d,
+                                                                int L, int vec,
                                                                 float* __restrict__ Ghat) {
-  extern __shared__ float sm[];
-  constexpr int W = kResidW;
-  constexpr int NW = kResidThreads / 32;
-  const int rows = N * ELL;
-  float* sg = sm;               // [rows][W]: row i*ELL + k' = g_{D_i}[k'*L + c0 ..]
-  float* ss = sm + rows * W;    // [ELL][W]: s
-  const int stripe = blockIdx.x;
-  const int c0 = stripe * W;
-  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  // ---- stage the stripe (zero past L and past d)
-  {
-    const int q = tid & 7;           // 16-byte quarter of a 128-byte row
-    const int c = c0 + 4 * q;
-    constexpr int RPP = kResidThreads / 8;
-    for (int r0 = 0; r0 < rows; r0 += RPP * 4) {
-      float4 v[4];
-#pragma unroll
-      for (int u = 0; u < 4; ++u) {
-        const int r = r0 + u * RPP + (tid >> 3);
-        v[u] = make_float4(0.f, 0.f, 0.f, 0.f);
-        if (r < rows) {
-          const int i = r / ELL, kp = r - i * ELL;
-          const long long col = (long long)kp * L + c;
-          const float* src = G + (size_t)i * d + col;
-          if (vec && c + 3 < L && col + 3 < d) {
-            v[u] = __ldg(reinterpret_cast<const float4*>(src));
-          } else {
-            float t[4] = {0.f, 0.f, 0.f, 0.f};
-            for (int e = 0; e < 4; ++e)
-              if (c + e < L && col + e < d) t[e] = __ldg(src + e);
-            v[u] = make_float4(t[0], t[1], t[2], t[3]);
-          }
-        }
-      }
-#pragma unroll
-      for (int u = 0; u < 4; ++u) {
-        const int r = r0 + u * RPP + (tid >> 3);
-        if (r < rows) *reinterpret_cast<float4*>(sg + r * W + 4 * q) = v[u];
-      }
-    }
-  }
-  __syncthreads();
-  // ---- s for the stripe, chunks added in order (the order k_gsum uses)
-  for (int t = tid; t < ELL * W; t += kResidThreads) {
-    const int k = t / W, c = t - k * W;
-    float acc = 0.f;
-    for (int i = 0; i < N; ++i) acc += sg[(i * ELL + k) * W + c];
-    ss[t] = acc;
-    const long long col = (long long)k * L + c0 + c;
-    if (gsum && blockIdx.y == 0 && c0 + c < L && col < d) gsum[col] = acc;
-  }
-  __syncthreads();
-  const int b0 = blockIdx.y * ppg;
-  const int b1 = min(npat, b0 + ppg);
-  bool ok[ELL];
-  float sr[ELL];
+  const int mt = blockIdx.x;
+  if (__ldg(rl.tflag + mt)) return;  // the GEMM writes this tile
+  const int r = blockIdx.y;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const long long M = (long long)npat * ELL;
+  const long long row0 = (long long)mt * 128;
+  const long long row_end = min(row0 + 128, M);
+  const int c = r * kResidW + threadIdx.x * 4;
+  const bool vecw = vec != 0;
+  // valid columns of this thread in block k (padding past L and past d), and s there
+  int nv[ELL];
+  float4 sv[ELL];
 #pragma unroll
   for (int k = 0; k < ELL; ++k) {
-    ok[k] = c0 + lane < L && (long long)k * L + c0 + lane < d;
-    sr[k] = ss[k * W + lane];
+    const long long col = (long long)k * L + c;
+    int n = min(4, L - c);
+    n = (int)min((long long)n, (long long)d - col);
+    nv[k] = n < 0 ? 0 : n;
+    sv[k] = nv[k] > 0 ? ld4(gsum, col, vecw, nv[k]) : make_float4(0.f, 0.f, 0.f, 0.f);
   }
-  // ---- exact patterns: ghat_b = s (zero error)
-  if (Ghat) {
-    for (int b = b0 + warp; b < b1; b += NW) {
-      if (__ldg(rl.nnz + b) != 0) continue;
-      float* o = Ghat + (size_t)b * d + c0 + lane;
+  const int b_lo = (int)(row0 / ELL), b_hi = (int)((row_end - 1) / ELL);
+  for (int b = b_lo; b <= b_hi; ++b) {
+    const size_t obase = (size_t)b * d;
+    const int nz = __ldg(rl.nnz + b);
 #pragma unroll
-      for (int k = 0; k < ELL; ++k) {
-        const long long row = (long long)b * ELL + k;
-        if (__ldg(rl.tflag + (row >> 7)) == 0 && ok[k]) __stcs(o + (size_t)k * L, sr[k]);
+    for (int k = 0; k < ELL; ++k) {
+      const long long row = (long long)b * ELL + k;
+      if (row < row0 || row >= row_end) continue;  // the neighbouring tile's row
+      if (nz == 0) {  // exact pattern: ghat_b = s, zero error
+        if (Ghat && nv[k] > 0) st4(Ghat, obase + (size_t)k * L + c, vecw, nv[k], sv[k]);
+        continue;
       }
-    }
-  }
-  // ---- rows with corrections, tile by tile from the scan's lists
-  const long long t_lo = ((long long)b0 * ELL) >> 7, t_hi = ((long long)b1 * ELL - 1) >> 7;
-  for (long long mt = t_lo; mt <= t_hi && b0 < b1; ++mt) {
-    if (__ldg(rl.tflag + mt)) continue;
-    const int cnt = __ldg(rl.tcount + mt);
-    for (int q = warp; q < cnt; q += NW) {
-      const int row = __ldg(rl.rowlist + mt * kResidRcap + q);
-      const int b = row / ELL, k = row - b * ELL;
-      if (b < b0 || b >= b1) continue;
-      const int nz = __ldg(rl.nnz + b);  // <= ksp: longer lists make the tile dense
-      float corr = 0.f;
+      // a corrected row (nz <= ksp: longer lists make the tile dense)
+      float4 cr = make_float4(0.f, 0.f, 0.f, 0.f);
       for (int e = 0; e < nz; ++e) {
         const int i = __ldg(rl.idx + (size_t)b * rl.ksp + e);
         const float* Dr = rl.D + ((size_t)b * rl.ksp + e) * ELL * ELL + k * ELL;
 #pragma unroll
-        for (int kp = 0; kp < ELL; ++kp) corr = fmaf(__ldg(Dr + kp), sg[(i * ELL + kp) * W + lane], corr);
+        for (int kp = 0; kp < ELL; ++kp) {
+          const float w = __ldg(Dr + kp);
+          if (nv[kp] == 0 || w == 0.f) continue;
+          const float4 g = ld4(G, (size_t)i * d + (size_t)kp * L + c, vecw, nv[kp]);
+          cr.x = fmaf(w, g.x, cr.x);
+          cr.y = fmaf(w, g.y, cr.y);
+          cr.z = fmaf(w, g.z, cr.z);
+          cr.w = fmaf(w, g.w, cr.w);
+        }
       }
-      // output column k*L + c0 + lane exists (padding past L and past d does not)
-      const bool col_ok = c0 + lane < L && (long long)k * L + c0 + lane < d;
-      if (Ghat && col_ok) __stcs(Ghat + (size_t)b * d + (size_t)k * L + c0 + lane, ss[k * W + lane] + corr);
+      // corrections only on the output columns that exist
+      float sq = nv[k] > 0 ? cr.x * cr.x : 0.f;
+      if (nv[k] > 1) sq = fmaf(cr.y, cr.y, sq);
+      if (nv[k] > 2) sq = fmaf(cr.z, cr.z, sq);
+      if (nv[k] > 3) sq = fmaf(cr.w, cr.w, sq);
+      if (Ghat && nv[k] > 0)
+        st4(Ghat, obase + (size_t)k * L + c, vecw, nv[k],
+            make_float4(sv[k].x + cr.x, sv[k].y + cr.y, sv[k].z + cr.z, sv[k].w + cr.w));
       if (rl.msp) {
-        float sq = col_ok ? corr * corr : 0.f;
 #pragma unroll
         for (int o = 16; o > 0; o >>= 1) sq += __shfl_xor_sync(0xffffffffu, sq, o);
-        if (lane == 0) rl.msp[((size_t)mt * kResidRcap + q) * rl.parts + stripe] = sq;
+        if (lane == 0) {
+          const int slot = __ldg(rl.rslot + row);
+          rl.msp[(size_t)slot * rl.parts + (size_t)r * (kResidThreads / 32) + warp] = sq;
+        }
       }
     }
   }
@@ -383,52 +359,33 @@ int launch_gsum(const float* G, int N, int d, float* gsum, cudaStream_t s) {
   return cuda_check(cudaGetLastError(), "k_gsum");
 }
 
-template <int ELL>
-static int launch_resid_t(dim3 grid, size_t smem, const float* G, const ResidLists& rl, int N,
-                          int npat, int d, int L, int ppg, int vec, float* gsum, float* Ghat,
-                          cudaStream_t s) {
-  static bool attr = false;
-  if (!attr) {
-    cudaError_t e = cudaFuncSetAttribute(k_decode_resid<ELL>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         (int)resid_smem(kResidMaxRows / ELL, ELL));
-    if (e != cudaSuccess) return cuda_check(e, "cudaFuncSetAttribute(k_decode_resid)");
-    attr = true;
-  }
-  k_decode_resid<ELL><<<grid, kResidThreads, smem, s>>>(G, rl, N, npat, d, L, ppg, vec, gsum, Ghat);
-  return GC_OK;
-}
-
-int launch_decode_resid(const float* G, const ResidLists& rl, int N, int ell, int npat, int d,
-                        float* gsum, float* Ghat, cudaStream_t s) {
+int launch_decode_resid(const float* G, const float* gsum, const ResidLists& rl, int ell, int npat,
+                        int d, float* Ghat, cudaStream_t s) {
   if (npat == 0) return GC_OK;
-  if (!resid_fits(N, ell)) return fail(GC_ERR_UNSUPPORTED, "residual decode: N*ell > %d", kResidMaxRows);
   const int L = (d + ell - 1) / ell;
-  const bool vec = d % 4 == 0 && L % 4 == 0 && reinterpret_cast<uintptr_t>(G) % 16 == 0;
-  const long long nstripes = (L + kResidW - 1) / kResidW;
-  const size_t smem = resid_smem(N, ell);
-  // enough blocks for a few per SM: the pattern groups split what the column
-  // stripes leave (each group stages its stripe again, from L2)
-  const int per_sm = std::max(1, std::min(8, (int)((200u << 10) / smem)));
-  const long long want = 2LL * per_sm * device_sm_count();
-  long long groups = std::max<long long>(1, (want + nstripes - 1) / nstripes);
-  groups = std::min<long long>(groups, std::min<long long>(npat, 65535));
-  const int ppg = (int)((npat + groups - 1) / groups);
-  groups = (npat + ppg - 1) / ppg;
-  if (nstripes > (1LL << 31) - 1) return fail(GC_ERR_UNSUPPORTED, "d too large");
-  dim3 grid((unsigned)nstripes, (unsigned)groups);
-  int rc;
+  const bool vec = d % 4 == 0 && L % 4 == 0 && reinterpret_cast<uintptr_t>(G) % 16 == 0 &&
+                   reinterpret_cast<uintptr_t>(gsum) % 16 == 0 &&
+                   (!Ghat || reinterpret_cast<uintptr_t>(Ghat) % 16 == 0);
+  const long long nmt = ((long long)npat * ell + 127) / 128;
+  const long long nranges = (L + kResidW - 1) / kResidW;
+  if (nmt > (1LL << 31) - 1 || nranges > 65535) return fail(GC_ERR_UNSUPPORTED, "residual decode grid too large");
+  // tiles fastest: the CTAs of one column range run side by side and share
+  // its chunk-gradient lines in L2
+  dim3 grid((unsigned)nmt, (unsigned)nranges);
+#define GC_RESID(E) \
+  case E: k_decode_resid<E><<<grid, kResidThreads, 0, s>>>(G, gsum, rl, npat, d, L, vec ? 1 : 0, Ghat); break;
   switch (ell) {
-    case 1: rc = launch_resid_t<1>(grid, smem, G, rl, N, npat, d, L, ppg, vec, gsum, Ghat, s); break;
-    case 2: rc = launch_resid_t<2>(grid, smem, G, rl, N, npat, d, L, ppg, vec, gsum, Ghat, s); break;
-    case 3: rc = launch_resid_t<3>(grid, smem, G, rl, N, npat, d, L, ppg, vec, gsum, Ghat, s); break;
-    case 4: rc = launch_resid_t<4>(grid, smem, G, rl, N, npat, d, L, ppg, vec, gsum, Ghat, s); break;
-    case 5: rc = launch_resid_t<5>(grid, smem, G, rl, N, npat, d, L, ppg, vec, gsum, Ghat, s); break;
-    case 6: rc = launch_resid_t<6>(grid, smem, G, rl, N, npat, d, L, ppg, vec, gsum, Ghat, s); break;
-    case 7: rc = launch_resid_t<7>(grid, smem, G, rl, N, npat, d, L, ppg, vec, gsum, Ghat, s); break;
-    case 8: rc = launch_resid_t<8>(grid, smem, G, rl, N, npat, d, L, ppg, vec, gsum, Ghat, s); break;
+    GC_RESID(1)
+    GC_RESID(2)
+    GC_RESID(3)
+    GC_RESID(4)
+    GC_RESID(5)
+    GC_RESID(6)
+    GC_RESID(7)
+    GC_RESID(8)
     default: return fail(GC_ERR_UNSUPPORTED, "ell=%d exceeds GC_MAX_ELL", ell);
   }
-  if (rc) return rc;
+#undef GC_RESID
   count_launches(1);
   return cuda_check(cudaGetLastError(), "k_decode_resid");
 }

@@ -25,11 +25,34 @@ namespace gc {
 // sweep position w in slot p (zero past its psi, for p >= delta and outside
 // the group), so every chunk step is DR/4 vector loads from shared memory and
 // DR*V FMAs with no branches; positions past the group's range add zeros.
+// Each thread keeps its next kEncStages - 1 chunk-stripe loads in flight:
+// cp.async copies its own columns of a coming (position, block) step into its
+// slots of a shared-memory ring (zero-filled past L and past d) and waits
+// with cp.async.wait_group, so no thread reads another's data and no barrier
+// or spin-wait is needed.
 // A transmission is summed over slots p ascending, blocks k ascending within
 // a slot -- the same order in the direct form, which a block whose workers'
 // orders are not cyclic (an explicit order) uses instead.
 constexpr int kEncThreads = 128;
 constexpr int kEncSmemFloats = 12288;  // staged coefficients (48 KB)
+constexpr int kEncStages = 8;          // ring of chunk-stripe steps per thread
+
+__device__ __forceinline__ uint32_t enc_smem_u32(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+// cp.async of `bytes` (4, 8 or 16) with zero fill past `valid` bytes
+template <int BYTES>
+__device__ __forceinline__ void cp_async_zfill(uint32_t dst, const float* src, int valid) {
+  if (BYTES == 16)
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src), "r"(valid) : "memory");
+  else if (BYTES == 8)
+    asm volatile("cp.async.ca.shared.global [%0], [%1], 8, %2;" ::"r"(dst), "l"(src), "r"(valid) : "memory");
+  else
+    asm volatile("cp.async.ca.shared.global [%0], [%1], 4, %2;" ::"r"(dst), "l"(src), "r"(valid) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory"); }
 
 __device__ __forceinline__ void enc_load(const float* __restrict__ gi, long long col, int c, int L,
                                          int d, bool vec, float* g, int V) {
@@ -69,6 +92,7 @@ __global__ void __launch_bounds__(kEncThreads)
              const int32_t* __restrict__ psi, int N, int m, int delta, int ell, int npat,
              const float* __restrict__ G, int d, int L, int J, int vec, float* __restrict__ T) {
   __shared__ __align__(16) float s_e[kEncSmemFloats];
+  __shared__ __align__(16) float s_ring[kEncStages * kEncThreads * V];
   __shared__ int s_np[256];               // processed counts of the group's workers (J <= 256)
   const int b = blockIdx.x;               // pattern fastest: blocks on one stripe share G in L2
   const int j0 = blockIdx.z * J, j1 = min(m, j0 + J);
@@ -123,6 +147,35 @@ __global__ void __launch_bounds__(kEncThreads)
   }
   __syncthreads();
   if (c >= L) return;  // no barrier below
+  // ring: this thread's V floats of each stage
+  const uint32_t ring = enc_smem_u32(s_ring) + threadIdx.x * (V * 4);
+  constexpr uint32_t kStage = kEncThreads * V * 4;
+  // the copy of step (iw, ik): columns c .. c+V-1 of block ik of the chunk at
+  // sweep position iw (positions past the group's range copy nothing)
+  int iw = 0, ik = 0, slot = 0;
+  auto issue = [&]() {
+    if (iw < W) {
+      const long long col = (long long)ik * L + c;
+      const float* src = G + (size_t)((j0 + iw) % N) * d + col;
+      int nv = min(V, L - c);
+      nv = (int)min((long long)nv, (long long)d - col);
+      const uint32_t dst = ring + slot * kStage;
+      if (vec) {
+        cp_async_zfill<V * 4>(dst, nv == V ? src : G, nv == V ? V * 4 : 0);
+      } else {
+#pragma unroll
+        for (int u = 0; u < V; ++u) cp_async_zfill<4>(dst + 4 * u, u < nv ? src + u : G, u < nv ? 4 : 0);
+      }
+    }
+    cp_async_commit();  // one group per step (possibly empty)
+    if (++ik == ell) {
+      ik = 0;
+      ++iw;
+    }
+    slot = (slot + 1) & (kEncStages - 1);
+  };
+  for (int q = 0; q < kEncStages - 1; ++q) issue();
+  int rs = 0;  // ring slot of the step being consumed
   float acc[DR][V];
 #pragma unroll
   for (int r = 0; r < DR; ++r)
@@ -135,11 +188,19 @@ __global__ void __launch_bounds__(kEncThreads)
     for (int u = 0; u < DR; ++u) {
       const int w = w0 + u;
       if (w >= W) break;
-      const int i = (j0 + w) % N;
-      const float* gi = G + (size_t)i * d;
       for (int k = 0; k < ell; ++k) {
+        issue();
+        cp_async_wait<kEncStages - 1>();  // this step's copy has landed
         float g[V];
-        enc_load(gi, (long long)k * L + c, c, L, d, vec != 0, g, V);
+        const float* gp = s_ring + (size_t)rs * kEncThreads * V + threadIdx.x * V;
+        if (V == 4) {
+          const float4 q = *reinterpret_cast<const float4*>(gp);
+          g[0] = q.x; g[V > 1 ? 1 : 0] = q.y; g[V > 2 ? 2 : 0] = q.z; g[V > 3 ? 3 : 0] = q.w;
+        } else {
+          const float2 q = *reinterpret_cast<const float2*>(gp);
+          g[0] = q.x; g[V > 1 ? 1 : 0] = q.y;
+        }
+        rs = (rs + 1) & (kEncStages - 1);
         const float4* e4 = reinterpret_cast<const float4*>(s_e + ((size_t)k * W + w) * DR);
 #pragma unroll
         for (int q = 0; q < DR / 4; ++q) {
@@ -163,6 +224,7 @@ __global__ void __launch_bounds__(kEncThreads)
       }
     }
   }
+  cp_async_wait<0>();  // no copy outlives the block
 }
 
 int launch_encode(const double* E, const int32_t* order, const int32_t* psi, int N, int m,
