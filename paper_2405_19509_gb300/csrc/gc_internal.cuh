@@ -136,7 +136,8 @@ struct ResidLists {
   int32_t* idx;        // [npat][ksp] their chunks, ascending
   float* D;            // [npat][ksp][ell][ell] Pi - I
   int32_t* tflag;      // [ntiles]
-  int32_t* any_dense;  // one word: some tile is on the GEMM
+  int32_t* dlist;      // [ntiles] the GEMM's tiles, ascending
+  int32_t* ndense;     // one word: entries of dlist
   int32_t* rslot;      // [npat*ell] slot of a corrected row of a residual tile, else -1
   int32_t* rowlist;    // [ntiles][kResidRcap] corrected rows of each tile, ascending
   int32_t* tcount;     // [ntiles] entries of rowlist

@@ -85,19 +85,13 @@ struct Params {
   int parts_per_row;    // num_n_tiles * (epilogue warps per TMEM lane quarter)
   long long spin_limit; // clock cycles a wait may take before the kernel gives up
   int stall;            // failure-path test: the TMA producer issues nothing
-  const int32_t* tflag; // per m-tile: nonzero = this kernel computes the tile's rows (null = all)
+  // The m-tiles this kernel computes (the others come from the residual
+  // decode): dlist[0 .. *ndense) in ascending order, written by the plan scan
+  // before the launch; null = every m-tile.
+  const int32_t* dlist;
+  const int32_t* ndense;
   uint32_t* status;
 };
-
-// The tiles a CTA computes: t, t + step, ... below t_last whose m-tile is
-// flagged for the GEMM (the other rows come from the residual decode).  Every
-// role walks the same sequence.
-__device__ __forceinline__ long long active_tile(const Params& p, long long t, long long t_last,
-                                                 long long step) {
-  if (p.tflag)
-    while (t < t_last && __ldg(p.tflag + (int)(t % p.num_m_tiles)) == 0) t += step;
-  return t;
-}
 
 using namespace tcw;
 
@@ -130,18 +124,6 @@ __global__ void __launch_bounds__(64 + 32 * EPI, 1)
   uint64_t* bempty = bfull + 1;       // BRES: MMAs on the B tile finished
   uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(bempty + 1);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_holder + 1);
-  // this CTA's tiles: t = t_first, t_first + t_step, ... < t_last
-  long long t_first, t_last, t_step;
-  if (BRES) {
-    t_first = (long long)blockIdx.x * p.num_tiles / gridDim.x;
-    t_last = (long long)(blockIdx.x + 1) * p.num_tiles / gridDim.x;
-    t_step = 1;
-  } else {
-    t_first = blockIdx.x;
-    t_last = p.num_tiles;
-    t_step = gridDim.x;
-  }
-
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
     for (int s = 0; s < STAGES; ++s) {
@@ -172,6 +154,24 @@ __global__ void __launch_bounds__(64 + 32 * EPI, 1)
   // launched as a programmatic dependent of the operand split: the prologue
   // above overlaps its tail, the operands are read only after this point
   asm volatile("griddepcontrol.wait;" ::: "memory");
+  // the tile space: nd listed m-tiles x the n-tiles, n-tile-major;
+  // this CTA's tiles are t = t_first, t_first + t_step, ... < t_last
+  const int nd = p.ndense ? *reinterpret_cast<volatile const int*>(p.ndense) : p.num_m_tiles;
+  const long long ntiles = (long long)nd * p.num_n_tiles;
+  long long t_first, t_last, t_step;
+  if (BRES) {
+    t_first = (long long)blockIdx.x * ntiles / gridDim.x;
+    t_last = (long long)(blockIdx.x + 1) * ntiles / gridDim.x;
+    t_step = 1;
+  } else {
+    t_first = blockIdx.x;
+    t_last = ntiles;
+    t_step = gridDim.x;
+  }
+  auto tile_mt = [&](long long t) -> int {
+    const int mi = (int)(t % nd);
+    return p.dlist ? __ldg(p.dlist + mi) : mi;
+  };
 
   if (warp == 0) {
     // ------------------------------------------------------------- producer
@@ -179,9 +179,8 @@ __global__ void __launch_bounds__(64 + 32 * EPI, 1)
       uint32_t it = 0, nb_loads = 0;
       int cur_nt = -1;
       bool ok = !p.stall;
-      for (long long t = active_tile(p, t_first, t_last, t_step); t < t_last && ok;
-           t = active_tile(p, t + t_step, t_last, t_step)) {
-        const int nt = (int)(t / p.num_m_tiles), mt = (int)(t % p.num_m_tiles);
+      for (long long t = t_first; t < t_last && ok; t += t_step) {
+        const int nt = (int)(t / nd), mt = tile_mt(t);
         if (nt != cur_nt) {
           // the MMAs on the previous B tile have finished before it is replaced
           if (nb_loads > 0 &&
@@ -213,9 +212,8 @@ __global__ void __launch_bounds__(64 + 32 * EPI, 1)
     } else if (lane == 0) {
       uint32_t it = 0;
       bool ok = !p.stall;
-      for (long long t = active_tile(p, t_first, t_last, t_step); t < t_last && ok;
-           t = active_tile(p, t + t_step, t_last, t_step)) {
-        const int nt = (int)(t / p.num_m_tiles), mt = (int)(t % p.num_m_tiles);
+      for (long long t = t_first; t < t_last && ok; t += t_step) {
+        const int nt = (int)(t / nd), mt = tile_mt(t);
         for (int kb = 0; kb < p.nkb; ++kb, ++it) {
           const int s = it % STAGES;
           const uint32_t ph = (it / STAGES) & 1;
@@ -241,9 +239,8 @@ __global__ void __launch_bounds__(64 + 32 * EPI, 1)
     if (lane == 0 && BRES) {
       uint32_t it = 0, tile_it = 0, nb_used = 0;
       int cur_nt = -1;
-      for (long long t = active_tile(p, t_first, t_last, t_step); t < t_last;
-           t = active_tile(p, t + t_step, t_last, t_step), ++tile_it) {
-        const int nt = (int)(t / p.num_m_tiles);
+      for (long long t = t_first; t < t_last; t += t_step, ++tile_it) {
+        const int nt = (int)(t / nd);
         if (nt != cur_nt) {
           if (!mbar_wait(bfull, nb_used & 1, abort_flag, p.status, p.spin_limit)) break;
           ++nb_used;
@@ -277,8 +274,7 @@ __global__ void __launch_bounds__(64 + 32 * EPI, 1)
         if (!ok) break;
         mma_commit(&tfull[ab]);
         // last tile on this B tile: hand it back once these MMAs complete
-        const long long tn = active_tile(p, t + t_step, t_last, t_step);
-        const bool last_on_b = tn >= t_last || (int)(tn / p.num_m_tiles) != nt;
+        const bool last_on_b = t + t_step >= t_last || (int)((t + t_step) / nd) != nt;
         if (last_on_b) mma_commit(bempty);
       }
       mma_commit(done);
@@ -287,8 +283,7 @@ __global__ void __launch_bounds__(64 + 32 * EPI, 1)
     } else if (lane == 0) {
       uint32_t it = 0, tile_it = 0;
       bool ok = true;
-      for (long long t = active_tile(p, t_first, t_last, t_step); t < t_last && ok;
-           t = active_tile(p, t + t_step, t_last, t_step), ++tile_it) {
+      for (long long t = t_first; t < t_last && ok; t += t_step, ++tile_it) {
         const int ab = tile_it & 1;
         if (!mbar_wait(&tempty[ab], ((tile_it >> 1) & 1) ^ 1, abort_flag, p.status, p.spin_limit))
           break;
@@ -333,10 +328,9 @@ __global__ void __launch_bounds__(64 + 32 * EPI, 1)
     const int cbeg = (e / 4) * SPAN;
     float* wbuf = outbuf + e * 2 * (OUT_BUF / 4);
     uint32_t tile_it = 0, chunk_it = 0;
-    for (long long t = active_tile(p, t_first, t_last, t_step); t < t_last;
-         t = active_tile(p, t + t_step, t_last, t_step), ++tile_it) {
+    for (long long t = t_first; t < t_last; t += t_step, ++tile_it) {
       const int ab = tile_it & 1;
-      const int nt = (int)(t / p.num_m_tiles), mt = (int)(t % p.num_m_tiles);
+      const int nt = (int)(t / nd), mt = tile_mt(t);
       // warp-uniform: the TMEM loads below are warp-collective
       const bool ready = mbar_wait(&tfull[ab], (tile_it >> 1) & 1, abort_flag, p.status, p.spin_limit);
       if (!__all_sync(0xffffffffu, ready)) break;
@@ -469,21 +463,26 @@ __global__ void k_split_c(const float* __restrict__ C, int M, int K, int Kp,
 // transposes the tile of 32 K-rows (kk = 32 y ..) by COLS columns
 // (c = COLS x ..) through shared memory: 16-byte loads along c, 16-byte
 // stores along kk (COLS = 128 for long rows, 32 when L is short and more
-// blocks are wanted).  Nothing is done when *any_dense is zero: no row tile
-// of the batch is on the GEMM.
+// blocks are wanted).  Blocks stride over the (column tile, K tile) pairs;
+// nothing is done when *ndense is zero: no row tile of the batch is on the
+// GEMM.
 template <int COLS>
 __global__ void __launch_bounds__(256) k_split_gt(const float* __restrict__ G, int N, int d,
                                                   int ell, int L, int Kp,
                                                   __nv_bfloat16* __restrict__ out,
-                                                  const int32_t* __restrict__ any_dense) {
+                                                  const int32_t* __restrict__ ndense) {
   constexpr int kSplitCols = COLS;
   constexpr int TPR = COLS / 4;            // threads per row of the load phase
   constexpr int RPP = 256 / TPR;           // rows per pass
   // the combine kernel may be scheduled now; it waits for this grid to finish
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
-  if (__ldg(any_dense) == 0) return;
+  if (ndense && __ldg(ndense) == 0) return;
   __shared__ float tile[32][kSplitCols + 1];
-  const int c0 = blockIdx.x * kSplitCols, k0 = blockIdx.y * 32;
+  const int ncx = (L + kSplitCols - 1) / kSplitCols;
+  const long long npair = (long long)ncx * (Kp / 32);
+  for (long long pr = blockIdx.x; pr < npair; pr += gridDim.x) {
+  __syncthreads();  // the previous pair's tile has been read
+  const int c0 = (int)(pr % ncx) * kSplitCols, k0 = (int)(pr / ncx) * 32;
   const int t = threadIdx.x;
   const int K = N * ell;
   const bool vec = (L % 4 == 0) && (d % 4 == 0) && (reinterpret_cast<uintptr_t>(G) % 16 == 0);
@@ -534,6 +533,7 @@ __global__ void __launch_bounds__(256) k_split_gt(const float* __restrict__ G, i
         dl[1] = make_uint4(lw[4], lw[5], lw[6], lw[7]);
       }
     }
+  }
   }
 }
 
@@ -703,13 +703,15 @@ int launch_apply(const __nv_bfloat16* Cs, const float* G, int N, int ell, int np
     if (rc) return rc;
   }
   {
-    if (L >= 16384) {
-      dim3 grid((L + 127) / 128, Kp / 32);
-      k_split_gt<128><<<grid, 256, 0, s>>>(G, N, d, ell, L, Kp, Gs, rl.any_dense);
-    } else {
-      dim3 grid((L + 31) / 32, Kp / 32);
-      k_split_gt<32><<<grid, 256, 0, s>>>(G, N, d, ell, L, Kp, Gs, rl.any_dense);
-    }
+    // a grid of a few blocks per SM striding over the tiles: it costs little
+    // to launch when no row tile is on the GEMM
+    const int cols = L >= 16384 ? 128 : 32;
+    const long long pairs = (long long)((L + cols - 1) / cols) * (Kp / 32);
+    const unsigned blocks = (unsigned)std::min<long long>(pairs, 8LL * device_sm_count());
+    if (cols == 128)
+      k_split_gt<128><<<blocks, 256, 0, s>>>(G, N, d, ell, L, Kp, Gs, rl.ndense);
+    else
+      k_split_gt<32><<<blocks, 256, 0, s>>>(G, N, d, ell, L, Kp, Gs, rl.ndense);
     count_launches(1);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return cuda_check(e, "k_split_gt");
@@ -745,7 +747,8 @@ int launch_apply(const __nv_bfloat16* Cs, const float* G, int N, int ell, int np
   p.Ghat = Ghat;
   p.gsum = grad_mse ? gsum : nullptr;
   p.msep = msep;
-  p.tflag = rl.tflag;
+  p.dlist = rl.dlist;
+  p.ndense = rl.ndense;
   p.status = status;
   p.spin_limit = wait_limit(kSpin);
   p.stall = take_stall(GC_STALL_COMBINE) ? 1 : 0;

@@ -19,8 +19,9 @@
 //                   ordered list of non-identity blocks (chunk, D) and its
 //                   length; per tile the ordered list of its rows that need
 //                   corrections (each gets a slot for its squared-error
-//                   partials) and the tile's path; the last CTA ORs the tile
-//                   flags into one "some tile is on the GEMM" word.
+//                   partials) and the tile's path; the last CTA lists the
+//                   GEMM's tiles in order (the GEMM and its operand split
+//                   walk only those).
 //   k_gsum          s = sum_i g_{D_i} over all of d (one pass over G).
 //   k_decode_resid  one CTA per (residual tile, 1024-column range of each
 //                   block): every row of the tile gets one contiguous 4 KB
@@ -48,8 +49,8 @@ size_t resid_ws_bytes(int N, int ell, int npat, int d) {
   return align_up((size_t)npat * sizeof(int32_t), 256) +
          align_up((size_t)npat * ksp * sizeof(int32_t), 256) +
          align_up((size_t)npat * ksp * ell * ell * sizeof(float), 256) +
-         align_up((size_t)nmt * sizeof(int32_t), 256) + align_up(sizeof(int32_t), 256) +
-         align_up((size_t)M * sizeof(int32_t), 256) +
+         align_up((size_t)nmt * sizeof(int32_t), 256) + align_up((size_t)nmt * sizeof(int32_t), 256) +
+         align_up(sizeof(int32_t), 256) + align_up((size_t)M * sizeof(int32_t), 256) +
          align_up((size_t)nmt * kResidRcap * sizeof(int32_t), 256) +
          align_up((size_t)nmt * sizeof(int32_t), 256) +
          align_up((size_t)nmt * kResidRcap * parts * sizeof(float), 256);
@@ -66,7 +67,8 @@ ResidLists carve_resid(Carve& c, int N, int ell, int npat, int d, bool want_mse)
   r.idx = c.take<int32_t>((size_t)npat * r.ksp);
   r.D = c.take<float>((size_t)npat * r.ksp * ell * ell);
   r.tflag = c.take<int32_t>(nmt);
-  r.any_dense = c.take<int32_t>(1);
+  r.dlist = c.take<int32_t>(nmt);
+  r.ndense = c.take<int32_t>(1);
   r.rslot = c.take<int32_t>(M);
   r.rowlist = c.take<int32_t>((size_t)nmt * kResidRcap);
   r.tcount = c.take<int32_t>(nmt);
@@ -79,9 +81,11 @@ ResidLists carve_resid(Carve& c, int N, int ell, int npat, int d, bool want_mse)
 // Plan scan: non-identity blocks per pattern, corrected rows and path per tile.
 // ---------------------------------------------------------------------------
 constexpr int kScanMaxPat = 130;  // patterns overlapping one 128-row tile
+constexpr int kScanThreads = 512;  // one warp per pattern at a time
+constexpr int kScanWarps = kScanThreads / 32;
 
 template <int ELL>
-__global__ void __launch_bounds__(128) k_plan_scan(const __nv_bfloat16* __restrict__ Cs, int Kp,
+__global__ void __launch_bounds__(kScanThreads) k_plan_scan(const __nv_bfloat16* __restrict__ Cs, int Kp,
                                                    int N, int npat, int budget, int policy,
                                                    ResidLists rl, unsigned int* done_counter) {
   const int mt = blockIdx.x;
@@ -92,10 +96,10 @@ __global__ void __launch_bounds__(128) k_plan_scan(const __nv_bfloat16* __restri
   const size_t plane = (size_t)M * Kp;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   __shared__ int s_cnt[kScanMaxPat];
-  __shared__ int s_or[4], s_sum[4], s_rows[4];
+  __shared__ int s_or[kScanWarps], s_sum[kScanWarps], s_rows[kScanWarps];
   __shared__ int s_last;
   int w_over = 0, w_sum = 0;
-  for (int b = b_lo + warp; b <= b_hi; b += 4) {
+  for (int b = b_lo + warp; b <= b_hi; b += kScanWarps) {
     // the tile holding the pattern's first row writes its list
     const bool owner = (long long)b * ELL >= row0;
     int count = 0;
@@ -138,15 +142,17 @@ __global__ void __launch_bounds__(128) k_plan_scan(const __nv_bfloat16* __restri
   }
   __syncthreads();
   // rows of this tile that need corrections, in row order: slot mt*RCAP + rank
+  // (thread t < 128 takes row row0 + t)
   const long long row = row0 + threadIdx.x;
-  const bool valid = row < M;
+  const bool valid = threadIdx.x < 128 && row < M;
   const bool ne = valid && s_cnt[(int)(row / ELL) - b_lo] > 0;
   const unsigned bal = __ballot_sync(0xffffffffu, ne);
   if (lane == 0) s_rows[warp] = __popc(bal);
   __syncthreads();
   int rank = __popc(bal & ((1u << lane) - 1u));
   for (int w = 0; w < warp; ++w) rank += s_rows[w];
-  const int nrows = s_rows[0] + s_rows[1] + s_rows[2] + s_rows[3];
+  int nrows = 0;
+  for (int w = 0; w < kScanWarps; ++w) nrows += s_rows[w];
   if (valid) {
     const bool slotted = ne && rank < kResidRcap;
     rl.rslot[row] = slotted ? mt * kResidRcap + rank : -1;
@@ -155,7 +161,7 @@ __global__ void __launch_bounds__(128) k_plan_scan(const __nv_bfloat16* __restri
   if (threadIdx.x == 0) {
     int over = 0;
     long long sum = 0;
-    for (int w = 0; w < 4; ++w) {
+    for (int w = 0; w < kScanWarps; ++w) {
       over |= s_or[w];
       sum += s_sum[w];
     }
@@ -176,14 +182,24 @@ __global__ void __launch_bounds__(128) k_plan_scan(const __nv_bfloat16* __restri
     const unsigned prev = atomicInc(done_counter, gridDim.x - 1);
     s_last = prev == gridDim.x - 1;
   }
-  __syncthreads();
+  __syncthreads();  // also: every read of s_rows above is done
   if (s_last) {
+    // every tile's flag is written: list the GEMM's tiles in ascending order
     __threadfence();
-    int any = 0;
-    for (int t = threadIdx.x; t < (int)gridDim.x; t += blockDim.x)
-      any |= *reinterpret_cast<volatile int*>(rl.tflag + t);
-    any = __syncthreads_or(any);
-    if (threadIdx.x == 0) *rl.any_dense = any;
+    int base = 0;
+    for (int t0 = 0; t0 < (int)gridDim.x; t0 += kScanThreads) {
+      const int t = t0 + threadIdx.x;
+      const bool f = t < (int)gridDim.x && *reinterpret_cast<volatile int*>(rl.tflag + t) != 0;
+      const unsigned bf = __ballot_sync(0xffffffffu, f);
+      if (lane == 0) s_rows[warp] = __popc(bf);
+      __syncthreads();
+      int pos = base + __popc(bf & ((1u << lane) - 1u));
+      for (int w = 0; w < warp; ++w) pos += s_rows[w];
+      if (f) rl.dlist[pos] = t;
+      for (int w = 0; w < kScanWarps; ++w) base += s_rows[w];
+      __syncthreads();
+    }
+    if (threadIdx.x == 0) *rl.ndense = base;
   }
 }
 
@@ -333,7 +349,7 @@ int launch_plan_scan(const __nv_bfloat16* Cs, int Kp, int N, int ell, int npat, 
   if (nmt == 0) return GC_OK;
   if (nmt > (1LL << 31) - 1) return fail(GC_ERR_UNSUPPORTED, "too many row tiles");
 #define GC_SCAN(E) \
-  case E: k_plan_scan<E><<<(unsigned)nmt, 128, 0, s>>>(Cs, Kp, N, npat, budget, policy, rl, done_counter); break;
+  case E: k_plan_scan<E><<<(unsigned)nmt, kScanThreads, 0, s>>>(Cs, Kp, N, npat, budget, policy, rl, done_counter); break;
   switch (ell) {
     GC_SCAN(1)
     GC_SCAN(2)
