@@ -266,7 +266,7 @@ __device__ __forceinline__ void st4(float* p, long long off, bool vec, int nvali
 }
 
 template <int ELL>
-__global__ void __launch_bounds__(kResidThreads, 2) k_decode_resid(const float* __restrict__ G,
+__global__ void __launch_bounds__(kResidThreads, ELL <= 4 ? 4 : 2) k_decode_resid(const float* __restrict__ G,
                                                                 const float* __restrict__ gsum,
                                                                 ResidLists rl, int npat, int d,
                                                                 int L, int vec,

@@ -86,18 +86,29 @@ __host__ __device__ inline int enc_group_max(int DR, int ell) {
   return j < 1 ? 1 : (j > 256 ? 256 : j);
 }
 
+// Shared memory of a block: the staged coefficients (diagonal layout, or the
+// direct layout of a non-cyclic group) and the ring.
+inline size_t enc_smem_bytes(int DR, int V, int ell, int delta, int J) {
+  const size_t diag = (size_t)ell * (J + DR - 1) * DR;
+  const size_t direct = (size_t)J * delta * ell;
+  return (std::max(diag, direct) + (size_t)kEncStages * kEncThreads * V) * sizeof(float);
+}
+
+// Four blocks per SM (three with a 32-slot ring): about 120 registers a thread.
 template <int DR, int V>
-__global__ void __launch_bounds__(kEncThreads)
+__global__ void __launch_bounds__(kEncThreads, DR == 32 ? 3 : 4)
     k_encode(const double* __restrict__ E, const int32_t* __restrict__ order,
              const int32_t* __restrict__ psi, int N, int m, int delta, int ell, int npat,
              const float* __restrict__ G, int d, int L, int J, int vec, float* __restrict__ T) {
-  __shared__ __align__(16) float s_e[kEncSmemFloats];
-  __shared__ __align__(16) float s_ring[kEncStages * kEncThreads * V];
+  extern __shared__ __align__(16) float s_dyn[];
   __shared__ int s_np[256];               // processed counts of the group's workers (J <= 256)
   const int b = blockIdx.x;               // pattern fastest: blocks on one stripe share G in L2
   const int j0 = blockIdx.z * J, j1 = min(m, j0 + J);
   const int nj = j1 - j0;
   const int de = delta * ell;
+  const int W = nj + DR - 1;              // sweep positions of the cyclic form
+  float* s_e = s_dyn;
+  float* s_ring = s_dyn + ((ell * W * DR > nj * de ? ell * W * DR : nj * de) + 3) / 4 * 4;
   const int c = (blockIdx.y * kEncThreads + threadIdx.x) * V;
   for (int t = threadIdx.x; t < nj; t += kEncThreads) {
     int np = psi[(size_t)b * m + j0 + t];
@@ -136,8 +147,7 @@ __global__ void __launch_bounds__(kEncThreads)
     }
     return;
   }
-  // diagonal staging: s_e[(k * W + w) * DR + p], w = 0 .. nj + DR - 2 sweep positions
-  const int W = nj + DR - 1;
+  // diagonal staging: s_e[(k * W + w) * DR + p]
   for (int t = threadIdx.x; t < ell * W * DR; t += kEncThreads) {
     const int p = t % DR, w = (t / DR) % W, k = t / (DR * W);
     const int jj = w - p;
@@ -150,71 +160,85 @@ __global__ void __launch_bounds__(kEncThreads)
   // ring: this thread's V floats of each stage
   const uint32_t ring = enc_smem_u32(s_ring) + threadIdx.x * (V * 4);
   constexpr uint32_t kStage = kEncThreads * V * 4;
-  // the copy of step (iw, ik): columns c .. c+V-1 of block ik of the chunk at
-  // sweep position iw (positions past the group's range copy nothing)
+  // every step copies V whole floats (vector rows, no padding in this thread's columns)
+  const bool full = vec && c + V <= L && (long long)ell * L <= d;
+  // issue cursor: step (iw, ik) = block ik of the chunk at sweep position iw
   int iw = 0, ik = 0, slot = 0;
+  int ich = j0 % N;
+  const float* gsrc = G + (size_t)ich * d + c;  // + ik * L
   auto issue = [&]() {
     if (iw < W) {
-      const long long col = (long long)ik * L + c;
-      const float* src = G + (size_t)((j0 + iw) % N) * d + col;
-      int nv = min(V, L - c);
-      nv = (int)min((long long)nv, (long long)d - col);
       const uint32_t dst = ring + slot * kStage;
-      if (vec) {
-        cp_async_zfill<V * 4>(dst, nv == V ? src : G, nv == V ? V * 4 : 0);
+      const float* src = gsrc + (size_t)ik * L;
+      if (full) {
+        cp_async_zfill<V * 4>(dst, src, V * 4);
       } else {
+        const long long col = (long long)ik * L + c;
+        int nv = min(V, L - c);
+        nv = (int)min((long long)nv, (long long)d - col);
+        if (vec) {
+          cp_async_zfill<V * 4>(dst, nv == V ? src : G, nv == V ? V * 4 : 0);
+        } else {
 #pragma unroll
-        for (int u = 0; u < V; ++u) cp_async_zfill<4>(dst + 4 * u, u < nv ? src + u : G, u < nv ? 4 : 0);
+          for (int u = 0; u < V; ++u) cp_async_zfill<4>(dst + 4 * u, u < nv ? src + u : G, u < nv ? 4 : 0);
+        }
       }
     }
     cp_async_commit();  // one group per step (possibly empty)
     if (++ik == ell) {
       ik = 0;
       ++iw;
+      if (++ich == N) ich = 0;
+      gsrc = G + (size_t)ich * d + c;
     }
     slot = (slot + 1) & (kEncStages - 1);
   };
   for (int q = 0; q < kEncStages - 1; ++q) issue();
+  const float* rd = s_ring + threadIdx.x * V;  // this thread's slot 0
   int rs = 0;  // ring slot of the step being consumed
   float acc[DR][V];
 #pragma unroll
   for (int r = 0; r < DR; ++r)
 #pragma unroll
     for (int v = 0; v < V; ++v) acc[r][v] = 0.f;
-  // sweep position w = vv - j0 holds chunk vv mod N; worker j0 + w - p takes it
+  // sweep position w holds chunk (j0 + w) mod N; worker j0 + w - p takes it
   // in slot p, ring slot (w - p) mod DR; worker j0 + w - DR + 1 is complete after it
+  const float* ecol = s_e;  // coefficients of (k = 0, w)
   for (int w0 = 0; w0 < W; w0 += DR) {
 #pragma unroll
     for (int u = 0; u < DR; ++u) {
       const int w = w0 + u;
       if (w >= W) break;
-      for (int k = 0; k < ell; ++k) {
-        issue();
-        cp_async_wait<kEncStages - 1>();  // this step's copy has landed
-        float g[V];
-        const float* gp = s_ring + (size_t)rs * kEncThreads * V + threadIdx.x * V;
-        if (V == 4) {
-          const float4 q = *reinterpret_cast<const float4*>(gp);
-          g[0] = q.x; g[V > 1 ? 1 : 0] = q.y; g[V > 2 ? 2 : 0] = q.z; g[V > 3 ? 3 : 0] = q.w;
-        } else {
-          const float2 q = *reinterpret_cast<const float2*>(gp);
-          g[0] = q.x; g[V > 1 ? 1 : 0] = q.y;
-        }
-        rs = (rs + 1) & (kEncStages - 1);
-        const float4* e4 = reinterpret_cast<const float4*>(s_e + ((size_t)k * W + w) * DR);
+      for (int kk = 0; kk < ell; ++kk) {
+        {
+          issue();
+          cp_async_wait<kEncStages - 1>();  // this step's copy has landed
+          float g[V];
+          const float* gp = rd + rs * (kEncThreads * V);
+          if (V == 4) {
+            const float4 q = *reinterpret_cast<const float4*>(gp);
+            g[0] = q.x; g[V > 1 ? 1 : 0] = q.y; g[V > 2 ? 2 : 0] = q.z; g[V > 3 ? 3 : 0] = q.w;
+          } else {
+            const float2 q = *reinterpret_cast<const float2*>(gp);
+            g[0] = q.x; g[V > 1 ? 1 : 0] = q.y;
+          }
+          rs = (rs + 1) & (kEncStages - 1);
+          const float4* e4 = reinterpret_cast<const float4*>(ecol + (size_t)kk * W * DR);
 #pragma unroll
-        for (int q = 0; q < DR / 4; ++q) {
-          const float4 e = e4[q];
-          const float ev[4] = {e.x, e.y, e.z, e.w};
+          for (int q = 0; q < DR / 4; ++q) {
+            const float4 e = e4[q];
+            const float ev[4] = {e.x, e.y, e.z, e.w};
 #pragma unroll
-          for (int h = 0; h < 4; ++h) {
-            const int p = 4 * q + h;
+            for (int h = 0; h < 4; ++h) {
+              const int p = 4 * q + h;
 #pragma unroll
-            for (int v = 0; v < V; ++v)
-              acc[(u - p) & (DR - 1)][v] = fmaf(ev[h], g[v], acc[(u - p) & (DR - 1)][v]);
+              for (int v = 0; v < V; ++v)
+                acc[(u - p) & (DR - 1)][v] = fmaf(ev[h], g[v], acc[(u - p) & (DR - 1)][v]);
+            }
           }
         }
       }
+      ecol += DR;
       const int jj = w - DR + 1;
       if (jj >= 0) {  // jj < nj since w < nj + DR - 1
         float* a = acc[(u + 1) & (DR - 1)];
@@ -225,6 +249,21 @@ __global__ void __launch_bounds__(kEncThreads)
     }
   }
   cp_async_wait<0>();  // no copy outlives the block
+}
+
+template <int DR, int V>
+static int launch_enc_t(dim3 grid, size_t smem, const double* E, const int32_t* order,
+                        const int32_t* psi, int N, int m, int delta, int ell, int npat,
+                        const float* G, int d, int L, int J, int vec, float* T, cudaStream_t s) {
+  static bool attr = false;
+  if (!attr) {
+    cudaError_t e = cudaFuncSetAttribute(k_encode<DR, V>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)((kEncSmemFloats + kEncStages * kEncThreads * V) * sizeof(float)));
+    if (e != cudaSuccess) return cuda_check(e, "cudaFuncSetAttribute(k_encode)");
+    attr = true;
+  }
+  k_encode<DR, V><<<grid, kEncThreads, smem, s>>>(E, order, psi, N, m, delta, ell, npat, G, d, L, J, vec, T);
+  return GC_OK;
 }
 
 int launch_encode(const double* E, const int32_t* order, const int32_t* psi, int N, int m,
@@ -249,9 +288,11 @@ int launch_encode(const double* E, const int32_t* order, const int32_t* psi, int
   const int ngroups = (m + J - 1) / J;
   if (npat > 2147483647 || stripes > 65535 || ngroups > 65535)
     return fail(GC_ERR_UNSUPPORTED, "encode grid too large");
+  const size_t smem = enc_smem_bytes(DR, V, ell, delta, J);
+  const dim3 grid((unsigned)npat, (unsigned)stripes, (unsigned)ngroups);
+  int rc;
 #define GC_ENC(R, VV) \
-  k_encode<R, VV><<<dim3((unsigned)npat, (unsigned)stripes, (unsigned)ngroups), kEncThreads, 0, s>>>( \
-      E, order, psi, N, m, delta, ell, npat, G, d, L, J, vec ? 1 : 0, T)
+  rc = launch_enc_t<R, VV>(grid, smem, E, order, psi, N, m, delta, ell, npat, G, d, L, J, vec, T, s)
   switch (DR) {
     case 4: GC_ENC(4, 4); break;
     case 8: GC_ENC(8, 4); break;
@@ -259,6 +300,7 @@ int launch_encode(const double* E, const int32_t* order, const int32_t* psi, int
     default: GC_ENC(32, 2); break;
   }
 #undef GC_ENC
+  if (rc) return rc;
   count_launches(1);
   return cuda_check(cudaGetLastError(), "k_encode");
 }
