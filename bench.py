@@ -1052,6 +1052,7 @@ def extra_workload(args):
             "value": rows[1]["GB/s"], "unit": "GB/s", "per_patterns": rows,
             "roofline": {"kernel": "k_encode", "bound": "hbm", "unit": "GB/s",
                          "achieved": rows[1]["GB/s"], "peak": hbm, "frac": rows[1]["frac_of_hbm"],
+                         "traffic": _traffic("k_encode", ["k_encode.cu"]),
                          "note": "algorithmic bytes per pattern: G read once (N d 4) + T written "
                                  "(m L 4); GB/s_G_once counts G once for the whole call",
                          "peak_source": f"{pk_src} hbm_gbs"},
