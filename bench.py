@@ -257,6 +257,36 @@ def _traffic(kernel, src_files):
     return e.get("dram_bytes_per_launch")
 
 
+def gemm_tile_fraction(psi, order, N, ell, ksp=None, rcap=32):
+    """Share of the decode's 128-row tiles that the library computes on the
+    tensor-core GEMM under its automatic policy (reporting only; the device
+    makes the same choice from the decode plan): a tile stays on the residual
+    path unless one of its patterns has more than ksp blocks with fewer than
+    ell copies, more than rcap of its rows need corrections, or its patterns
+    average more than ceil(N*ell/64) such blocks."""
+    m, delta = order.shape
+    D = np.zeros((psi.shape[0], N), dtype=np.int64)
+    for j in range(m):
+        for p in range(delta):
+            i = order[j, p]
+            if i >= 0:
+                D[:, i] += psi[:, j] > p
+    nnz = (D < ell).sum(axis=1)
+    ksp = ksp or min(N, 32 if ell <= 2 else (16 if ell <= 4 else 8))
+    budget = max(1, -(-N * ell // 64))
+    M = psi.shape[0] * ell
+    row_pat = np.arange(M) // ell
+    dense = 0
+    ntile = (M + 127) // 128
+    for t in range(ntile):
+        rows = np.arange(t * 128, min(M, t * 128 + 128))
+        pats = np.unique(row_pat[rows])
+        corrected = int((nnz[row_pat[rows]] > 0).sum())
+        if np.any(nnz[pats] > ksp) or corrected > rcap or nnz[pats].sum() > budget * len(pats):
+            dense += 1
+    return dense / ntile
+
+
 def oracle_decode_sample(cfg, ell, G32, psi, cols, min_patterns, max_seconds):
     """Time the fp64 oracle on a bounded sample of the decode workload.
 
@@ -672,8 +702,11 @@ def logistic_arm(args, rank, world, local_rank):
     ce_b = [torch.empty(npat, dtype=torch.float64, device=dev) for _ in range(2)]
     est_b = [torch.empty(npat, dtype=torch.float64, device=dev) for _ in range(2)]
     mse_b = [torch.empty(npat, dtype=torch.float64, device=dev) for _ in range(2)]
-    G_s = torch.empty(N, d, dtype=torch.float32, device=dev)
-    plan_s = torch.empty(int(gc.lib.gc_decode_plan_bytes(N, ell, npat)), dtype=torch.uint8, device=dev)
+    # the chunk gradients and the decode plan are double-buffered too: the
+    # batched decode of step t reads them while step t + 1 computes its own
+    G_b = [torch.empty(N, d, dtype=torch.float32, device=dev) for _ in range(2)]
+    plan_b = [torch.empty(int(gc.lib.gc_decode_plan_bytes(N, ell, npat)), dtype=torch.uint8, device=dev)
+              for _ in range(2)]
     Gh_s = torch.empty(npat, d, dtype=torch.float32, device=dev)
     T_s = torch.empty(1, m, L, dtype=torch.float32, device=dev)
     E_s = torch.empty(1, m, delta, ell, dtype=torch.float64, device=dev)
@@ -683,25 +716,26 @@ def logistic_arm(args, rank, world, local_rank):
     bi = [0]  # buffer the stage functions use (set before each capture / eager call)
 
     def stage_a():
-        gc.gc_chunk_grads(X, y, w, N, n_c, gc.GC_LOGISTIC, G=G_s, loss_out=loss_b[bi[0]], ws=wsA)
+        gc.gc_chunk_grads(X, y, w, N, n_c, gc.GC_LOGISTIC, G=G_b[bi[0]], loss_out=loss_b[bi[0]], ws=wsA)
 
     # set-up, once per (R, assignment) like the assignment itself: the holder
     # table and Algorithm 1's solution for every (chunk, holder subset)
     prep = gc.gc_decode_prepare(Rd, ell, od, N, m, delta)
 
     def stage_b():  # Algorithm 1 for the batch -> decode plan (psi side, no G needed)
-        gc.gc_decode_plan_prepared(prep, Rd, ell, N, m, delta, psi_b[bi[0]], plan=plan_s,
+        gc.gc_decode_plan_prepared(prep, Rd, ell, N, m, delta, psi_b[bi[0]], plan=plan_b[bi[0]],
                                    coef_err=ce_b[bi[0]], est=est_b[bi[0]], ws=wsB)
 
     def stage_c():  # batched decode-combine from the plan and G
-        gc.gc_decode_apply(plan_s, ell, N, npat, G_s, Ghat=Gh_s, grad_mse=mse_b[bi[0]], ws=wsC)
+        gc.gc_decode_apply(plan_b[bi[0]], ell, N, npat, G_b[bi[0]], Ghat=Gh_s, grad_mse=mse_b[bi[0]],
+                           ws=wsC)
 
     def stage_d1():  # Algorithm 1 for the live realization (independent of G)
         gc.gc_find_encoding_coeff(Rd, ell, od, N, m, delta, live_b[bi[0]], E=E_s, C=False,
                                   delta_out=False, support=False, coef_err=False, est=False, ws=wsD)
 
     def stage_d2():  # eq. (2) encode, PS decode, update
-        gc.gc_encode_with_coeffs(E_s, ell, od, N, m, delta, live_b[bi[0]], G_s, T=T_s)
+        gc.gc_encode_with_coeffs(E_s, ell, od, N, m, delta, live_b[bi[0]], G_b[bi[0]], T=T_s)
         gc.gc_decode_tx(Rd, ell, m, T_s, d, ghat=gh_s)
         gc.gc_sgd_step(w, gh_s[0], cfg.lr, cfg.Ntil)
 
@@ -724,12 +758,14 @@ def logistic_arm(args, rank, world, local_rank):
     torch.cuda.synchronize()
     serial_ms = [ser_ev[2 * si].elapsed_time(ser_ev[2 * si + 1]) for si in range(len(stages))]
 
-    # two graphs per step: the main stream runs the long kernels, high-priority
-    # side streams run the small, independent ones beside them (their blocks
-    # then take free SM room before further CTAs of the long kernels), all
-    # joined back at the end of the graph:
-    #   g1: chunk gradients (A)        || Algorithm 1, live (D1) || Algorithm 1, batch (B)
-    #   g2: batched decode-combine (C) || live encode / decode / update (D2)
+    # two graphs per step on two streams.  g1 runs the chunk gradients (A)
+    # with Algorithm 1 for the live realization (D1) and for the batch (B) on
+    # high-priority side streams beside it, then the live encode / decode /
+    # update (D2), which gives the next step's w.  g2 is the batched decode
+    # (C); it needs A and B of its step but nothing of the next one, so it
+    # runs on its own stream while g1 of the next step streams X (the chunk
+    # gradients and the plan are double-buffered; a step's g1 waits for the
+    # decode of two steps before, which read its buffers).
     n0 = gc.gc_kernel_launches()
     cap_stream = torch.cuda.Stream(dev)
     cap_hi = [torch.cuda.Stream(dev, priority=-1) for _ in range(2)]
@@ -765,8 +801,9 @@ def logistic_arm(args, rank, world, local_rank):
         g2.append(torch.cuda.CUDAGraph())
         with torch.cuda.graph(g1[b], stream=cap_stream):
             fork_join([stage_a], [stage_d1], [stage_b])
+            stage_d2()
         with torch.cuda.graph(g2[b], stream=cap_stream):
-            fork_join([stage_c], [stage_d2])
+            stage_c()
         if b == 0:
             launches_per_step = gc.gc_kernel_launches() - n0
     # instrumented copies of buffer 0's graphs for every EVERY-th timed step:
@@ -784,15 +821,18 @@ def logistic_arm(args, rank, world, local_rank):
         g2i.append(torch.cuda.CUDAGraph())
         with torch.cuda.graph(g1i[j], stream=cap_stream):
             fork_join([timed(stage_a, kev[j][0])], [stage_d1], [stage_b])
+            stage_d2()
         with torch.cuda.graph(g2i[j], stream=cap_stream):
-            fork_join([timed(stage_c, kev[j][1])], [stage_d2])
+            timed(stage_c, kev[j][1])()
     torch.cuda.synchronize()
 
     stream = torch.cuda.current_stream(dev)
+    dec_stream = torch.cuda.Stream(dev)  # the batched decode (g2)
 
     copy_stream = torch.cuda.Stream(dev)
     ev_ready = [torch.cuda.Event() for _ in range(2)]  # inputs of the buffer's next step are in
-    ev_done = [torch.cuda.Event() for _ in range(2)]   # the buffer's step has finished
+    ev_g1 = [torch.cuda.Event() for _ in range(2)]     # the buffer's g1 has finished
+    ev_done = [torch.cuda.Event() for _ in range(2)]   # the buffer's step (g1 and g2) has finished
     ev_out = [torch.cuda.Event() for _ in range(2)]    # the buffer's results have been read out
 
     def put_inputs(t, b, src):
@@ -817,20 +857,24 @@ def logistic_arm(args, rank, world, local_rank):
             assert b == 0
             ga, gb = g1i[(k // EVERY) % NE], g2i[(k // EVERY) % NE]
 
-        def rec(i):
+        def rec(i, st):
             if evs is not None:
-                evs[i].record(stream)
+                evs[i].record(st)
         if t_next is not None:
             put_inputs(t_next, 1 - b, src)
         stream.wait_event(ev_ready[b])
-        stream.wait_event(ev_out[b])  # results of step k - 2 have been read out
-        rec(0)
+        stream.wait_event(ev_done[b])  # the decode of step k - 2 has read this buffer's G and plan
+        stream.wait_event(ev_out[b])   # results of step k - 2 have been read out
+        rec(0, stream)
         ga.replay()
-        rec(1)
-        rec(2)
-        gb.replay()
-        rec(3)
-        ev_done[b].record(stream)
+        rec(1, stream)
+        ev_g1[b].record(stream)
+        dec_stream.wait_event(ev_g1[b])
+        with torch.cuda.stream(dec_stream):
+            rec(2, dec_stream)
+            gb.replay()
+            rec(3, dec_stream)
+        ev_done[b].record(dec_stream)
         if outs is not None:
             with torch.cuda.stream(copy_stream):
                 copy_stream.wait_event(ev_done[b])
@@ -876,6 +920,7 @@ def logistic_arm(args, rank, world, local_rank):
     put_inputs(batch[0], 0, src_dev)
     for k in range(K):
         run_step(k, batch[k], batch[k + 1] if k + 1 < K else None, src_dev, evs.get(k))
+    stream.wait_stream(dec_stream)
     t_end.record(stream)
     torch.cuda.synchronize()
     barrier()
@@ -928,7 +973,7 @@ def logistic_arm(args, rank, world, local_rank):
     # ---- roofline of the dominant stage
     pk, pk_src = peaks()
     hbm = float(pk["hbm_gbs"])
-    names = ["k_chunkgrad", "k_patterns", "k_combine_tc", "k_patterns(live)",
+    names = ["k_chunkgrad", "k_patterns", "gc_decode_apply", "k_patterns(live)",
              "encode+decode_tx+sgd"]
     alg_bytes = [
         cfg.Ntil * d * 4 + cfg.Ntil * 4 + N * d * 4,                          # X, y read; G written
@@ -937,7 +982,7 @@ def logistic_arm(args, rank, world, local_rank):
         m * 4 + m * delta * ell * 8,                                          # psi read; E written
         N * d * 4 + m * L * 4 * 2 + d * 4 * 3,                                # G read; T; ghat; w
     ]
-    srcs = [["k_chunkgrad.cu"], ["k_solve.cu"], ["k_combine_tc.cu"], ["k_solve.cu"],
+    srcs = [["k_chunkgrad.cu"], ["k_solve.cu"], ["k_decode_resid.cu"], ["k_solve.cu"],
             ["k_encode.cu"]]
     # the dominant kernel: the longer of the two HBM-bound calls on the
     # critical path (chunk gradients in g1, decode-combine in g2)
@@ -947,19 +992,17 @@ def logistic_arm(args, rank, world, local_rank):
     roofline = {"kernel": names[dom], "bound": "hbm", "achieved": achieved, "peak": hbm,
                 "unit": "GB/s", "frac": achieved / hbm, "peak_source": f"{pk_src} hbm_gbs",
                 "traffic": _traffic(names[dom], srcs[dom]),
-                "timing": "CUDA events recorded by event nodes inside the step's graph, on the "
-                          "kernel's stream, around its call (the kernel with its helper kernels: "
-                          "the chunk-gradient reduction, or the operand split and MSE reduction), "
-                          f"in every {EVERY}th timed step (the last {n_used} averaged), with the "
-                          "side-stream work running beside it",
+                "timing": "CUDA events recorded by event nodes inside the step's graphs, on the "
+                          "call's stream, around the call (the chunk-gradient kernel with its "
+                          "reduction; the batched decode with its scan, s and MSE reduction), "
+                          f"in every {EVERY}th timed step (the last {n_used} averaged); the "
+                          "decode of step t runs beside the chunk gradients of step t + 1",
                 "call_ms": {"k_chunkgrad (+ reduction)": float(call_ms[0]),
-                            "k_combine_tc (+ split, MSE reduction)": float(call_ms[1])},
+                            "gc_decode_apply": float(call_ms[1])},
                 "call_frac_of_hbm": {"k_chunkgrad": float(alg_bytes[0] / (call_ms[0] / 1e3) / 1e9 / hbm),
-                                     "k_combine_tc": float(alg_bytes[2] / (call_ms[1] / 1e3) / 1e9 / hbm)},
-                "graph_ms": {"k_chunkgrad || Algorithm 1": float(stage_ms[0]),
-                             "k_combine_tc || live encode/decode/update": float(stage_ms[1])},
-                "graph_frac_of_hbm": {"k_chunkgrad": float(alg_bytes[0] / (stage_ms[0] / 1e3) / 1e9 / hbm),
-                                      "k_combine_tc": float(alg_bytes[2] / (stage_ms[1] / 1e3) / 1e9 / hbm)},
+                                     "gc_decode_apply": float(alg_bytes[2] / (call_ms[1] / 1e3) / 1e9 / hbm)},
+                "graph_ms": {"g1: k_chunkgrad || Algorithm 1, then live encode/decode/update": float(stage_ms[0]),
+                             "g2: batched decode": float(stage_ms[1])},
                 "serial_stage_ms": {n: float(v) for n, v in zip(names, serial_ms)}}
 
     line = {
@@ -1079,20 +1122,28 @@ def extra_workload(args):
         wsM = gc.Workspace(dev)
         res = {}
         t_mse_tot = 0.0
-        for p in (0.3, 0.5, 0.7):
-            pd = torch.from_numpy(make_patterns(cfg, p=p)).to(dev)
-            t = _time_ms(torch, lambda: gc.gc_mse(Rd, ell, od, N, m, delta, pd, G, ws=wsM), 3)
-            out = gc.gc_mse(Rd, ell, od, N, m, delta, pd, G, ws=wsM)
-            gc.gc_status(wsM)
-            res[str(p)] = {"ms": t, "mean_grad_mse": float(out["grad_mse"].mean()),
-                           "mean_coef_err": float(out["coef_err"].mean()),
-                           "mean_est": float(out["est"].mean())}
-            t_mse_tot += t
         L = -(-d // ell)
         useful = 2.0 * npat * ell * (N * ell) * L
         Kp = -(-N * ell // 64) * 64
         issued = 3 * 2.0 * npat * ell * Kp * L
+        bf16s = float(pk.get("bf16_tflops_sustained", bf16))
+        for p in (0.3, 0.5, 0.7):
+            psi_h = make_patterns(cfg, p=p)
+            pd = torch.from_numpy(psi_h).to(dev)
+            t = _time_ms(torch, lambda: gc.gc_mse(Rd, ell, od, N, m, delta, pd, G, ws=wsM), 3)
+            out = gc.gc_mse(Rd, ell, od, N, m, delta, pd, G, ws=wsM)
+            gc.gc_status(wsM)
+            gf = gemm_tile_fraction(psi_h, order, N, ell)
+            res[str(p)] = {"ms": t, "patterns/s": npat / (t / 1e3), "gemm_tile_frac": gf,
+                           "mean_grad_mse": float(out["grad_mse"].mean()),
+                           "mean_coef_err": float(out["coef_err"].mean()),
+                           "mean_est": float(out["est"].mean())}
+            if gf > 0.99:
+                res[str(p)].update({"issued_tflops": issued / (t / 1e3) / 1e12,
+                                    "useful_tflops": useful / (t / 1e3) / 1e12})
+            t_mse_tot += t
         t_mse = t_mse_tot / 3
+        t_dense = res["0.3"]["ms"]
         line.update({
             "metric": f"patterns/sec (MSE only, m=N=64, delta=8, d=65536, 10^5 patterns, l={ell})",
             "value": npat / (t_mse / 1e3), "unit": "patterns/s",
@@ -1100,12 +1151,15 @@ def extra_workload(args):
                             "frac_of_hbm": cfg.Ntil * d * 2 / (t_cg / 1e3) / 1e9 / hbm,
                             "TFLOP/s": 4.0 * cfg.Ntil * d / (t_cg / 1e3) / 1e12},
             "per_p": res,
-            "roofline": {"kernel": "k_combine_tc (MSE only)", "bound": "tensor", "unit": "TFLOP/s",
-                         "achieved": issued / (t_mse / 1e3) / 1e12, "peak": bf16,
-                         "frac": issued / (t_mse / 1e3) / 1e12 / bf16,
-                         "useful_tflops": useful / (t_mse / 1e3) / 1e12,
-                         "note": "timed gc_mse includes Algorithm 1 for the 10^5 patterns",
-                         "peak_source": f"{pk_src} bf16_tflops"},
+            "roofline": {"kernel": "k_combine_tc (MSE only; p = 0.3, whose row tiles are all on the GEMM)",
+                         "bound": "tensor", "unit": "TFLOP/s",
+                         "achieved": issued / (t_dense / 1e3) / 1e12, "peak": bf16s,
+                         "frac": issued / (t_dense / 1e3) / 1e12 / bf16s,
+                         "useful_tflops": useful / (t_dense / 1e3) / 1e12,
+                         "note": "issued = three bf16 MMAs per K step over the padded K; the timed gc_mse "
+                                 "includes Algorithm 1 for the 10^5 patterns; p = 0.5 and 0.7 take the "
+                                 "residual path (gemm_tile_frac per p)",
+                         "peak_source": f"{pk_src} bf16_tflops_sustained"},
             "dtype": "bf16 X, f32 otherwise",
             "config": {"workload": f"sweep m=N=64 delta=8 d=65536 n_c=1024 bf16 npat=10^5 ell={ell}",
                        "l2": "inputs larger than L2 (X 8.6 GB)"}})

@@ -252,19 +252,77 @@ __global__ void __launch_bounds__(128) k_gsum(const float* __restrict__ G, int N
 // ---------------------------------------------------------------------------
 __device__ __forceinline__ float4 ld4(const float* p, long long off, bool vec, int nvalid) {
   if (vec && nvalid == 4) return __ldg(reinterpret_cast<const float4*>(p + off));
-  float v[4] = {0.f, 0.f, 0.f, 0.f};
-  for (int u = 0; u < nvalid; ++u) v[u] = __ldg(p + off + u);
-  return make_float4(v[0], v[1], v[2], v[3]);
+  float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
+  if (nvalid > 0) v.x = __ldg(p + off);
+  if (nvalid > 1) v.y = __ldg(p + off + 1);
+  if (nvalid > 2) v.z = __ldg(p + off + 2);
+  if (nvalid > 3) v.w = __ldg(p + off + 3);
+  return v;
 }
 __device__ __forceinline__ void st4(float* p, long long off, bool vec, int nvalid, float4 v) {
   if (vec && nvalid == 4) {
     __stcs(reinterpret_cast<float4*>(p + off), v);  // written once, never re-read here
     return;
   }
-  const float a[4] = {v.x, v.y, v.z, v.w};
-  for (int u = 0; u < nvalid; ++u) __stcs(p + off + u, a[u]);
+  if (nvalid > 0) __stcs(p + off, v.x);
+  if (nvalid > 1) __stcs(p + off + 1, v.y);
+  if (nvalid > 2) __stcs(p + off + 2, v.z);
+  if (nvalid > 3) __stcs(p + off + 3, v.w);
 }
 
+// One corrected row (pattern b, block k) over this thread's 4 columns:
+// ghat = s + sum_e sum_k' D_e[k][k'] g_{i_e}[k'L + c], and its squared-error
+// partial (one per warp) into the row's slot.
+template <int ELL>
+__device__ __forceinline__ void resid_row(const float* __restrict__ G, const ResidLists& rl, int b,
+                                          int k, long long row, int r, int c, int d, int L,
+                                          bool vecw, const int (&nv)[ELL], const float4 (&sv)[ELL],
+                                          float* __restrict__ Ghat) {
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int nz = __ldg(rl.nnz + b);  // <= ksp: longer lists make the tile dense
+  float4 cr = make_float4(0.f, 0.f, 0.f, 0.f);
+  for (int e = 0; e < nz; ++e) {
+    const int i = __ldg(rl.idx + (size_t)b * rl.ksp + e);
+    const float* Dr = rl.D + ((size_t)b * rl.ksp + e) * ELL * ELL + k * ELL;
+#pragma unroll
+    for (int kp = 0; kp < ELL; ++kp) {
+      const float w = __ldg(Dr + kp);
+      if (nv[kp] == 0 || w == 0.f) continue;
+      const float4 g = ld4(G, (size_t)i * d + (size_t)kp * L + c, vecw, nv[kp]);
+      cr.x = fmaf(w, g.x, cr.x);
+      cr.y = fmaf(w, g.y, cr.y);
+      cr.z = fmaf(w, g.z, cr.z);
+      cr.w = fmaf(w, g.w, cr.w);
+    }
+  }
+  int nvk = 0;
+  float4 svk = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+  for (int kk = 0; kk < ELL; ++kk)
+    if (kk == k) {
+      nvk = nv[kk];
+      svk = sv[kk];
+    }
+  // corrections only on the output columns that exist
+  float sq = nvk > 0 ? cr.x * cr.x : 0.f;
+  if (nvk > 1) sq = fmaf(cr.y, cr.y, sq);
+  if (nvk > 2) sq = fmaf(cr.z, cr.z, sq);
+  if (nvk > 3) sq = fmaf(cr.w, cr.w, sq);
+  if (Ghat && nvk > 0)
+    st4(Ghat, (size_t)b * d + (size_t)k * L + c, vecw, nvk,
+        make_float4(svk.x + cr.x, svk.y + cr.y, svk.z + cr.z, svk.w + cr.w));
+  if (rl.msp) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) sq += __shfl_xor_sync(0xffffffffu, sq, o);
+    if (lane == 0) {
+      const int slot = __ldg(rl.rslot + row);
+      rl.msp[(size_t)slot * rl.parts + (size_t)r * (kResidThreads / 32) + warp] = sq;
+    }
+  }
+}
+
+// Block (tile mt, range r, row slice z): rows [row0 + z*rps, row0 + (z+1)*rps)
+// of the tile (rps = 128 / gridDim.z; slices give small batches more blocks).
 template <int ELL>
 __global__ void __launch_bounds__(kResidThreads, ELL <= 4 ? 4 : 2) k_decode_resid(const float* __restrict__ G,
                                                                 const float* __restrict__ gsum,
@@ -273,11 +331,14 @@ __global__ void __launch_bounds__(kResidThreads, ELL <= 4 ? 4 : 2) k_decode_resi
                                                                 float* __restrict__ Ghat) {
   const int mt = blockIdx.x;
   if (__ldg(rl.tflag + mt)) return;  // the GEMM writes this tile
+  const int cnt = __ldg(rl.tcount + mt);
+  if (!Ghat && cnt == 0) return;     // errors only and every pattern exact: nothing to do
   const int r = blockIdx.y;
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const long long M = (long long)npat * ELL;
-  const long long row0 = (long long)mt * 128;
-  const long long row_end = min(row0 + 128, M);
+  const int rps = 128 / gridDim.z;
+  const long long lo = (long long)mt * 128 + (long long)blockIdx.z * rps;
+  const long long hi = min(lo + rps, M);
+  if (lo >= hi) return;
   const int c = r * kResidW + threadIdx.x * 4;
   const bool vecw = vec != 0;
   // valid columns of this thread in block k (padding past L and past d), and s there
@@ -289,51 +350,28 @@ __global__ void __launch_bounds__(kResidThreads, ELL <= 4 ? 4 : 2) k_decode_resi
     int n = min(4, L - c);
     n = (int)min((long long)n, (long long)d - col);
     nv[k] = n < 0 ? 0 : n;
-    sv[k] = nv[k] > 0 ? ld4(gsum, col, vecw, nv[k]) : make_float4(0.f, 0.f, 0.f, 0.f);
+    sv[k] = (Ghat && nv[k] > 0) ? ld4(gsum, col, vecw, nv[k]) : make_float4(0.f, 0.f, 0.f, 0.f);
   }
-  const int b_lo = (int)(row0 / ELL), b_hi = (int)((row_end - 1) / ELL);
+  if (!Ghat) {
+    // errors only: the tile's listed rows in this slice
+    for (int q = 0; q < cnt; ++q) {
+      const int row = __ldg(rl.rowlist + (size_t)mt * kResidRcap + q);
+      if (row < lo || row >= hi) continue;
+      resid_row<ELL>(G, rl, row / ELL, row % ELL, row, r, c, d, L, vecw, nv, sv, nullptr);
+    }
+    return;
+  }
+  const int b_lo = (int)(lo / ELL), b_hi = (int)((hi - 1) / ELL);
   for (int b = b_lo; b <= b_hi; ++b) {
-    const size_t obase = (size_t)b * d;
     const int nz = __ldg(rl.nnz + b);
 #pragma unroll
     for (int k = 0; k < ELL; ++k) {
       const long long row = (long long)b * ELL + k;
-      if (row < row0 || row >= row_end) continue;  // the neighbouring tile's row
+      if (row < lo || row >= hi) continue;  // another slice's or tile's row
       if (nz == 0) {  // exact pattern: ghat_b = s, zero error
-        if (Ghat && nv[k] > 0) st4(Ghat, obase + (size_t)k * L + c, vecw, nv[k], sv[k]);
-        continue;
-      }
-      // a corrected row (nz <= ksp: longer lists make the tile dense)
-      float4 cr = make_float4(0.f, 0.f, 0.f, 0.f);
-      for (int e = 0; e < nz; ++e) {
-        const int i = __ldg(rl.idx + (size_t)b * rl.ksp + e);
-        const float* Dr = rl.D + ((size_t)b * rl.ksp + e) * ELL * ELL + k * ELL;
-#pragma unroll
-        for (int kp = 0; kp < ELL; ++kp) {
-          const float w = __ldg(Dr + kp);
-          if (nv[kp] == 0 || w == 0.f) continue;
-          const float4 g = ld4(G, (size_t)i * d + (size_t)kp * L + c, vecw, nv[kp]);
-          cr.x = fmaf(w, g.x, cr.x);
-          cr.y = fmaf(w, g.y, cr.y);
-          cr.z = fmaf(w, g.z, cr.z);
-          cr.w = fmaf(w, g.w, cr.w);
-        }
-      }
-      // corrections only on the output columns that exist
-      float sq = nv[k] > 0 ? cr.x * cr.x : 0.f;
-      if (nv[k] > 1) sq = fmaf(cr.y, cr.y, sq);
-      if (nv[k] > 2) sq = fmaf(cr.z, cr.z, sq);
-      if (nv[k] > 3) sq = fmaf(cr.w, cr.w, sq);
-      if (Ghat && nv[k] > 0)
-        st4(Ghat, obase + (size_t)k * L + c, vecw, nv[k],
-            make_float4(sv[k].x + cr.x, sv[k].y + cr.y, sv[k].z + cr.z, sv[k].w + cr.w));
-      if (rl.msp) {
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) sq += __shfl_xor_sync(0xffffffffu, sq, o);
-        if (lane == 0) {
-          const int slot = __ldg(rl.rslot + row);
-          rl.msp[(size_t)slot * rl.parts + (size_t)r * (kResidThreads / 32) + warp] = sq;
-        }
+        if (nv[k] > 0) st4(Ghat, (size_t)b * d + (size_t)k * L + c, vecw, nv[k], sv[k]);
+      } else {
+        resid_row<ELL>(G, rl, b, k, row, r, c, d, L, vecw, nv, sv, Ghat);
       }
     }
   }
@@ -386,8 +424,11 @@ int launch_decode_resid(const float* G, const float* gsum, const ResidLists& rl,
   const long long nranges = (L + kResidW - 1) / kResidW;
   if (nmt > (1LL << 31) - 1 || nranges > 65535) return fail(GC_ERR_UNSUPPORTED, "residual decode grid too large");
   // tiles fastest: the CTAs of one column range run side by side and share
-  // its chunk-gradient lines in L2
-  dim3 grid((unsigned)nmt, (unsigned)nranges);
+  // its chunk-gradient lines in L2; small batches split each tile's rows
+  // over up to 8 blocks so that every SM has a few
+  int slices = 1;
+  while (slices < 8 && nmt * nranges * slices < 16LL * device_sm_count()) slices *= 2;
+  dim3 grid((unsigned)nmt, (unsigned)nranges, (unsigned)slices);
 #define GC_RESID(E) \
   case E: k_decode_resid<E><<<grid, kResidThreads, 0, s>>>(G, gsum, rl, npat, d, L, vec ? 1 : 0, Ghat); break;
   switch (ell) {
