@@ -196,11 +196,14 @@ __global__ void __launch_bounds__(kEncThreads, DR == 32 ? 3 : 4)
   for (int q = 0; q < kEncStages - 1; ++q) issue();
   const float* rd = s_ring + threadIdx.x * V;  // this thread's slot 0
   int rs = 0;  // ring slot of the step being consumed
-  float acc[DR][V];
+  // accumulators as column pairs: one packed two-wide FMA (__ffma2_rn, the
+  // same rounding as two fmaf) per pair
+  constexpr int V2 = V / 2;
+  float2 acc[DR][V2];
 #pragma unroll
   for (int r = 0; r < DR; ++r)
 #pragma unroll
-    for (int v = 0; v < V; ++v) acc[r][v] = 0.f;
+    for (int v = 0; v < V2; ++v) acc[r][v] = make_float2(0.f, 0.f);
   // sweep position w holds chunk (j0 + w) mod N; worker j0 + w - p takes it
   // in slot p, ring slot (w - p) mod DR; worker j0 + w - DR + 1 is complete after it
   const float* ecol = s_e;  // coefficients of (k = 0, w)
@@ -213,14 +216,14 @@ __global__ void __launch_bounds__(kEncThreads, DR == 32 ? 3 : 4)
         {
           issue();
           cp_async_wait<kEncStages - 1>();  // this step's copy has landed
-          float g[V];
+          float2 g[V2];
           const float* gp = rd + rs * (kEncThreads * V);
           if (V == 4) {
             const float4 q = *reinterpret_cast<const float4*>(gp);
-            g[0] = q.x; g[V > 1 ? 1 : 0] = q.y; g[V > 2 ? 2 : 0] = q.z; g[V > 3 ? 3 : 0] = q.w;
+            g[0] = make_float2(q.x, q.y);
+            g[V2 > 1 ? 1 : 0] = make_float2(q.z, q.w);
           } else {
-            const float2 q = *reinterpret_cast<const float2*>(gp);
-            g[0] = q.x; g[V > 1 ? 1 : 0] = q.y;
+            g[0] = *reinterpret_cast<const float2*>(gp);
           }
           rs = (rs + 1) & (kEncStages - 1);
           const float4* e4 = reinterpret_cast<const float4*>(ecol + (size_t)kk * W * DR);
@@ -231,9 +234,10 @@ __global__ void __launch_bounds__(kEncThreads, DR == 32 ? 3 : 4)
 #pragma unroll
             for (int h = 0; h < 4; ++h) {
               const int p = 4 * q + h;
+              const float2 e2 = make_float2(ev[h], ev[h]);
 #pragma unroll
-              for (int v = 0; v < V; ++v)
-                acc[(u - p) & (DR - 1)][v] = fmaf(ev[h], g[v], acc[(u - p) & (DR - 1)][v]);
+              for (int v = 0; v < V2; ++v)
+                acc[(u - p) & (DR - 1)][v] = __ffma2_rn(e2, g[v], acc[(u - p) & (DR - 1)][v]);
             }
           }
         }
@@ -241,10 +245,15 @@ __global__ void __launch_bounds__(kEncThreads, DR == 32 ? 3 : 4)
       ecol += DR;
       const int jj = w - DR + 1;
       if (jj >= 0) {  // jj < nj since w < nj + DR - 1
-        float* a = acc[(u + 1) & (DR - 1)];
-        enc_store<V>(T + ((size_t)b * m + j0 + jj) * L + c, c, L, vec != 0, a);
+        float2* a2 = acc[(u + 1) & (DR - 1)];
+        float a[V];
 #pragma unroll
-        for (int v = 0; v < V; ++v) a[v] = 0.f;
+        for (int v = 0; v < V2; ++v) {
+          a[2 * v] = a2[v].x;
+          a[2 * v + 1] = a2[v].y;
+          a2[v] = make_float2(0.f, 0.f);
+        }
+        enc_store<V>(T + ((size_t)b * m + j0 + jj) * L + c, c, L, vec != 0, a);
       }
     }
   }
