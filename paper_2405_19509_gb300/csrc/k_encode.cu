@@ -147,14 +147,22 @@ __global__ void __launch_bounds__(kEncThreads, DR == 32 ? 3 : 4)
     }
     return;
   }
-  // diagonal staging: s_e[(k * W + w) * DR + p]
-  for (int t = threadIdx.x; t < ell * W * DR; t += kEncThreads) {
-    const int p = t % DR, w = (t / DR) % W, k = t / (DR * W);
-    const int jj = w - p;
-    float e = 0.f;
-    if (jj >= 0 && jj < nj && p < s_np[jj]) e = (float)Eb[(size_t)jj * de + p * ell + k];
-    s_e[t] = e;
-  }
+  // diagonal staging: s_e[(k * W + w) * DR + p]; a thread fills the DR slots
+  // of one (k, w) with four 16-byte stores
+  for (int k = 0; k < ell; ++k)
+    for (int w = threadIdx.x; w < W; w += kEncThreads) {
+      float4* dst = reinterpret_cast<float4*>(s_e + ((size_t)k * W + w) * DR);
+#pragma unroll 1
+      for (int q = 0; q < DR / 4; ++q) {
+        float e[4];
+#pragma unroll
+        for (int h = 0; h < 4; ++h) {
+          const int p = 4 * q + h, jj = w - p;
+          e[h] = (jj >= 0 && jj < nj && p < s_np[jj]) ? (float)Eb[(size_t)jj * de + p * ell + k] : 0.f;
+        }
+        dst[q] = make_float4(e[0], e[1], e[2], e[3]);
+      }
+    }
   __syncthreads();
   if (c >= L) return;  // no barrier below
   // ring: this thread's V floats of each stage
