@@ -271,3 +271,48 @@ def test_combine_non_projector_matrix(gc):
             assert_mse_close(float(res["grad_mse"][b]), mref[b], floor, f"{name} mse b={b}")
             assert_mse_close(float(mo[b]), mref[b], floor, f"{name} mse-only b={b}")
     assert np.max(np.abs(got["dense"] - got["residual"])) <= 1e-5 * np.max(np.abs(ref))
+
+
+@pytest.mark.parametrize("ell", [5, 8])
+def test_large_ell_both_paths(gc, ell):
+    """The widest communication factors of the build: N = m = 10 chunks and
+    workers, delta = 8, l = 5 and 8 (at l = 8 exact recovery needs every copy;
+    lists hold 8 blocks, so longer ones send their tiles to the GEMM), d not a
+    multiple of l.  Mostly exact patterns, mild stragglers and a few uniform
+    ones; every pattern against the oracle under each policy."""
+    N = m = 10
+    delta, d, npat = 8, 1003, 300
+    order = O.cyclic_order(N, m, delta)
+    rng = np.random.default_rng(70 + ell)
+    R = rng.standard_normal((ell, m))
+    # exact patterns; mild stragglers (a few consecutive workers stop up to 6
+    # chunks early: a few blocks below l copies); every 12th pattern uniform
+    psi = np.full((npat, m), delta, dtype=np.int32)
+    every = 3 if ell == 5 else 8   # a 128-row tile holds 25 patterns at l = 5, 16 at l = 8
+    for b in range(npat):
+        if b % (4 * every) == 5:
+            psi[b] = rng.integers(0, delta + 1, size=m)
+        elif b % every == 1:
+            j0 = rng.integers(0, m)
+            for t in range(int(rng.integers(1, 4))):
+                psi[b, (j0 + t) % m] = delta - int(rng.integers(1, 7))
+    G32 = rng.standard_normal((N, d)).astype(np.float32)
+    Gref = G32.astype(np.float64)
+    gsum = Gref.sum(axis=0)
+    floor = 1e-8 * float(gsum @ gsum) / d
+    Rd, od, pd = dev_tensors(R, order, psi)
+    Gd = torch.from_numpy(G32).cuda()
+    out = {k: _decode(gc, v, Rd, ell, od, N, m, delta, pd, Gd) for k, v in _policies(gc).items()}
+    nnz = (_copies(order, psi, N) < ell).sum(axis=1)
+    assert (nnz == 0).any() and (nnz > 8).any()
+    res_rows = _residual_rows(nnz, ell, 8)
+    assert res_rows.mean() > 0.3 and (np.repeat(nnz, ell)[res_rows] > 0).any()
+    cache = {}
+    for b in range(npat):
+        key = psi[b].tobytes()
+        if key not in cache:
+            cache[key] = O.run_pattern(R, order, psi[b], N, Gref, want_transmit=False)
+        r = cache[key]
+        for k, res in out.items():
+            assert_grad_close(to_np(res["Ghat"][b]), r.ghat, f"{k} l={ell} b={b}")
+            assert_mse_close(float(res["grad_mse"][b]), r.grad_mse, floor, f"{k} l={ell} mse b={b}")
