@@ -455,6 +455,9 @@ def decode_arm(args, rank, world, local_rank):
 
     stream = torch.cuda.current_stream(dev)
     copy_stream = torch.cuda.Stream(dev)
+    NCOPY = 4
+    d2h_streams = [torch.cuda.Stream(dev) for _ in range(NCOPY)]
+    ev_d2h = [torch.cuda.Event() for _ in range(NCOPY)]
     ev_ready = [torch.cuda.Event() for _ in range(2)]
     ev_done = [torch.cuda.Event() for _ in range(2)]
     ev_out = [torch.cuda.Event() for _ in range(2)]
@@ -478,12 +481,21 @@ def decode_arm(args, rank, world, local_rank):
         g.replay()
         ev_done[b].record(stream)
         if outs is not None:
+            # the decoded gradients leave in NCOPY row blocks on their own
+            # streams (one copy engine each), the errors on the copy stream
+            for q, cs in enumerate(d2h_streams):
+                rows = slice(q * npat // NCOPY, (q + 1) * npat // NCOPY)
+                with torch.cuda.stream(cs):
+                    cs.wait_event(ev_done[b])
+                    outs["Ghat"][rows].copy_(Gh_b[b][rows], non_blocking=True)
+                    ev_d2h[q].record(cs)
             with torch.cuda.stream(copy_stream):
                 copy_stream.wait_event(ev_done[b])
-                outs["Ghat"].copy_(Gh_b[b], non_blocking=True)
                 outs["ce"][k].copy_(ce_b[b], non_blocking=True)
                 outs["est"][k].copy_(est_b[b], non_blocking=True)
                 outs["mse"][k].copy_(mse_b[b], non_blocking=True)
+                for q in range(NCOPY):
+                    copy_stream.wait_event(ev_d2h[q])
                 ev_out[b].record(copy_stream)
 
     import torch.distributed as tdist

@@ -134,6 +134,11 @@ def test_wait_limit_knob_validation():
     assert gc.lib.gc_set_wait_limit(0) == 0
     assert gc.lib.gc_inject_stall(8) == -1
     assert gc.lib.gc_inject_stall(0) == 0
+    # decode path policy: the three documented values, anything else rejected
+    assert gc.lib.gc_set_decode_policy(3) == -1
+    assert gc.lib.gc_set_decode_policy(-1) == -1
+    for pol in (gc.GC_DECODE_DENSE, gc.GC_DECODE_RESIDUAL, gc.GC_DECODE_AUTO):
+        assert gc.lib.gc_set_decode_policy(pol) == 0
 
 
 def test_batched_chunk_grads_validation():
