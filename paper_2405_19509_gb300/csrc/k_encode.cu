@@ -20,11 +20,15 @@ namespace gc {
 // window of chunks has passed.  The chunk gradients are read once per
 // (pattern, worker group) instead of once per worker and slot.
 // Block = (pattern b, column stripe, worker group [j0, j1)).  The ring has DR
-// slots (DR = the power of two >= delta); the coefficients are staged
-// diagonally, s_d[k][w][p] = E[b][j0 + w - p][p][k] for the worker that holds
-// sweep position w in slot p (zero past its psi, for p >= delta and outside
-// the group), so every chunk step is DR/4 vector loads from shared memory and
-// DR*V FMAs with no branches; positions past the group's range add zeros.
+// slots (DR = the power of two >= delta): worker j0 + jj accumulates in ring
+// slot jj mod DR.  The coefficients are staged by ring slot,
+// s_e[k][w][s] = E[b][j0 + jj][p][k] with p = (w - s) mod DR and jj = w - p
+// (the worker in slot s takes the chunk at sweep position w as its p-th; zero
+// past its psi, for p >= delta and outside the group), so every chunk step is
+// DR/4 vector loads from shared memory and DR*V FMAs with no branches, and the
+// accumulators pair up by slot: one packed two-wide FMA takes the
+// coefficients of slots (2r, 2r+1) as they lie in shared memory and one
+// column's value twice.  Positions past the group's range add zeros.
 // Each thread keeps its next kEncStages - 1 chunk-stripe loads in flight:
 // cp.async copies its own columns of a coming (position, block) step into its
 // slots of a shared-memory ring (zero-filled past L and past d) and waits
@@ -147,22 +151,38 @@ __global__ void __launch_bounds__(kEncThreads, DR == 32 ? 3 : 4)
     }
     return;
   }
-  // diagonal staging: s_e[(k * W + w) * DR + p]; a thread fills the DR slots
-  // of one (k, w) with four 16-byte stores
-  for (int k = 0; k < ell; ++k)
-    for (int w = threadIdx.x; w < W; w += kEncThreads) {
-      float4* dst = reinterpret_cast<float4*>(s_e + ((size_t)k * W + w) * DR);
-#pragma unroll 1
-      for (int q = 0; q < DR / 4; ++q) {
-        float e[4];
-#pragma unroll
-        for (int h = 0; h < 4; ++h) {
-          const int p = 4 * q + h, jj = w - p;
-          e[h] = (jj >= 0 && jj < nj && p < s_np[jj]) ? (float)Eb[(size_t)jj * de + p * ell + k] : 0.f;
+  // staging by ring slot, s_e[(k * W + w) * DR + s]: zero everywhere, then
+  // each coefficient E[b][j0 + jj][p][k] (p < psi) lands at w = jj + p,
+  // s = jj mod DR.  A thread takes whole workers (its loads, the worker's
+  // p * ell + k run, are independent and go out together); consecutive
+  // threads take consecutive workers, so the scattered stores hit distinct
+  // banks (stride DR + 1 words).
+  {
+    float4* z = reinterpret_cast<float4*>(s_e);
+    const int nz = ell * W * DR / 4;
+    for (int t = threadIdx.x; t < nz; t += kEncThreads) z[t] = make_float4(0.f, 0.f, 0.f, 0.f);
+  }
+  __syncthreads();
+  {
+    const int kstep = W * DR;                     // next block k
+    const int pstep = DR - (ell - 1) * W * DR;    // last block -> next slot p
+    for (int jj = threadIdx.x; jj < nj; jj += kEncThreads) {
+      const double* ej = Eb + (size_t)jj * de;
+      float* sj = s_e + jj * (DR + 1) - (jj & ~(DR - 1));  // (jj + p) * DR + jj mod DR at p = 0
+      const int n = s_np[jj] * ell;
+      int off = 0, k = 0;
+#pragma unroll 8
+      for (int t = 0; t < n; ++t) {
+        sj[off] = (float)__ldg(ej + t);
+        if (++k == ell) {
+          k = 0;
+          off += pstep;
+        } else {
+          off += kstep;
         }
-        dst[q] = make_float4(e[0], e[1], e[2], e[3]);
       }
     }
+  }
   __syncthreads();
   if (c >= L) return;  // no barrier below
   // ring: this thread's V floats of each stage
@@ -170,14 +190,15 @@ __global__ void __launch_bounds__(kEncThreads, DR == 32 ? 3 : 4)
   constexpr uint32_t kStage = kEncThreads * V * 4;
   // every step copies V whole floats (vector rows, no padding in this thread's columns)
   const bool full = vec && c + V <= L && (long long)ell * L <= d;
-  // issue cursor: step (iw, ik) = block ik of the chunk at sweep position iw
+  // issue cursor: step (iw, ik) = block ik of the chunk at sweep position iw,
+  // read from src = G + ich * d + ik * L + c
   int iw = 0, ik = 0, slot = 0;
   int ich = j0 % N;
-  const float* gsrc = G + (size_t)ich * d + c;  // + ik * L
+  const float* src = G + (size_t)ich * d + c;
+  const int to_next = d - (ell - 1) * L;  // last block of a chunk -> first of the next
   auto issue = [&]() {
     if (iw < W) {
       const uint32_t dst = ring + slot * kStage;
-      const float* src = gsrc + (size_t)ik * L;
       if (full) {
         cp_async_zfill<V * 4>(dst, src, V * 4);
       } else {
@@ -196,70 +217,82 @@ __global__ void __launch_bounds__(kEncThreads, DR == 32 ? 3 : 4)
     if (++ik == ell) {
       ik = 0;
       ++iw;
-      if (++ich == N) ich = 0;
-      gsrc = G + (size_t)ich * d + c;
+      src += to_next;
+      if (++ich == N) {
+        ich = 0;
+        src = G + c;
+      }
+    } else {
+      src += L;
     }
     slot = (slot + 1) & (kEncStages - 1);
   };
   for (int q = 0; q < kEncStages - 1; ++q) issue();
   const float* rd = s_ring + threadIdx.x * V;  // this thread's slot 0
   int rs = 0;  // ring slot of the step being consumed
-  // accumulators as column pairs: one packed two-wide FMA (__ffma2_rn, the
-  // same rounding as two fmaf) per pair
-  constexpr int V2 = V / 2;
-  float2 acc[DR][V2];
+  // accumulators paired by ring slot: acc[r][v] = (slot 2r, slot 2r + 1) of
+  // column v; one packed two-wide FMA (__ffma2_rn, the same rounding as two
+  // fmaf) per pair
+  float2 acc[DR / 2][V];
 #pragma unroll
-  for (int r = 0; r < DR; ++r)
+  for (int r = 0; r < DR / 2; ++r)
 #pragma unroll
-    for (int v = 0; v < V2; ++v) acc[r][v] = make_float2(0.f, 0.f);
-  // sweep position w holds chunk (j0 + w) mod N; worker j0 + w - p takes it
-  // in slot p, ring slot (w - p) mod DR; worker j0 + w - DR + 1 is complete after it
+    for (int v = 0; v < V; ++v) acc[r][v] = make_float2(0.f, 0.f);
+  // sweep position w holds chunk (j0 + w) mod N; worker j0 + w - DR + 1, in
+  // ring slot (w + 1) mod DR, is complete after it
   const float* ecol = s_e;  // coefficients of (k = 0, w)
+  const int kstride = W * DR;  // <= kEncSmemFloats
   for (int w0 = 0; w0 < W; w0 += DR) {
 #pragma unroll
     for (int u = 0; u < DR; ++u) {
       const int w = w0 + u;
       if (w >= W) break;
-      for (int kk = 0; kk < ell; ++kk) {
-        {
-          issue();
-          cp_async_wait<kEncStages - 1>();  // this step's copy has landed
-          float2 g[V2];
-          const float* gp = rd + rs * (kEncThreads * V);
-          if (V == 4) {
-            const float4 q = *reinterpret_cast<const float4*>(gp);
-            g[0] = make_float2(q.x, q.y);
-            g[V2 > 1 ? 1 : 0] = make_float2(q.z, q.w);
-          } else {
-            g[0] = *reinterpret_cast<const float2*>(gp);
-          }
-          rs = (rs + 1) & (kEncStages - 1);
-          const float4* e4 = reinterpret_cast<const float4*>(ecol + (size_t)kk * W * DR);
+      const float* ek = ecol;
+      for (int kk = 0; kk < ell; ++kk, ek += kstride) {
+        issue();
+        cp_async_wait<kEncStages - 1>();  // this step's copy has landed
+        float g[V];
+        const float* gp = rd + rs * (kEncThreads * V);
+        if (V == 4) {
+          const float4 q = *reinterpret_cast<const float4*>(gp);
+          g[0] = q.x;
+          g[1 % V] = q.y;
+          g[2 % V] = q.z;
+          g[3 % V] = q.w;
+        } else {
+          const float2 q = *reinterpret_cast<const float2*>(gp);
+          g[0] = q.x;
+          g[1 % V] = q.y;
+        }
+        rs = (rs + 1) & (kEncStages - 1);
+        const float4* e4 = reinterpret_cast<const float4*>(ek);
 #pragma unroll
-          for (int q = 0; q < DR / 4; ++q) {
-            const float4 e = e4[q];
-            const float ev[4] = {e.x, e.y, e.z, e.w};
+        for (int q = 0; q < DR / 4; ++q) {
+          const float4 e = e4[q];
+          const float2 lo = make_float2(e.x, e.y), hi = make_float2(e.z, e.w);
 #pragma unroll
-            for (int h = 0; h < 4; ++h) {
-              const int p = 4 * q + h;
-              const float2 e2 = make_float2(ev[h], ev[h]);
-#pragma unroll
-              for (int v = 0; v < V2; ++v)
-                acc[(u - p) & (DR - 1)][v] = __ffma2_rn(e2, g[v], acc[(u - p) & (DR - 1)][v]);
-            }
+          for (int v = 0; v < V; ++v) {
+            const float2 gg = make_float2(g[v], g[v]);
+            acc[2 * q][v] = __ffma2_rn(lo, gg, acc[2 * q][v]);
+            acc[2 * q + 1][v] = __ffma2_rn(hi, gg, acc[2 * q + 1][v]);
           }
         }
       }
       ecol += DR;
       const int jj = w - DR + 1;
       if (jj >= 0) {  // jj < nj since w < nj + DR - 1
-        float2* a2 = acc[(u + 1) & (DR - 1)];
+        const int sc = (u + 1) & (DR - 1);  // compile-time: u is unrolled
         float a[V];
 #pragma unroll
-        for (int v = 0; v < V2; ++v) {
-          a[2 * v] = a2[v].x;
-          a[2 * v + 1] = a2[v].y;
-          a2[v] = make_float2(0.f, 0.f);
+        for (int v = 0; v < V; ++v) {
+          float2& pr = acc[sc >> 1][v];
+          if (sc & 1) {
+            a[v] = pr.y;
+            pr.y = 0.f;
+          } else {
+            a[v] = pr.x;
+            pr.x = 0.f;
+          }
         }
         enc_store<V>(T + ((size_t)b * m + j0 + jj) * L + c, c, L, vec != 0, a);
       }
