@@ -84,6 +84,37 @@ __device__ __forceinline__ void enc_store(float* __restrict__ Tr, int c, int L, 
   }
 }
 
+// Move the accumulators of ring slot S (half S & 1 of pair S >> 1) to a and
+// clear them.
+template <int DR, int V, int S>
+__device__ __forceinline__ void enc_take(float2 (&acc)[DR / 2][V], float* a) {
+#pragma unroll
+  for (int v = 0; v < V; ++v) {
+    float2& pr = acc[S >> 1][v];
+    if (S & 1) {
+      a[v] = pr.y;
+      pr.y = 0.f;
+    } else {
+      a[v] = pr.x;
+      pr.x = 0.f;
+    }
+  }
+}
+
+// enc_take of slot sc in [LO, HI), by binary search on sc
+template <int DR, int V, int LO, int HI>
+__device__ __forceinline__ void enc_take_any(float2 (&acc)[DR / 2][V], int sc, float* a) {
+  if constexpr (HI - LO == 1) {
+    enc_take<DR, V, LO>(acc, a);
+  } else {
+    constexpr int MID = (LO + HI) / 2;
+    if (sc < MID)
+      enc_take_any<DR, V, LO, MID>(acc, sc, a);
+    else
+      enc_take_any<DR, V, MID, HI>(acc, sc, a);
+  }
+}
+
 // Workers per group so that the diagonal staging fits (and at most 256).
 __host__ __device__ inline int enc_group_max(int DR, int ell) {
   const int j = kEncSmemFloats / (ell * DR) - DR;
@@ -241,12 +272,13 @@ __global__ void __launch_bounds__(kEncThreads, DR == 32 ? 3 : 4)
   // sweep position w holds chunk (j0 + w) mod N; worker j0 + w - DR + 1, in
   // ring slot (w + 1) mod DR, is complete after it
   const float* ecol = s_e;  // coefficients of (k = 0, w)
+  float* tout = T + ((size_t)b * m + j0) * L + c;  // transmission of the next worker to complete
   const int kstride = W * DR;  // <= kEncSmemFloats
-  for (int w0 = 0; w0 < W; w0 += DR) {
-#pragma unroll
-    for (int u = 0; u < DR; ++u) {
-      const int w = w0 + u;
-      if (w >= W) break;
+  // one copy of the step's code for every w (the FMAs do not depend on w);
+  // the completed slot is taken through a switch on its index
+#pragma unroll 1
+  for (int w = 0; w < W; ++w) {
+    {
       const float* ek = ecol;
       for (int kk = 0; kk < ell; ++kk, ek += kstride) {
         issue();
@@ -281,20 +313,10 @@ __global__ void __launch_bounds__(kEncThreads, DR == 32 ? 3 : 4)
       ecol += DR;
       const int jj = w - DR + 1;
       if (jj >= 0) {  // jj < nj since w < nj + DR - 1
-        const int sc = (u + 1) & (DR - 1);  // compile-time: u is unrolled
         float a[V];
-#pragma unroll
-        for (int v = 0; v < V; ++v) {
-          float2& pr = acc[sc >> 1][v];
-          if (sc & 1) {
-            a[v] = pr.y;
-            pr.y = 0.f;
-          } else {
-            a[v] = pr.x;
-            pr.x = 0.f;
-          }
-        }
-        enc_store<V>(T + ((size_t)b * m + j0 + jj) * L + c, c, L, vec != 0, a);
+        enc_take_any<DR, V, 0, DR>(acc, (w + 1) & (DR - 1), a);
+        enc_store<V>(tout, c, L, vec != 0, a);
+        tout += L;
       }
     }
   }

@@ -243,6 +243,38 @@ def test_decode_full(gc, decode_data, ell, nsamp):
     torch.cuda.empty_cache()
 
 
+@pytest.mark.parametrize("npat", [1, 8])
+def test_decode_encode_full(gc, decode_data, npat):
+    """Eq. (2) at the decode batch's shape (m = N = 256, delta = 16, the
+    16-slot ring, L = 2^19) for one pattern and for eight: the transmissions
+    of every worker on 4096 columns of each block against the oracle on those
+    columns (the encode treats columns independently); patterns: every worker
+    done, a mixed straggler pattern, and the rest drawn from the workload."""
+    cfg, Gd, G32 = decode_data
+    N, m, delta, d, ell = cfg.N, cfg.m, cfg.delta, cfg.d, 2
+    L = d // ell
+    psi = make_patterns(cfg)[:npat].copy()
+    psi[0] = delta
+    if npat > 1:
+        psi[1] = np.random.default_rng(41).integers(0, delta + 1, size=m)
+    R = make_R(cfg, ell)
+    order = O.cyclic_order(N, m, delta)
+    Rd, od, pd = dev_tensors(R, order, psi)
+    T = gc.gc_encode(Rd, ell, od, N, m, delta, pd, Gd)
+    torch.cuda.synchronize()
+    rng = np.random.default_rng(300 + npat)
+    cols = np.unique(np.concatenate([np.arange(1024), np.arange(L - 1024, L),
+                                     rng.choice(L, size=2048, replace=False)]))
+    full_cols = np.concatenate([k * L + cols for k in range(ell)])
+    Gs = G32[:, full_cols].astype(np.float64)
+    Ts = to_np(T.index_select(2, torch.from_numpy(cols).cuda()))
+    for b in sorted({0, npat - 1} | ({1} if npat > 1 else set())):
+        r = O.run_pattern(R, order, psi[b], N, Gs, want_transmit=True)
+        assert rel_inf(Ts[b], r.T) <= 1e-4, f"encode npat={npat} b={b} (sampled columns)"
+    del T
+    torch.cuda.empty_cache()
+
+
 # ------------------------------------------------------------------ coded SGD (m = 128)
 def _sgd_run_gpu(gc, cfg, data, ell, iters):
     N, m, delta = cfg.N, cfg.m, cfg.delta

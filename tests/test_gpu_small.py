@@ -330,6 +330,35 @@ def test_encode_long_rows(gc, explicit, npat):
             assert float(T[b].abs().max()) == 0.0
 
 
+@pytest.mark.parametrize("delta,d", [(5, 2600), (9, 2599), (16, 2600), (16, 2599), (17, 2600), (32, 2600)])
+def test_encode_ring_sizes(gc, delta, d):
+    """Eq. (2) through every ring size of the chunk sweep (8, 16 and 32
+    slots, with delta below and at the ring size), on three column stripes
+    with a ragged last one (L = 1300), 16-byte vectors (d = 2600) and scalar
+    columns with a padded last block (d = 2599); the patterns include every
+    worker done, none done, and mixed.  Few patterns, so the launch also
+    splits the workers into groups (each group sweeps its own chunks)."""
+    rng = np.random.default_rng(700 + delta + d)
+    N = m = 40
+    ell = 2
+    order = O.cyclic_order(N, m, delta)
+    R = rng.standard_normal((ell, m))
+    psi = rng.integers(0, delta + 1, size=(4, m)).astype(np.int32)
+    psi[0] = delta
+    psi[1] = 0
+    psi[2, ::3] = 0
+    G = rng.standard_normal((N, d)).astype(np.float32)
+    Rd, od, pd = dev_tensors(R, order, psi)
+    T = to_np(gc.gc_encode(Rd, ell, od, N, m, delta, pd, torch.from_numpy(G).cuda()))
+    G64 = G.astype(np.float64)
+    for b in range(psi.shape[0]):
+        r = O.run_pattern(R, order, psi[b], N, G64, want_transmit=True)
+        if np.max(np.abs(r.T)) > 0:
+            assert rel_inf(T[b], r.T) <= 1e-4, f"delta={delta} d={d} pattern {b}"
+        else:
+            assert float(np.abs(T[b]).max()) == 0.0
+
+
 @pytest.mark.parametrize("ell", [1, 3])
 def test_decode_plan_then_apply(gc, ell):
     """gc_decode_plan (psi side) then gc_decode_apply (data side) equals
