@@ -130,7 +130,9 @@ inline size_t enc_smem_bytes(int DR, int V, int ell, int delta, int J) {
 }
 
 // Four blocks per SM (three with a 32-slot ring): about 120 registers a thread.
-template <int DR, int V>
+// A step of the sweep is KB consecutive blocks k of one chunk (KB divides
+// ell): one copy group, one wait and KB times DR*V FMAs.
+template <int DR, int V, int KB>
 __global__ void __launch_bounds__(kEncThreads, DR == 32 ? 3 : 4)
     k_encode(const double* __restrict__ E, const int32_t* __restrict__ order,
              const int32_t* __restrict__ psi, int N, int m, int delta, int ell, int npat,
@@ -216,36 +218,43 @@ __global__ void __launch_bounds__(kEncThreads, DR == 32 ? 3 : 4)
   }
   __syncthreads();
   if (c >= L) return;  // no barrier below
-  // ring: this thread's V floats of each stage
+  // ring of NST stages, each [kb][thread][V]: this thread's V floats of each block
+  constexpr int NST = kEncStages / KB;
   const uint32_t ring = enc_smem_u32(s_ring) + threadIdx.x * (V * 4);
-  constexpr uint32_t kStage = kEncThreads * V * 4;
+  constexpr uint32_t kBlk = kEncThreads * V * 4;
+  constexpr uint32_t kStage = kBlk * KB;
   // every step copies V whole floats (vector rows, no padding in this thread's columns)
   const bool full = vec && c + V <= L && (long long)ell * L <= d;
-  // issue cursor: step (iw, ik) = block ik of the chunk at sweep position iw,
-  // read from src = G + ich * d + ik * L + c
+  // issue cursor: step (iw, ik) = blocks ik .. ik + KB - 1 of the chunk at
+  // sweep position iw, read from src = G + ich * d + ik * L + c
   int iw = 0, ik = 0, slot = 0;
   int ich = j0 % N;
   const float* src = G + (size_t)ich * d + c;
-  const int to_next = d - (ell - 1) * L;  // last block of a chunk -> first of the next
+  const int to_next = d - (ell - KB) * L;  // last step of a chunk -> first of the next
   auto issue = [&]() {
     if (iw < W) {
-      const uint32_t dst = ring + slot * kStage;
-      if (full) {
-        cp_async_zfill<V * 4>(dst, src, V * 4);
-      } else {
-        const long long col = (long long)ik * L + c;
-        int nv = min(V, L - c);
-        nv = (int)min((long long)nv, (long long)d - col);
-        if (vec) {
-          cp_async_zfill<V * 4>(dst, nv == V ? src : G, nv == V ? V * 4 : 0);
-        } else {
 #pragma unroll
-          for (int u = 0; u < V; ++u) cp_async_zfill<4>(dst + 4 * u, u < nv ? src + u : G, u < nv ? 4 : 0);
+      for (int kb = 0; kb < KB; ++kb) {
+        const uint32_t dst = ring + slot * kStage + kb * kBlk;
+        const float* sk = src + (size_t)kb * L;
+        if (full) {
+          cp_async_zfill<V * 4>(dst, sk, V * 4);
+        } else {
+          const long long col = (long long)(ik + kb) * L + c;
+          int nv = min(V, L - c);
+          nv = (int)min((long long)nv, (long long)d - col);
+          if (vec) {
+            cp_async_zfill<V * 4>(dst, nv == V ? sk : G, nv == V ? V * 4 : 0);
+          } else {
+#pragma unroll
+            for (int u = 0; u < V; ++u) cp_async_zfill<4>(dst + 4 * u, u < nv ? sk + u : G, u < nv ? 4 : 0);
+          }
         }
       }
     }
     cp_async_commit();  // one group per step (possibly empty)
-    if (++ik == ell) {
+    ik += KB;
+    if (ik == ell) {
       ik = 0;
       ++iw;
       src += to_next;
@@ -254,13 +263,13 @@ __global__ void __launch_bounds__(kEncThreads, DR == 32 ? 3 : 4)
         src = G + c;
       }
     } else {
-      src += L;
+      src += (size_t)KB * L;
     }
-    slot = (slot + 1) & (kEncStages - 1);
+    slot = (slot + 1) & (NST - 1);
   };
-  for (int q = 0; q < kEncStages - 1; ++q) issue();
-  const float* rd = s_ring + threadIdx.x * V;  // this thread's slot 0
-  int rs = 0;  // ring slot of the step being consumed
+  for (int q = 0; q < NST - 1; ++q) issue();
+  const float* rd = s_ring + threadIdx.x * V;  // this thread's block 0 of stage 0
+  int rs = 0;  // ring stage of the step being consumed
   // accumulators paired by ring slot: acc[r][v] = (slot 2r, slot 2r + 1) of
   // column v; one packed two-wide FMA (__ffma2_rn, the same rounding as two
   // fmaf) per pair
@@ -280,33 +289,37 @@ __global__ void __launch_bounds__(kEncThreads, DR == 32 ? 3 : 4)
   for (int w = 0; w < W; ++w) {
     {
       const float* ek = ecol;
-      for (int kk = 0; kk < ell; ++kk, ek += kstride) {
+      for (int kk = 0; kk < ell; kk += KB) {
         issue();
-        cp_async_wait<kEncStages - 1>();  // this step's copy has landed
-        float g[V];
-        const float* gp = rd + rs * (kEncThreads * V);
-        if (V == 4) {
-          const float4 q = *reinterpret_cast<const float4*>(gp);
-          g[0] = q.x;
-          g[1 % V] = q.y;
-          g[2 % V] = q.z;
-          g[3 % V] = q.w;
-        } else {
-          const float2 q = *reinterpret_cast<const float2*>(gp);
-          g[0] = q.x;
-          g[1 % V] = q.y;
-        }
-        rs = (rs + 1) & (kEncStages - 1);
-        const float4* e4 = reinterpret_cast<const float4*>(ek);
+        cp_async_wait<NST - 1>();  // this step's copies have landed
+        const float* gs = rd + rs * (kEncThreads * V * KB);
+        rs = (rs + 1) & (NST - 1);
 #pragma unroll
-        for (int q = 0; q < DR / 4; ++q) {
-          const float4 e = e4[q];
-          const float2 lo = make_float2(e.x, e.y), hi = make_float2(e.z, e.w);
+        for (int kb = 0; kb < KB; ++kb, ek += kstride) {
+          float g[V];
+          const float* gp = gs + kb * (kEncThreads * V);
+          if (V == 4) {
+            const float4 q = *reinterpret_cast<const float4*>(gp);
+            g[0] = q.x;
+            g[1 % V] = q.y;
+            g[2 % V] = q.z;
+            g[3 % V] = q.w;
+          } else {
+            const float2 q = *reinterpret_cast<const float2*>(gp);
+            g[0] = q.x;
+            g[1 % V] = q.y;
+          }
+          const float4* e4 = reinterpret_cast<const float4*>(ek);
 #pragma unroll
-          for (int v = 0; v < V; ++v) {
-            const float2 gg = make_float2(g[v], g[v]);
-            acc[2 * q][v] = __ffma2_rn(lo, gg, acc[2 * q][v]);
-            acc[2 * q + 1][v] = __ffma2_rn(hi, gg, acc[2 * q + 1][v]);
+          for (int q = 0; q < DR / 4; ++q) {
+            const float4 e = e4[q];
+            const float2 lo = make_float2(e.x, e.y), hi = make_float2(e.z, e.w);
+#pragma unroll
+            for (int v = 0; v < V; ++v) {
+              const float2 gg = make_float2(g[v], g[v]);
+              acc[2 * q][v] = __ffma2_rn(lo, gg, acc[2 * q][v]);
+              acc[2 * q + 1][v] = __ffma2_rn(hi, gg, acc[2 * q + 1][v]);
+            }
           }
         }
       }
@@ -323,18 +336,18 @@ __global__ void __launch_bounds__(kEncThreads, DR == 32 ? 3 : 4)
   cp_async_wait<0>();  // no copy outlives the block
 }
 
-template <int DR, int V>
+template <int DR, int V, int KB>
 static int launch_enc_t(dim3 grid, size_t smem, const double* E, const int32_t* order,
                         const int32_t* psi, int N, int m, int delta, int ell, int npat,
                         const float* G, int d, int L, int J, int vec, float* T, cudaStream_t s) {
   static bool attr = false;
   if (!attr) {
-    cudaError_t e = cudaFuncSetAttribute(k_encode<DR, V>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    cudaError_t e = cudaFuncSetAttribute(k_encode<DR, V, KB>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          (int)((kEncSmemFloats + kEncStages * kEncThreads * V) * sizeof(float)));
     if (e != cudaSuccess) return cuda_check(e, "cudaFuncSetAttribute(k_encode)");
     attr = true;
   }
-  k_encode<DR, V><<<grid, kEncThreads, smem, s>>>(E, order, psi, N, m, delta, ell, npat, G, d, L, J, vec, T);
+  k_encode<DR, V, KB><<<grid, kEncThreads, smem, s>>>(E, order, psi, N, m, delta, ell, npat, G, d, L, J, vec, T);
   return GC_OK;
 }
 
@@ -363,8 +376,11 @@ int launch_encode(const double* E, const int32_t* order, const int32_t* psi, int
   const size_t smem = enc_smem_bytes(DR, V, ell, delta, J);
   const dim3 grid((unsigned)npat, (unsigned)stripes, (unsigned)ngroups);
   int rc;
-#define GC_ENC(R, VV) \
-  rc = launch_enc_t<R, VV>(grid, smem, E, order, psi, N, m, delta, ell, npat, G, d, L, J, vec, T, s)
+  // two blocks of a chunk per step when ell is even
+#define GC_ENC(R, VV)                                                                               \
+  rc = ell % 2 == 0                                                                                 \
+           ? launch_enc_t<R, VV, 2>(grid, smem, E, order, psi, N, m, delta, ell, npat, G, d, L, J, vec, T, s) \
+           : launch_enc_t<R, VV, 1>(grid, smem, E, order, psi, N, m, delta, ell, npat, G, d, L, J, vec, T, s)
   switch (DR) {
     case 4: GC_ENC(4, 4); break;
     case 8: GC_ENC(8, 4); break;

@@ -330,17 +330,19 @@ def test_encode_long_rows(gc, explicit, npat):
             assert float(T[b].abs().max()) == 0.0
 
 
-@pytest.mark.parametrize("delta,d", [(5, 2600), (9, 2599), (16, 2600), (16, 2599), (17, 2600), (32, 2600)])
-def test_encode_ring_sizes(gc, delta, d):
+@pytest.mark.parametrize("delta,d,ell", [(5, 2600, 2), (9, 2599, 2), (16, 2600, 2), (16, 2599, 2),
+                                         (17, 2600, 2), (32, 2600, 2), (16, 2600, 1), (16, 2600, 3),
+                                         (16, 2604, 4), (16, 2601, 4)])
+def test_encode_ring_sizes(gc, delta, d, ell):
     """Eq. (2) through every ring size of the chunk sweep (8, 16 and 32
-    slots, with delta below and at the ring size), on three column stripes
-    with a ragged last one (L = 1300), 16-byte vectors (d = 2600) and scalar
-    columns with a padded last block (d = 2599); the patterns include every
-    worker done, none done, and mixed.  Few patterns, so the launch also
-    splits the workers into groups (each group sweeps its own chunks)."""
-    rng = np.random.default_rng(700 + delta + d)
+    slots, with delta below and at the ring size), with one block of a chunk
+    per step (l odd) and two (l even), on column stripes with a ragged last
+    one (L = 1300 at l = 2), 16-byte vectors (d = 2600, 2604) and scalar
+    columns with padded last blocks (d = 2599, 2601); the patterns include
+    every worker done, none done, and mixed.  Few patterns, so the launch
+    also splits the workers into groups (each group sweeps its own chunks)."""
+    rng = np.random.default_rng(700 + delta + d + 10 * ell)
     N = m = 40
-    ell = 2
     order = O.cyclic_order(N, m, delta)
     R = rng.standard_normal((ell, m))
     psi = rng.integers(0, delta + 1, size=(4, m)).astype(np.int32)
@@ -354,7 +356,7 @@ def test_encode_ring_sizes(gc, delta, d):
     for b in range(psi.shape[0]):
         r = O.run_pattern(R, order, psi[b], N, G64, want_transmit=True)
         if np.max(np.abs(r.T)) > 0:
-            assert rel_inf(T[b], r.T) <= 1e-4, f"delta={delta} d={d} pattern {b}"
+            assert rel_inf(T[b], r.T) <= 1e-4, f"delta={delta} d={d} l={ell} pattern {b}"
         else:
             assert float(np.abs(T[b]).max()) == 0.0
 
