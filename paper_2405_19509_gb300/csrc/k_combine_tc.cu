@@ -568,7 +568,36 @@ __global__ void k_mse_reduce_tiles(const float* __restrict__ msep, int parts,
       }
     }
     float s = 0.f;
-    for (int t = lane; t < n; t += 32) s += __ldg(r + t);
+    if (n % 4 == 0 && (reinterpret_cast<uintptr_t>(r) & 15) == 0) {
+      // 16-byte loads, four in flight a lane (a row has up to a few thousand partials)
+      const float4* r4 = reinterpret_cast<const float4*>(r);
+      const int n4 = n / 4;
+      float4 a[4];
+#pragma unroll
+      for (int u = 0; u < 4; ++u) a[u] = make_float4(0.f, 0.f, 0.f, 0.f);
+      int t = lane;
+      for (; t + 96 < n4; t += 128) {
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+          const float4 x = __ldg(r4 + t + 32 * u);
+          a[u].x += x.x;
+          a[u].y += x.y;
+          a[u].z += x.z;
+          a[u].w += x.w;
+        }
+      }
+      for (; t < n4; t += 32) {
+        const float4 x = __ldg(r4 + t);
+        a[0].x += x.x;
+        a[0].y += x.y;
+        a[0].z += x.z;
+        a[0].w += x.w;
+      }
+#pragma unroll
+      for (int u = 0; u < 4; ++u) s += (a[u].x + a[u].y) + (a[u].z + a[u].w);
+    } else {
+      for (int t = lane; t < n; t += 32) s += __ldg(r + t);
+    }
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
     tot += s;

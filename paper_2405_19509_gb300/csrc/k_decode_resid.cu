@@ -88,6 +88,9 @@ template <int ELL>
 __global__ void __launch_bounds__(kScanThreads) k_plan_scan(const __nv_bfloat16* __restrict__ Cs, int Kp,
                                                    int N, int npat, int budget, int policy,
                                                    ResidLists rl, unsigned int* done_counter) {
+  // the sum of the chunk gradients (next in the stream) does not read the
+  // lists: let it start now
+  if (threadIdx.x == 0) asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   const int mt = blockIdx.x;
   const long long M = (long long)npat * ELL;
   const long long row0 = (long long)mt * 128;
@@ -206,8 +209,8 @@ __global__ void __launch_bounds__(kScanThreads) k_plan_scan(const __nv_bfloat16*
 // ---------------------------------------------------------------------------
 // s = sum_i g_{D_i} (chunks added in order 0..N-1).
 // ---------------------------------------------------------------------------
-__global__ void __launch_bounds__(128) k_gsum(const float* __restrict__ G, int N, int d, int vec,
-                                              float* __restrict__ gsum) {
+__device__ __forceinline__ void gsum_cols(const float* __restrict__ G, int N, int d, int vec,
+                                          float* __restrict__ gsum) {
   const long long c0 = ((long long)blockIdx.x * blockDim.x + threadIdx.x) * 4;
   if (c0 >= d) return;
   if (vec) {
@@ -243,6 +246,17 @@ __global__ void __launch_bounds__(128) k_gsum(const float* __restrict__ G, int N
       gsum[c] = acc;
     }
   }
+}
+
+// Launched as a programmatic dependent of the plan scan, which it does not
+// read: the two run side by side.  It waits for the scan before it exits, so
+// that work ordered after it (the residual decode, which reads both) finds
+// the scan complete.
+__global__ void __launch_bounds__(128) k_gsum(const float* __restrict__ G, int N, int d, int vec,
+                                              float* __restrict__ gsum) {
+  gsum_cols(G, N, d, vec, gsum);
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+  asm volatile("griddepcontrol.wait;" ::: "memory");
 }
 
 // ---------------------------------------------------------------------------
@@ -329,6 +343,9 @@ __global__ void __launch_bounds__(kResidThreads, ELL <= 4 ? 4 : 2) k_decode_resi
                                                                 ResidLists rl, int npat, int d,
                                                                 int L, int vec,
                                                                 float* __restrict__ Ghat) {
+  // a programmatic dependent of the sum of the chunk gradients: s and the
+  // scan's lists are complete once this wait returns
+  asm volatile("griddepcontrol.wait;" ::: "memory");
   const int mt = blockIdx.x;
   if (__ldg(rl.tflag + mt)) return;  // the GEMM writes this tile
   const int cnt = __ldg(rl.tcount + mt);
@@ -408,9 +425,19 @@ int launch_gsum(const float* G, int N, int d, float* gsum, cudaStream_t s) {
   const bool vec = d % 4 == 0 && reinterpret_cast<uintptr_t>(G) % 16 == 0 &&
                    reinterpret_cast<uintptr_t>(gsum) % 16 == 0;
   const long long quads = ((long long)d + 3) / 4;
-  k_gsum<<<(unsigned)((quads + 127) / 128), 128, 0, s>>>(G, N, d, vec ? 1 : 0, gsum);
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = dim3((unsigned)((quads + 127) / 128));
+  cfg.blockDim = dim3(128);
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  cudaError_t e = cudaLaunchKernelEx(&cfg, k_gsum, G, N, d, vec ? 1 : 0, gsum);
+  if (e != cudaSuccess) return cuda_check(e, "cudaLaunchKernelEx(k_gsum)");
   count_launches(1);
-  return cuda_check(cudaGetLastError(), "k_gsum");
+  return GC_OK;
 }
 
 int launch_decode_resid(const float* G, const float* gsum, const ResidLists& rl, int ell, int npat,
@@ -429,8 +456,19 @@ int launch_decode_resid(const float* G, const float* gsum, const ResidLists& rl,
   int slices = 1;
   while (slices < 8 && nmt * nranges * slices < 16LL * device_sm_count()) slices *= 2;
   dim3 grid((unsigned)nmt, (unsigned)nranges, (unsigned)slices);
+  // a programmatic dependent of k_gsum (the launch overlaps its tail)
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = grid;
+  cfg.blockDim = dim3(kResidThreads);
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  cudaError_t e = cudaSuccess;
 #define GC_RESID(E) \
-  case E: k_decode_resid<E><<<grid, kResidThreads, 0, s>>>(G, gsum, rl, npat, d, L, vec ? 1 : 0, Ghat); break;
+  case E: e = cudaLaunchKernelEx(&cfg, k_decode_resid<E>, G, gsum, rl, npat, d, L, vec ? 1 : 0, Ghat); break;
   switch (ell) {
     GC_RESID(1)
     GC_RESID(2)
@@ -443,8 +481,9 @@ int launch_decode_resid(const float* G, const float* gsum, const ResidLists& rl,
     default: return fail(GC_ERR_UNSUPPORTED, "ell=%d exceeds GC_MAX_ELL", ell);
   }
 #undef GC_RESID
+  if (e != cudaSuccess) return cuda_check(e, "cudaLaunchKernelEx(k_decode_resid)");
   count_launches(1);
-  return cuda_check(cudaGetLastError(), "k_decode_resid");
+  return GC_OK;
 }
 
 }  // namespace gc
