@@ -28,6 +28,7 @@
 
 #include <algorithm>
 #include <mutex>
+#include <type_traits>
 
 #include "gc_internal.cuh"
 
@@ -240,7 +241,7 @@ struct Ring {
 
 // NT consumer threads (warps 0 .. NW-1) plus one producer warp (warp NW).
 template <typename T, int CL, int NT, int NVT, int RBM>
-__global__ void __launch_bounds__(NT + 32, 1) k_chunkgrad(CGArgs a) {
+__device__ __forceinline__ void chunkgrad_body(const CGArgs& a) {
   constexpr int V = Vec<T>::V;
   constexpr int NW = NT / 32;
   extern __shared__ __align__(128) unsigned char smem[];
@@ -569,6 +570,11 @@ __global__ void __launch_bounds__(NT + 32, 1) k_chunkgrad(CGArgs a) {
   if (CL > 1) cluster_sync_all();  // no CTA leaves while a peer may still address it
 }
 
+template <typename T, int CL, int NT, int NVT, int RBM>
+__global__ void __launch_bounds__(NT + 32, 1) k_chunkgrad(CGArgs a) {
+  chunkgrad_body<T, CL, NT, NVT, RBM>(a);
+}
+
 // G[i][col] = sum of the partials of chunk i, clusters in increasing order.
 // Block (x, i): chunk i, columns [x*256, (x+1)*256), one column per thread;
 // the contributing clusters and their slot offsets are computed once per
@@ -656,19 +662,25 @@ Plan make_plan(int N, int n_c, int d, int x_dtype, bool tma_ok) {
   // 32 KB slices in clusters of 4 (each thread then holds 32 columns; measured
   // 12% faster at d = 65536 than 16 KB slices in clusters of 8).
   if (x_dtype == GC_BF16 && p.CL == 8 && row_bytes <= 4 * 32768) p.CL = 4;
+  // fp32 rows of up to 256 KB take 64 KB slices in clusters of 4 (144 SMs
+  // instead of 120), rows of up to 512 KB 64 KB slices in clusters of 8;
+  // each thread then holds 32 columns, one row a stage
+  if (x_dtype != GC_BF16 && p.CL == 8 && row_bytes <= 4 * 65536) p.CL = 4;
   p.use_tma = tma_ok && (row_bytes % 16 == 0) && (d % (p.CL * p.V) == 0);
   p.Wc = p.use_tma ? d / p.CL : (int)align_up((size_t)((d + p.CL - 1) / p.CL), (size_t)p.V);
   const int nv = p.Wc / p.V;  // 16-byte vectors per row slice (<= 2048 by the slice caps)
   p.NT = nv >= 1024 ? 512 : (nv >= 256 ? 256 : 128);
   if (cps == 2 && p.NT == 512) p.NT = 256;  // only when nv <= 1024 (16 KB slices)
   const int need = (nv + p.NT - 1) / p.NT;
-  p.NVT = need <= 1 ? 1 : (need <= 2 ? 2 : 4);
+  p.NVT = need <= 1 ? 1 : (need <= 2 ? 2 : (need <= 4 ? 4 : 8));
   // every vector of the slice has a thread, and (NT, NVT) is an instantiated shape:
-  // NT = 128 with NVT <= 2, NT = 256 or 512 with NVT <= 4
-  p.valid = (long long)p.NVT * p.NT >= nv && (p.NT > 128 || p.NVT <= 2);
+  // NT = 128 with NVT <= 2, NT = 256 or 512 with NVT <= 4, and fp32 in
+  // clusters of 4 or 8 with NT = 512, NVT = 8
+  p.valid = (long long)p.NVT * p.NT >= nv && (p.NT > 128 || p.NVT <= 2) &&
+            (p.NVT < 8 || (x_dtype != GC_BF16 && p.NT == 512 && p.CL >= 4));
   // stage row stride: one vector per (thread, u), so reads need no bounds
   p.ld_s = p.NVT * p.NT * p.V;
-  p.RBM = p.NVT >= 4 ? 2 : 4;
+  p.RBM = p.NVT >= 8 ? 1 : (p.NVT >= 4 ? 2 : 4);
   p.RB = p.RBM;
   while (p.RB > 1 && n_c % p.RB != 0) p.RB /= 2;
   const size_t stage_bytes = (size_t)p.RBM * p.ld_s * esz;
@@ -721,6 +733,10 @@ int launch_one(const Plan& p, const CGArgs& a, cudaStream_t s) {
 template <typename T, int CL>
 int dispatch_nt(const Plan& p, const CGArgs& a, cudaStream_t s) {
   if (p.NT == 512) {
+    if (p.NVT == 8) {
+      if constexpr (std::is_same<T, float>::value && CL >= 4) return launch_one<T, CL, 512, 8, 1>(p, a, s);
+      return fail(GC_ERR_UNSUPPORTED, "chunk-gradient shape not built");
+    }
     if (p.NVT == 4) return launch_one<T, CL, 512, 4, 2>(p, a, s);
     if (p.NVT == 2) return launch_one<T, CL, 512, 2, 4>(p, a, s);
     return launch_one<T, CL, 512, 1, 4>(p, a, s);
@@ -771,6 +787,10 @@ int occ_one(const Plan& p) {
 template <typename T, int CL>
 int occ_nt(const Plan& p) {
   if (p.NT == 512) {
+    if (p.NVT == 8) {
+      if constexpr (std::is_same<T, float>::value && CL >= 4) return occ_one<T, CL, 512, 8, 1>(p);
+      return 1;
+    }
     if (p.NVT == 4) return occ_one<T, CL, 512, 4, 2>(p);
     if (p.NVT == 2) return occ_one<T, CL, 512, 2, 4>(p);
     return occ_one<T, CL, 512, 1, 4>(p);
@@ -793,10 +813,10 @@ int occ_cl(const Plan& p) {
 }
 // Clusters of this plan that can be resident at once (cached per shape).
 int max_active_clusters(const Plan& p, int x_dtype) {
-  static int cache[2][4][3][3] = {};
+  static int cache[2][4][3][4] = {};
   const int ci = p.CL == 2 ? 1 : (p.CL == 4 ? 2 : 3);
   const int ni = p.NT == 512 ? 0 : (p.NT == 256 ? 1 : 2);
-  const int vi = p.NVT == 4 ? 0 : (p.NVT == 2 ? 1 : 2);
+  const int vi = p.NVT == 8 ? 3 : (p.NVT == 4 ? 0 : (p.NVT == 2 ? 1 : 2));
   int& c = cache[x_dtype == GC_BF16][ci][ni][vi];
   if (c == 0) c = x_dtype == GC_BF16 ? occ_cl<__nv_bfloat16>(p) : occ_cl<float>(p);
   return c;

@@ -188,7 +188,9 @@ def test_large_ell_and_explicit_uneven(gc):
     (4096, 16, 2, torch.float32, 1),     # one CTA per row
     (16384, 8, 3, torch.float32, 0),     # cluster of 2
     (32768, 4, 2, torch.float32, 1),     # cluster of 4
-    (65536, 4, 2, torch.float32, 0),     # cluster of 8
+    (65536, 4, 2, torch.float32, 0),     # cluster of 4 with 64 KB slices (8 vectors a thread)
+    (40000, 3, 2, torch.float32, 1),     # cluster of 4, 8-vector threads partly past the slice
+    (40001, 2, 2, torch.float32, 0),     # the same without TMA (row not a 16-byte multiple)
     (65536, 8, 2, torch.bfloat16, 0),    # bf16, cluster of 4 with 32 KB slices
     (131072, 2, 2, torch.bfloat16, 1),   # bf16, cluster of 8 with 32 KB slices
     (16384, 3, 3, torch.float32, 1),     # cluster of 2, one row per stage (3 rows a chunk)
