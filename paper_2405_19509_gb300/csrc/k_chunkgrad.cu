@@ -332,21 +332,28 @@ __device__ __forceinline__ void chunkgrad_body(const CGArgs& a) {
     }
   } else {
     // ------------------------------------------------------------ consumer warps
-    float wv[NVT][V];
+    // w and the gradient accumulators as column pairs: the passes use packed
+    // two-wide FMAs (__ffma2_rn, the rounding of two fmaf)
+    constexpr int V2 = V / 2;
+    float2 wv[NVT][V2];
 #pragma unroll
     for (int u = 0; u < NVT; ++u) {
       const int v = tid + u * NT;
 #pragma unroll
       for (int e = 0; e < V; ++e) {
         const int col = c0 + v * V + e;
-        wv[u][e] = (v < nvs && col < a.d) ? a.w[col] : 0.f;
+        const float wc = (v < nvs && col < a.d) ? a.w[col] : 0.f;
+        if (e & 1)
+          wv[u][e >> 1].y = wc;
+        else
+          wv[u][e >> 1].x = wc;
       }
     }
-    float acc[NVT][V];
+    float2 acc[NVT][V2];
 #pragma unroll
     for (int u = 0; u < NVT; ++u)
 #pragma unroll
-      for (int e = 0; e < V; ++e) acc[u][e] = 0.f;
+      for (int e = 0; e < V2; ++e) acc[u][e] = make_float2(0.f, 0.f);
     const long long first_chunk = r0 / a.n_c;
     long long cur = -1;     // chunk whose gradient acc holds
     long long next_row = r0;  // first row past chunk `cur` (a batch never straddles chunks: RB | n_c)
@@ -360,7 +367,7 @@ __device__ __forceinline__ void chunkgrad_body(const CGArgs& a) {
 #pragma unroll
           for (int e = 0; e < V; ++e) {
             const int col = c0 + v * V + e;
-            if (col < a.d) dst[col] = acc[u][e];
+            if (col < a.d) dst[col] = (e & 1) ? acc[u][e >> 1].y : acc[u][e >> 1].x;
           }
         }
       }
@@ -393,17 +400,21 @@ __device__ __forceinline__ void chunkgrad_body(const CGArgs& a) {
     // lane-parallel over (warp, row) pairs) and, with clusters, sent to every
     // peer.  Returns the CTA sums in every lane.
     auto dots = [&](int n, auto&& xget, float (&z)[RBM]) {
+      // two packed partial sums a row (vectors u even / odd), so that the
+      // FMA chain of a row is a quarter as long
       float pd[RBM];
 #pragma unroll
       for (int r = 0; r < RBM; ++r) {
-        pd[r] = 0.f;
+        float2 p2[2] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
 #pragma unroll
         for (int u = 0; u < NVT; ++u) {
           float x[V];
           Vec<T>::unpack(xget(r, u), x);
 #pragma unroll
-          for (int e = 0; e < V; ++e) pd[r] = fmaf(x[e], wv[u][e], pd[r]);
+          for (int e = 0; e < V2; ++e)
+            p2[u & 1] = __ffma2_rn(make_float2(x[2 * e], x[2 * e + 1]), wv[u][e], p2[u & 1]);
         }
+        pd[r] = (p2[0].x + p2[0].y) + (p2[1].x + p2[1].y);
       }
       constexpr int kRowShift = 5 - (RBM >= 4 ? 2 : (RBM >= 2 ? 1 : 0));
       const float ws_ = warp_sum_rows<RBM>(pd, lane);
@@ -464,7 +475,7 @@ __device__ __forceinline__ void chunkgrad_body(const CGArgs& a) {
 #pragma unroll
         for (int u = 0; u < NVT; ++u)
 #pragma unroll
-          for (int e = 0; e < V; ++e) acc[u][e] = 0.f;
+          for (int e = 0; e < V2; ++e) acc[u][e] = make_float2(0.f, 0.f);
         cur = cur < 0 ? first_chunk : cur + 1;
         next_row = (cur + 1) * a.n_c;
       }
@@ -504,12 +515,14 @@ __device__ __forceinline__ void chunkgrad_body(const CGArgs& a) {
       // ---- pass 2
 #pragma unroll
       for (int r = 0; r < RBM; ++r) {
+        const float2 rr = make_float2(res[r], res[r]);
 #pragma unroll
         for (int u = 0; u < NVT; ++u) {
           float x[V];
           Vec<T>::unpack(xget(r, u), x);
 #pragma unroll
-          for (int e = 0; e < V; ++e) acc[u][e] = fmaf(res[r], x[e], acc[u][e]);
+          for (int e = 0; e < V2; ++e)
+            acc[u][e] = __ffma2_rn(rr, make_float2(x[2 * e], x[2 * e + 1]), acc[u][e]);
         }
       }
     };
