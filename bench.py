@@ -705,20 +705,21 @@ def logistic_arm(args, rank, world, local_rank):
     psi_all = torch.from_numpy(psi_host).to(dev)
     live_all = torch.from_numpy(live_host).to(dev)
     # static buffers
-    # step inputs and per-step results are double-buffered (index t % 2) so
-    # that step t + 1's inputs are copied in, and step t - 1's results out,
+    # step inputs and per-step results are triple-buffered (index t % NB) so
+    # that step t + 1's inputs are copied in, and earlier steps' results out,
     # on a copy stream while step t runs
-    psi_b = [torch.empty(npat, m, dtype=torch.int32, device=dev) for _ in range(2)]
-    live_b = [torch.empty(1, m, dtype=torch.int32, device=dev) for _ in range(2)]
-    loss_b = [torch.zeros(1, dtype=torch.float64, device=dev) for _ in range(2)]
-    ce_b = [torch.empty(npat, dtype=torch.float64, device=dev) for _ in range(2)]
-    est_b = [torch.empty(npat, dtype=torch.float64, device=dev) for _ in range(2)]
-    mse_b = [torch.empty(npat, dtype=torch.float64, device=dev) for _ in range(2)]
-    # the chunk gradients and the decode plan are double-buffered too: the
+    NB = 3
+    psi_b = [torch.empty(npat, m, dtype=torch.int32, device=dev) for _ in range(NB)]
+    live_b = [torch.empty(1, m, dtype=torch.int32, device=dev) for _ in range(NB)]
+    loss_b = [torch.zeros(1, dtype=torch.float64, device=dev) for _ in range(NB)]
+    ce_b = [torch.empty(npat, dtype=torch.float64, device=dev) for _ in range(NB)]
+    est_b = [torch.empty(npat, dtype=torch.float64, device=dev) for _ in range(NB)]
+    mse_b = [torch.empty(npat, dtype=torch.float64, device=dev) for _ in range(NB)]
+    # the chunk gradients and the decode plan are triple-buffered too: the
     # batched decode of step t reads them while step t + 1 computes its own
-    G_b = [torch.empty(N, d, dtype=torch.float32, device=dev) for _ in range(2)]
+    G_b = [torch.empty(N, d, dtype=torch.float32, device=dev) for _ in range(NB)]
     plan_b = [torch.empty(int(gc.lib.gc_decode_plan_bytes(N, ell, npat)), dtype=torch.uint8, device=dev)
-              for _ in range(2)]
+              for _ in range(NB)]
     Gh_s = torch.empty(npat, d, dtype=torch.float32, device=dev)
     T_s = torch.empty(1, m, L, dtype=torch.float32, device=dev)
     E_s = torch.empty(1, m, delta, ell, dtype=torch.float64, device=dev)
@@ -746,10 +747,9 @@ def logistic_arm(args, rank, world, local_rank):
         gc.gc_find_encoding_coeff(Rd, ell, od, N, m, delta, live_b[bi[0]], E=E_s, C=False,
                                   delta_out=False, support=False, coef_err=False, est=False, ws=wsD)
 
-    def stage_d2():  # eq. (2) encode, PS decode, update
-        gc.gc_encode_with_coeffs(E_s, ell, od, N, m, delta, live_b[bi[0]], G_b[bi[0]], T=T_s)
-        gc.gc_decode_tx(Rd, ell, m, T_s, d, ghat=gh_s)
-        gc.gc_sgd_step(w, gh_s[0], cfg.lr, cfg.Ntil)
+    def stage_d2():  # eq. (2) encode, PS decode, update: one launch
+        gc.gc_live_step(E_s, Rd, ell, od, N, m, delta, live_b[bi[0]], G_b[bi[0]], w, cfg.lr,
+                        cfg.Ntil, T=T_s, ghat=gh_s)
 
     stages = [stage_a, stage_b, stage_c, stage_d1, stage_d2]
     # eager run: allocates workspaces, checks the device status words
@@ -760,15 +760,30 @@ def logistic_arm(args, rank, world, local_rank):
     for ws in (wsA, wsB, wsC, wsD):
         gc.gc_status(ws)
     torch.cuda.synchronize()
-    # serial breakdown (untimed, informational): each stage alone, in order
-    ser_ev = [torch.cuda.Event(enable_timing=True) for _ in range(2 * len(stages))]
-    for rep in range(4):
-        for si, f in enumerate(stages):
-            ser_ev[2 * si].record()
+    # each stage alone (informational, before the timed loop): its own graph
+    # replayed back to back, events on the replay stream; w is restored after
+    # the repeated updates
+    w_saved = w.clone()
+    alone_stream = torch.cuda.Stream(dev)
+    bi[0] = 0
+    alone_ms = []
+    for f in stages:
+        ga_ = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(ga_, stream=alone_stream):
             f()
-            ser_ev[2 * si + 1].record()
+        with torch.cuda.stream(alone_stream):
+            ga_.replay()
+            ea0 = torch.cuda.Event(enable_timing=True)
+            ea1 = torch.cuda.Event(enable_timing=True)
+            ea0.record(alone_stream)
+            for _ in range(10):
+                ga_.replay()
+            ea1.record(alone_stream)
+        torch.cuda.synchronize()
+        alone_ms.append(ea0.elapsed_time(ea1) / 10)
+        del ga_
+    w.copy_(w_saved)
     torch.cuda.synchronize()
-    serial_ms = [ser_ev[2 * si].elapsed_time(ser_ev[2 * si + 1]) for si in range(len(stages))]
 
     # two graphs per step on two streams.  g1 runs the chunk gradients (A)
     # with Algorithm 1 for the live realization (D1) and for the batch (B) on
@@ -776,8 +791,8 @@ def logistic_arm(args, rank, world, local_rank):
     # update (D2), which gives the next step's w.  g2 is the batched decode
     # (C); it needs A and B of its step but nothing of the next one, so it
     # runs on its own stream while g1 of the next step streams X (the chunk
-    # gradients and the plan are double-buffered; a step's g1 waits for the
-    # decode of two steps before, which read its buffers).
+    # gradients and the plan are triple-buffered; a step's g1 waits for the
+    # decode of three steps before, which read its buffers).
     n0 = gc.gc_kernel_launches()
     cap_stream = torch.cuda.Stream(dev)
     cap_hi = [torch.cuda.Stream(dev, priority=-1) for _ in range(2)]
@@ -807,7 +822,7 @@ def logistic_arm(args, rank, world, local_rank):
         return g
 
     g1, g2 = [], []
-    for b in range(2):
+    for b in range(NB):
         bi[0] = b
         g1.append(torch.cuda.CUDAGraph())
         g2.append(torch.cuda.CUDAGraph())
@@ -823,7 +838,7 @@ def logistic_arm(args, rank, world, local_rank):
     # decode-combine call (C) on their own stream inside the graph; NE copies
     # with their own events, cycled, so the last NE instrumented steps each
     # leave a sample
-    EVERY, NE = 8, 8
+    EVERY, NE = 8 * NB, 8
     kev = [[[torch.cuda.Event(enable_timing=True, external=True) for _ in range(2)] for _ in range(2)]
            for _ in range(NE)]
     g1i, g2i = [], []
@@ -838,14 +853,19 @@ def logistic_arm(args, rank, world, local_rank):
             timed(stage_c, kev[j][1])()
     torch.cuda.synchronize()
 
-    stream = torch.cuda.current_stream(dev)
-    dec_stream = torch.cuda.Stream(dev)  # the batched decode (g2)
+    # g1 (the chunk gradients and the update: the step's critical path) on a
+    # high-priority stream, g2 (the batched decode) on a low-priority one:
+    # when SMs free up the block scheduler takes g1's blocks first, so the
+    # decode's many small blocks do not hold the chunk-gradient kernel (one
+    # block per SM) back
+    stream = torch.cuda.Stream(dev, priority=-1)
+    dec_stream = torch.cuda.Stream(dev, priority=0)  # the batched decode (g2)
 
     copy_stream = torch.cuda.Stream(dev)
-    ev_ready = [torch.cuda.Event() for _ in range(2)]  # inputs of the buffer's next step are in
-    ev_g1 = [torch.cuda.Event() for _ in range(2)]     # the buffer's g1 has finished
-    ev_done = [torch.cuda.Event() for _ in range(2)]   # the buffer's step (g1 and g2) has finished
-    ev_out = [torch.cuda.Event() for _ in range(2)]    # the buffer's results have been read out
+    ev_ready = [torch.cuda.Event() for _ in range(NB)]  # inputs of the buffer's next step are in
+    ev_g1 = [torch.cuda.Event() for _ in range(NB)]     # the buffer's g1 has finished
+    ev_done = [torch.cuda.Event() for _ in range(NB)]   # the buffer's step (g1 and g2) has finished
+    ev_out = [torch.cuda.Event() for _ in range(NB)]    # the buffer's results have been read out
 
     def put_inputs(t, b, src):
         """Copy step t's realizations into buffer b on the copy stream, once
@@ -857,13 +877,13 @@ def logistic_arm(args, rank, world, local_rank):
             ev_ready[b].record(copy_stream)
 
     def run_step(k, t, t_next, src, evs=None, outs=None):
-        """Step k on realization batch t (buffer k % 2, whose inputs are
+        """Step k on realization batch t (buffer k % NB, whose inputs are
         already being copied in); queues the copy of batch t_next into the
         other buffer, runs g1 and g2 and, with `outs`, copies the step's
         results to host memory on the copy stream.  With evs (instrumented
         steps, buffer 0) evs[0..3] bracket g1 and g2 and the graphs are the
         instrumented copy (k // EVERY) % NE."""
-        b = k % 2
+        b = k % NB
         ga, gb = g1[b], g2[b]
         if evs is not None:
             assert b == 0
@@ -873,13 +893,14 @@ def logistic_arm(args, rank, world, local_rank):
             if evs is not None:
                 evs[i].record(st)
         if t_next is not None:
-            put_inputs(t_next, 1 - b, src)
+            put_inputs(t_next, (k + 1) % NB, src)
         stream.wait_event(ev_ready[b])
-        stream.wait_event(ev_done[b])  # the decode of step k - 2 has read this buffer's G and plan
-        stream.wait_event(ev_out[b])   # results of step k - 2 have been read out
-        rec(0, stream)
-        ga.replay()
-        rec(1, stream)
+        stream.wait_event(ev_done[b])  # the decode of step k - NB has read this buffer's G and plan
+        stream.wait_event(ev_out[b])   # results of step k - NB have been read out
+        with torch.cuda.stream(stream):  # replay() launches on the current stream
+            rec(0, stream)
+            ga.replay()
+            rec(1, stream)
         ev_g1[b].record(stream)
         dec_stream.wait_event(ev_g1[b])
         with torch.cuda.stream(dec_stream):
@@ -1015,7 +1036,9 @@ def logistic_arm(args, rank, world, local_rank):
                                      "gc_decode_apply": float(alg_bytes[2] / (call_ms[1] / 1e3) / 1e9 / hbm)},
                 "graph_ms": {"g1: k_chunkgrad || Algorithm 1, then live encode/decode/update": float(stage_ms[0]),
                              "g2: batched decode": float(stage_ms[1])},
-                "serial_stage_ms": {n: float(v) for n, v in zip(names, serial_ms)}}
+                "alone_graph_ms": {n: float(v) for n, v in zip(names, alone_ms)},
+                "alone_frac_of_hbm": {names[i]: float(alg_bytes[i] / (alone_ms[i] / 1e3) / 1e9 / hbm)
+                                      for i in (0, 2)}}
 
     line = {
         "metric": METRIC_LOGISTIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K,

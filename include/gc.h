@@ -423,6 +423,29 @@ int gc_mse(const double* R, int ell, const int32_t* order, int N, int m, int del
  */
 int gc_sgd_step(float* w, const float* ghat, int d, float lr, int64_t Ntil, void* stream);
 
+/* ---- one live realization: eq. (2) encode, Sec. II-B decode, Sec. I update --
+ * For one straggler pattern psi (m int32, device) with its coefficients E
+ * (m x delta x ell fp64, gc_find_encoding_coeff), in one kernel:
+ *   T[j][c]       = sum_{p < psi[j]} sum_k E[j][p][k] g_{D_order[j][p]}[k*L + c]   (eq. 2)
+ *   ghat[k*L + c] = sum_j R[k][j] T[j][c]                                         (Sec. II-B)
+ *   w[k*L + c]   -= lr * ghat[k*L + c] / Ntil                                     (Sec. I)
+ * for k*L + c < d, with the same float32 operations in the same order as
+ * gc_encode_with_coeffs, gc_decode_tx and gc_sgd_step, so T, ghat and w
+ * equal theirs bit for bit.  One launch instead of three: the update that
+ * the next step's chunk gradients wait for.
+ *   R      device ell x m fp64.  order device m x delta int32.
+ *   G      device N x d float32 chunk gradients.
+ *   w      device d float32, updated in place.
+ *   T      NULL or device m x L float32 output (the transmissions).
+ *   ghat   NULL or device d float32 output (the decoded gradient).
+ * E, R, the order and psi are staged in shared memory:
+ * (m*delta*ell + ell*m + m*delta + m) * 4 bytes must not exceed 96 KB
+ * (GC_ERR_UNSUPPORTED otherwise).  No workspace.
+ */
+int gc_live_step(const double* E, const double* R, int ell, const int32_t* order, int N, int m,
+                 int delta, const int32_t* psi, const float* G, int d, float lr, int64_t Ntil,
+                 float* w, float* T, float* ghat, void* stream);
+
 #ifdef __cplusplus
 }
 #endif

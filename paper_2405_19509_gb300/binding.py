@@ -77,6 +77,7 @@ _sig("gc_decode_combine", _i, _p, _i, _i, _i, _p, _i, _p, _p, _p, _sz, _p)
 _sig("gc_mse_workspace", _sz, _i, _i, _i, _i, _i, _i)
 _sig("gc_mse", _i, _p, _i, _p, _i, _i, _i, _p, _i, _p, _i, _p, _p, _p, _p, _sz, _p)
 _sig("gc_sgd_step", _i, _p, _p, _i, _f, _i64, _p)
+_sig("gc_live_step", _i, _p, _p, _i, _p, _i, _i, _i, _p, _p, _i, _f, _i64, _p, _p, _p, _p)
 
 
 class GCError(RuntimeError):
@@ -531,4 +532,23 @@ def gc_sgd_step(w, ghat, lr: float, Ntil: int):
     d = w.shape[0]
     _check(lib.gc_sgd_step(_dev(w, torch.float32, "w", (d,)), _dev(ghat, torch.float32, "ghat", (d,)),
                            d, float(lr), int(Ntil), _stream()))
+    return w
+
+
+def gc_live_step(E, R, ell, order, N, m, delta, psi, G, w, lr: float, Ntil: int, T=None, ghat=None):
+    """One live realization in one launch: eq. (2) transmissions, their PS
+    decode and the update of w (in place).  E is the pattern's m x delta x ell
+    float64 coefficients (a 1 x m x delta x ell batch is accepted), psi its m
+    processed counts; T (m x L) and ghat (d) are written when given."""
+    d = G.shape[1]
+    L = block_length(d, ell)
+    _check(lib.gc_live_step(_dev(E.reshape(m, delta, ell), torch.float64, "E", (m, delta, ell)),
+                            _dev(R, torch.float64, "R", (ell, m)), ell,
+                            _dev(order, torch.int32, "order", (m, delta)), N, m, delta,
+                            _dev(psi.reshape(m), torch.int32, "psi", (m,)),
+                            _dev(G, torch.float32, "G", (N, d)), d, float(lr), int(Ntil),
+                            _dev(w, torch.float32, "w", (d,)),
+                            None if T is None else _dev(T.reshape(m, L), torch.float32, "T", (m, L)),
+                            None if ghat is None else _dev(ghat.reshape(d), torch.float32, "ghat", (d,)),
+                            _stream()))
     return w

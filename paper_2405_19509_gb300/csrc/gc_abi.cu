@@ -569,4 +569,17 @@ int gc_sgd_step(float* w, const float* ghat, int d, float lr, int64_t Ntil, void
   return launch_sgd(w, ghat, d, lr, Ntil, as_stream(stream));
 }
 
+int gc_live_step(const double* E, const double* R, int ell, const int32_t* order, int N, int m,
+                 int delta, const int32_t* psi, const float* G, int d, float lr, int64_t Ntil,
+                 float* w, float* T, float* ghat, void* stream) {
+  NvtxRange nvtx_("gc_live_step");
+  int rc = check_dims(N, m, delta, ell, 1);
+  if (rc) return rc;
+  if (d < 1 || Ntil < 1) return fail(GC_ERR_SHAPE, "d and Ntil must be >= 1");
+  if (!E || !R || !order || !psi || !G || !w)
+    return fail(GC_ERR_ARG, "E, R, order, psi, G and w must be non-NULL");
+  return launch_live_step(E, R, ell, order, N, m, delta, psi, G, d, lr, Ntil, w, T, ghat,
+                          as_stream(stream));
+}
+
 }  // extern "C"

@@ -121,6 +121,9 @@ int launch_encode(const double* E, const int32_t* order, const int32_t* psi, int
 int launch_decode_tx(const double* R, int ell, int m, const float* T, int npat, int d, float* ghat,
                      cudaStream_t s);
 int launch_sgd(float* w, const float* ghat, int d, float lr, int64_t Ntil, cudaStream_t s);
+int launch_live_step(const double* E, const double* R, int ell, const int32_t* order, int N, int m,
+                     int delta, const int32_t* psi, const float* G, int d, float lr, int64_t Ntil,
+                     float* w, float* T, float* ghat, cudaStream_t s);
 
 // ---- batched decode in residual form (k_decode_resid.cu) -----------------
 // Per pattern the ordered list of decode blocks that differ from I_ell (chunk

@@ -482,4 +482,141 @@ int launch_sgd(float* w, const float* ghat, int d, float lr, int64_t Ntil, cudaS
   return cuda_check(cudaGetLastError(), "k_sgd");
 }
 
+// One live realization in one pass (eq. 2, Sec. II-B, Sec. I).  Thread c
+// forms T[j][c] for every worker j (slots p ascending, blocks k ascending, as
+// k_encode; the slots past psi_j and the padding past d add zeros there and
+// are skipped here, which leaves every sum unchanged), then
+// ghat[k*L + c] = sum_j R[k][j] T[j][c] (j ascending, as k_decode_tx), then
+// w[k*L + c] -= scale * ghat[k*L + c] (as k_sgd): the same fp32 operations in
+// the same order, so T, ghat and w equal those of the three separate calls.
+// E, R, the order and psi are staged in shared memory, and with SG the
+// block's 64 columns of every chunk block too (all loads in flight at once;
+// the sums then read shared memory instead of a chain of cache loads).
+constexpr int kLiveThreads = 64;
+template <int ELL, bool SG>
+__global__ void __launch_bounds__(kLiveThreads) k_live_step(const double* __restrict__ E,
+                                                  const double* __restrict__ R,
+                                                  const int32_t* __restrict__ order,
+                                                  const int32_t* __restrict__ psi, int N, int m,
+                                                  int delta, const float* __restrict__ G, int d,
+                                                  int L, float scale, float* __restrict__ w,
+                                                  float* __restrict__ T, float* __restrict__ ghat) {
+  extern __shared__ float s_live[];
+  const int ne = m * delta * ELL;
+  float* s_g = s_live;                                  // [N][ELL][kLiveThreads] with SG
+  float* s_e = s_g + (SG ? N * ELL * kLiveThreads : 0); // [m][delta][ELL]
+  float* s_r = s_e + ne;                                // [ELL][m]
+  int* s_ord = reinterpret_cast<int*>(s_r + ELL * m);   // [m][delta]
+  int* s_np = s_ord + m * delta;                        // [m]
+  const int c0 = blockIdx.x * kLiveThreads;
+  if (SG) {
+    for (int t = threadIdx.x; t < N * ELL * kLiveThreads; t += kLiveThreads) {
+      const int row = t / kLiveThreads, cc = c0 + t % kLiveThreads;
+      const int i = row / ELL, k = row - i * ELL;
+      const long long col = (long long)k * L + cc;
+      s_g[t] = (cc < L && col < d) ? __ldg(G + (size_t)i * d + col) : 0.f;
+    }
+  }
+  for (int t = threadIdx.x; t < ne; t += kLiveThreads) s_e[t] = (float)E[t];
+  for (int t = threadIdx.x; t < ELL * m; t += kLiveThreads) s_r[t] = (float)R[t];
+  for (int t = threadIdx.x; t < m * delta; t += kLiveThreads) s_ord[t] = order[t];
+  for (int t = threadIdx.x; t < m; t += kLiveThreads) {
+    const int np = psi[t];
+    s_np[t] = np < 0 ? 0 : (np > delta ? delta : np);  // as the encode: bad values are flagged by the solve
+  }
+  __syncthreads();
+  const int c = c0 + threadIdx.x;
+  if (c >= L) return;
+  float acc[ELL];
+#pragma unroll
+  for (int k = 0; k < ELL; ++k) acc[k] = 0.f;
+  for (int j = 0; j < m; ++j) {
+    float t = 0.f;
+    const int np = s_np[j];
+    for (int p = 0; p < np; ++p) {
+      const int i = s_ord[j * delta + p];
+      if (i < 0 || i >= N) continue;
+      const float* ej = s_e + (j * delta + p) * ELL;
+#pragma unroll
+      for (int k = 0; k < ELL; ++k) {
+        const long long col = (long long)k * L + c;
+        if (col < d) {
+          const float g = SG ? s_g[(i * ELL + k) * kLiveThreads + threadIdx.x] : __ldg(G + (size_t)i * d + col);
+          t = fmaf(ej[k], g, t);
+        }
+      }
+    }
+    if (T) T[(size_t)j * L + c] = t;
+#pragma unroll
+    for (int k = 0; k < ELL; ++k) acc[k] = fmaf(s_r[k * m + j], t, acc[k]);
+  }
+#pragma unroll
+  for (int k = 0; k < ELL; ++k) {
+    const long long col = (long long)k * L + c;
+    if (col < d) {
+      if (ghat) ghat[col] = acc[k];
+      w[col] = fmaf(-scale, acc[k], w[col]);
+    }
+  }
+}
+
+constexpr size_t kLiveSmemMax = 96 * 1024;
+
+template <int ELL, bool SG>
+static cudaError_t launch_live_t(unsigned blocks, size_t smem, const double* E, const double* R,
+                                 const int32_t* order, const int32_t* psi, int N, int m, int delta,
+                                 const float* G, int d, int L, float scale, float* w, float* T,
+                                 float* ghat, cudaStream_t s) {
+  static bool attr = false;
+  if (!attr) {
+    const cudaError_t e = cudaFuncSetAttribute(k_live_step<ELL, SG>,
+                                               cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                               (int)kLiveSmemMax);
+    if (e != cudaSuccess) return e;
+    attr = true;
+  }
+  k_live_step<ELL, SG><<<blocks, kLiveThreads, smem, s>>>(E, R, order, psi, N, m, delta, G, d, L,
+                                                          scale, w, T, ghat);
+  return cudaSuccess;
+}
+
+int launch_live_step(const double* E, const double* R, int ell, const int32_t* order, int N, int m,
+                     int delta, const int32_t* psi, const float* G, int d, float lr, int64_t Ntil,
+                     float* w, float* T, float* ghat, cudaStream_t s) {
+  const int L = (d + ell - 1) / ell;
+  const size_t base = ((size_t)m * delta * ell + (size_t)ell * m) * sizeof(float) +
+                      ((size_t)m * delta + m) * sizeof(int);
+  if (base > kLiveSmemMax)
+    return fail(GC_ERR_UNSUPPORTED, "live step: m*delta*ell=%lld too large to stage",
+                (long long)m * delta * ell);
+  const size_t gbytes = (size_t)N * ell * kLiveThreads * sizeof(float);
+  const bool sg = base + gbytes <= kLiveSmemMax;
+  const size_t smem = base + (sg ? gbytes : 0);
+  const float scale = (float)((double)lr / (double)Ntil);
+  const unsigned blocks = (unsigned)((L + kLiveThreads - 1) / kLiveThreads);
+  cudaError_t e = cudaSuccess;
+#define GC_LIVE(E_)                                                                              \
+  case E_:                                                                                       \
+    e = sg ? launch_live_t<E_, true>(blocks, smem, E, R, order, psi, N, m, delta, G, d, L, scale, \
+                                     w, T, ghat, s)                                              \
+           : launch_live_t<E_, false>(blocks, smem, E, R, order, psi, N, m, delta, G, d, L,      \
+                                      scale, w, T, ghat, s);                                     \
+    break;
+  switch (ell) {
+    GC_LIVE(1)
+    GC_LIVE(2)
+    GC_LIVE(3)
+    GC_LIVE(4)
+    GC_LIVE(5)
+    GC_LIVE(6)
+    GC_LIVE(7)
+    GC_LIVE(8)
+    default: return fail(GC_ERR_UNSUPPORTED, "ell=%d exceeds GC_MAX_ELL", ell);
+  }
+#undef GC_LIVE
+  if (e != cudaSuccess) return cuda_check(e, "cudaFuncSetAttribute(k_live_step)");
+  count_launches(1);
+  return cuda_check(cudaGetLastError(), "k_live_step");
+}
+
 }  // namespace gc

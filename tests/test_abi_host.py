@@ -102,6 +102,15 @@ def test_device_entry_validation_before_launch():
     assert L.gc_decode_tx(q, 9, 6, q, 1, 64, q, None) == -3
     assert L.gc_sgd_step(None, q, 8, ctypes.c_float(0.1), 10, None) == -1
     assert L.gc_sgd_step(ctypes.c_void_p(16), ctypes.c_void_p(16), 0, ctypes.c_float(0.1), 10, None) == -2
+    # the live step: NULL inputs, bad shapes, unsupported ell, staging too large
+    assert L.gc_live_step(None, q, 2, q, 6, 6, 3, q, q, 64, ctypes.c_float(0.1), 10, q, None, None,
+                          None) == -1
+    assert L.gc_live_step(q, q, 2, q, 6, 6, 3, q, q, 0, ctypes.c_float(0.1), 10, q, None, None,
+                          None) == -2
+    assert L.gc_live_step(q, q, 9, q, 6, 6, 3, q, q, 64, ctypes.c_float(0.1), 10, q, None, None,
+                          None) == -3
+    assert L.gc_live_step(q, q, 8, q, 4096, 4096, 32, q, q, 64, ctypes.c_float(0.1), 10, q, None,
+                          None, None) == -3
     # workspace missing / too small / misaligned
     need = L.gc_decode_batch_workspace(6, 6, 3, 2, 4, 64)
     assert need > 256

@@ -363,6 +363,51 @@ def test_encode_ring_sizes(gc, delta, d, ell):
             assert float(np.abs(T[b]).max()) == 0.0
 
 
+@pytest.mark.parametrize("N,m,delta,d,ell,explicit", [
+    (6, 6, 3, 64, 2, False),        # the tiny configuration
+    (20, 20, 4, 4099, 3, False),    # padded last block (3 * 1367 > 4099)
+    (128, 128, 6, 8192, 2, False),  # the coded-SGD shape
+    (12, 6, 2, 130, 2, True),       # explicit, non-cyclic order
+    (40, 40, 16, 1000, 1, False),   # l = 1
+    (256, 256, 16, 2002, 2, False), # N*l too large to stage the columns: chunk gradients read directly
+])
+def test_live_step_matches_three_calls(gc, N, m, delta, d, ell, explicit):
+    """gc_live_step (one launch) gives the same T, ghat and w, bit for bit, as
+    gc_encode_with_coeffs + gc_decode_tx + gc_sgd_step; ghat agrees with the
+    oracle's Sec. II-B decode of the eq. (2) transmissions."""
+    rng = np.random.default_rng(900 + N + d + ell)
+    if explicit:
+        order = rng.permutation(N).astype(np.int32).reshape(m, delta)
+    else:
+        order = O.cyclic_order(N, m, delta)
+    R = rng.standard_normal((ell, m))
+    psi = rng.integers(0, delta + 1, size=(1, m)).astype(np.int32)
+    psi[0, 0] = delta
+    G = rng.standard_normal((N, d)).astype(np.float32)
+    w0 = rng.standard_normal(d).astype(np.float32)
+    Rd, od, pd = dev_tensors(R, order, psi)
+    Gd = torch.from_numpy(G).cuda()
+    E = gc.gc_find_encoding_coeff(Rd, ell, od, N, m, delta, pd, C=False)["E"]
+    lr, Ntil = 0.25, 1000
+    T1 = gc.gc_encode_with_coeffs(E, ell, od, N, m, delta, pd, Gd)
+    gh1 = gc.gc_decode_tx(Rd, ell, m, T1, d)
+    w1 = torch.from_numpy(w0).cuda()
+    gc.gc_sgd_step(w1, gh1[0], lr, Ntil)
+    L = gc.block_length(d, ell)
+    T2 = torch.empty(m, L, dtype=torch.float32, device="cuda")
+    gh2 = torch.empty(d, dtype=torch.float32, device="cuda")
+    w2 = torch.from_numpy(w0).cuda()
+    gc.gc_live_step(E, Rd, ell, od, N, m, delta, pd, Gd, w2, lr, Ntil, T=T2, ghat=gh2)
+    w3 = torch.from_numpy(w0).cuda()
+    gc.gc_live_step(E, Rd, ell, od, N, m, delta, pd, Gd, w3, lr, Ntil)   # no T, no ghat
+    torch.cuda.synchronize()
+    assert torch.equal(T2, T1[0])
+    assert torch.equal(gh2, gh1[0])
+    assert torch.equal(w2, w1) and torch.equal(w3, w1)
+    r = O.run_pattern(R, order, psi[0], N, G.astype(np.float64), want_transmit=True)
+    assert_grad_close(to_np(gh2), r.ghat, "live step ghat")
+
+
 @pytest.mark.parametrize("ell", [1, 3])
 def test_decode_plan_then_apply(gc, ell):
     """gc_decode_plan (psi side) then gc_decode_apply (data side) equals
