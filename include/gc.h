@@ -438,9 +438,9 @@ int gc_sgd_step(float* w, const float* ghat, int d, float lr, int64_t Ntil, void
  *   w      device d float32, updated in place.
  *   T      NULL or device m x L float32 output (the transmissions).
  *   ghat   NULL or device d float32 output (the decoded gradient).
- * E, R, the order and psi are staged in shared memory:
- * (m*delta*ell + ell*m + m*delta + m) * 4 bytes must not exceed 96 KB
- * (GC_ERR_UNSUPPORTED otherwise).  No workspace.
+ * E, R, the order, psi and the transmissions of 32 columns are staged in
+ * shared memory: (m*delta*ell + ell*m + 32*m + m*delta + m) * 4 bytes must
+ * not exceed 96 KB (GC_ERR_UNSUPPORTED otherwise).  No workspace.
  */
 int gc_live_step(const double* E, const double* R, int ell, const int32_t* order, int N, int m,
                  int delta, const int32_t* psi, const float* G, int d, float lr, int64_t Ntil,

@@ -482,17 +482,18 @@ int launch_sgd(float* w, const float* ghat, int d, float lr, int64_t Ntil, cudaS
   return cuda_check(cudaGetLastError(), "k_sgd");
 }
 
-// One live realization in one pass (eq. 2, Sec. II-B, Sec. I).  Thread c
-// forms T[j][c] for every worker j (slots p ascending, blocks k ascending, as
+// One live realization in one pass (eq. 2, Sec. II-B, Sec. I).  A block
+// takes kLiveCols columns c; its warp w forms T[j][c] for the workers
+// j = w, w + kLiveWG, ... (slots p ascending, blocks k ascending, as
 // k_encode; the slots past psi_j and the padding past d add zeros there and
-// are skipped here, which leaves every sum unchanged), then
-// ghat[k*L + c] = sum_j R[k][j] T[j][c] (j ascending, as k_decode_tx), then
-// w[k*L + c] -= scale * ghat[k*L + c] (as k_sgd): the same fp32 operations in
-// the same order, so T, ghat and w equal those of the three separate calls.
-// E, R, the order and psi are staged in shared memory, and with SG the
-// block's 64 columns of every chunk block too (all loads in flight at once;
-// the sums then read shared memory instead of a chain of cache loads).
-constexpr int kLiveThreads = 64;
+// are skipped here, which leaves every sum unchanged) into shared memory;
+// then warp 0 forms ghat[k*L + c] = sum_j R[k][j] T[j][c] (j ascending, as
+// k_decode_tx) and w[k*L + c] -= scale * ghat[k*L + c] (as k_sgd): the same
+// fp32 operations in the same order, so T, ghat and w equal those of the
+// three separate calls.  E, R, the order and psi are staged in shared
+// memory, and with SG the block's columns of every chunk block too (loaded
+// with all the block's loads in flight).
+constexpr int kLiveCols = 32, kLiveWG = 8, kLiveThreads = kLiveCols * kLiveWG;
 template <int ELL, bool SG>
 __global__ void __launch_bounds__(kLiveThreads) k_live_step(const double* __restrict__ E,
                                                   const double* __restrict__ R,
@@ -503,15 +504,18 @@ __global__ void __launch_bounds__(kLiveThreads) k_live_step(const double* __rest
                                                   float* __restrict__ T, float* __restrict__ ghat) {
   extern __shared__ float s_live[];
   const int ne = m * delta * ELL;
-  float* s_g = s_live;                                  // [N][ELL][kLiveThreads] with SG
-  float* s_e = s_g + (SG ? N * ELL * kLiveThreads : 0); // [m][delta][ELL]
+  float* s_g = s_live;                                  // [N][ELL][kLiveCols] with SG
+  float* s_t = s_g + (SG ? N * ELL * kLiveCols : 0);    // [m][kLiveCols]
+  float* s_e = s_t + m * kLiveCols;                     // [m][delta][ELL]
   float* s_r = s_e + ne;                                // [ELL][m]
   int* s_ord = reinterpret_cast<int*>(s_r + ELL * m);   // [m][delta]
   int* s_np = s_ord + m * delta;                        // [m]
-  const int c0 = blockIdx.x * kLiveThreads;
+  const int cl = threadIdx.x % kLiveCols, wg = threadIdx.x / kLiveCols;
+  const int c0 = blockIdx.x * kLiveCols;
   if (SG) {
-    for (int t = threadIdx.x; t < N * ELL * kLiveThreads; t += kLiveThreads) {
-      const int row = t / kLiveThreads, cc = c0 + t % kLiveThreads;
+#pragma unroll 4
+    for (int t = threadIdx.x; t < N * ELL * kLiveCols; t += kLiveThreads) {
+      const int row = t / kLiveCols, cc = c0 + t % kLiveCols;
       const int i = row / ELL, k = row - i * ELL;
       const long long col = (long long)k * L + cc;
       s_g[t] = (cc < L && col < d) ? __ldg(G + (size_t)i * d + col) : 0.f;
@@ -525,12 +529,9 @@ __global__ void __launch_bounds__(kLiveThreads) k_live_step(const double* __rest
     s_np[t] = np < 0 ? 0 : (np > delta ? delta : np);  // as the encode: bad values are flagged by the solve
   }
   __syncthreads();
-  const int c = c0 + threadIdx.x;
-  if (c >= L) return;
-  float acc[ELL];
-#pragma unroll
-  for (int k = 0; k < ELL; ++k) acc[k] = 0.f;
-  for (int j = 0; j < m; ++j) {
+  const int c = c0 + cl;
+  const bool live = c < L;
+  for (int j = wg; j < m; j += kLiveWG) {
     float t = 0.f;
     const int np = s_np[j];
     for (int p = 0; p < np; ++p) {
@@ -540,13 +541,22 @@ __global__ void __launch_bounds__(kLiveThreads) k_live_step(const double* __rest
 #pragma unroll
       for (int k = 0; k < ELL; ++k) {
         const long long col = (long long)k * L + c;
-        if (col < d) {
-          const float g = SG ? s_g[(i * ELL + k) * kLiveThreads + threadIdx.x] : __ldg(G + (size_t)i * d + col);
+        if (live && col < d) {
+          const float g = SG ? s_g[(i * ELL + k) * kLiveCols + cl] : __ldg(G + (size_t)i * d + col);
           t = fmaf(ej[k], g, t);
         }
       }
     }
-    if (T) T[(size_t)j * L + c] = t;
+    s_t[j * kLiveCols + cl] = t;
+    if (T && live) T[(size_t)j * L + c] = t;
+  }
+  __syncthreads();
+  if (wg != 0 || !live) return;
+  float acc[ELL];
+#pragma unroll
+  for (int k = 0; k < ELL; ++k) acc[k] = 0.f;
+  for (int j = 0; j < m; ++j) {
+    const float t = s_t[j * kLiveCols + cl];
 #pragma unroll
     for (int k = 0; k < ELL; ++k) acc[k] = fmaf(s_r[k * m + j], t, acc[k]);
   }
@@ -584,16 +594,16 @@ int launch_live_step(const double* E, const double* R, int ell, const int32_t* o
                      int delta, const int32_t* psi, const float* G, int d, float lr, int64_t Ntil,
                      float* w, float* T, float* ghat, cudaStream_t s) {
   const int L = (d + ell - 1) / ell;
-  const size_t base = ((size_t)m * delta * ell + (size_t)ell * m) * sizeof(float) +
+  const size_t base = ((size_t)m * delta * ell + (size_t)ell * m + (size_t)m * kLiveCols) * sizeof(float) +
                       ((size_t)m * delta + m) * sizeof(int);
   if (base > kLiveSmemMax)
-    return fail(GC_ERR_UNSUPPORTED, "live step: m*delta*ell=%lld too large to stage",
-                (long long)m * delta * ell);
-  const size_t gbytes = (size_t)N * ell * kLiveThreads * sizeof(float);
+    return fail(GC_ERR_UNSUPPORTED, "live step: m=%d, delta=%d, ell=%d too large to stage", m,
+                delta, ell);
+  const size_t gbytes = (size_t)N * ell * kLiveCols * sizeof(float);
   const bool sg = base + gbytes <= kLiveSmemMax;
   const size_t smem = base + (sg ? gbytes : 0);
   const float scale = (float)((double)lr / (double)Ntil);
-  const unsigned blocks = (unsigned)((L + kLiveThreads - 1) / kLiveThreads);
+  const unsigned blocks = (unsigned)((L + kLiveCols - 1) / kLiveCols);
   cudaError_t e = cudaSuccess;
 #define GC_LIVE(E_)                                                                              \
   case E_:                                                                                       \
