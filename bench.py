@@ -257,36 +257,6 @@ def _traffic(kernel, src_files):
     return e.get("dram_bytes_per_launch")
 
 
-def gemm_tile_fraction(psi, order, N, ell, ksp=None, rcap=32):
-    """Share of the decode's 128-row tiles that the library computes on the
-    tensor-core GEMM under its automatic policy (reporting only; the device
-    makes the same choice from the decode plan): a tile stays on the residual
-    path unless one of its patterns has more than ksp blocks with fewer than
-    ell copies, more than rcap of its rows need corrections, or its patterns
-    average more than ceil(N*ell/64) such blocks."""
-    m, delta = order.shape
-    D = np.zeros((psi.shape[0], N), dtype=np.int64)
-    for j in range(m):
-        for p in range(delta):
-            i = order[j, p]
-            if i >= 0:
-                D[:, i] += psi[:, j] > p
-    nnz = (D < ell).sum(axis=1)
-    ksp = ksp or min(N, 32 if ell <= 2 else (16 if ell <= 4 else 8))
-    budget = max(1, -(-N * ell // 64))
-    M = psi.shape[0] * ell
-    row_pat = np.arange(M) // ell
-    dense = 0
-    ntile = (M + 127) // 128
-    for t in range(ntile):
-        rows = np.arange(t * 128, min(M, t * 128 + 128))
-        pats = np.unique(row_pat[rows])
-        corrected = int((nnz[row_pat[rows]] > 0).sum())
-        if np.any(nnz[pats] > ksp) or corrected > rcap or nnz[pats].sum() > budget * len(pats):
-            dense += 1
-    return dense / ntile
-
-
 def oracle_decode_sample(cfg, ell, G32, psi, cols, min_patterns, max_seconds):
     """Time the fp64 oracle on a bounded sample of the decode workload.
 
@@ -1155,30 +1125,47 @@ def extra_workload(args):
         Rd = torch.from_numpy(make_R(cfg, ell)).to(dev)
         od = torch.from_numpy(order).to(dev)
         wsM = gc.Workspace(dev)
+        wsP, wsA2 = gc.Workspace(dev), gc.Workspace(dev)
         res = {}
         t_mse_tot = 0.0
         L = -(-d // ell)
-        useful = 2.0 * npat * ell * (N * ell) * L
-        Kp = -(-N * ell // 64) * 64
-        issued = 3 * 2.0 * npat * ell * Kp * L
-        bf16s = float(pk.get("bf16_tflops_sustained", bf16))
+        K = N * ell
+        Kp = -(-K // 64) * 64
+        # FP32 multiply-add peak from the unit counts: 128 lanes an SM, 2 flops each
+        sm_count = torch.cuda.get_device_properties(dev).multi_processor_count
+        fp32_peak = sm_count * 128 * 2 * 2.07e9 / 1e12
+        ntile = -(-K // 64)
+        gram_flops = 2.0 * (ntile * (ntile + 1) // 2) * 64 * 64 * L  # upper-triangle 64 x 64 tiles
         for p in (0.3, 0.5, 0.7):
             psi_h = make_patterns(cfg, p=p)
             pd = torch.from_numpy(psi_h).to(dev)
             t = _time_ms(torch, lambda: gc.gc_mse(Rd, ell, od, N, m, delta, pd, G, ws=wsM), 3)
             out = gc.gc_mse(Rd, ell, od, N, m, delta, pd, G, ws=wsM)
             gc.gc_status(wsM)
-            gf = gemm_tile_fraction(psi_h, order, N, ell)
-            res[str(p)] = {"ms": t, "patterns/s": npat / (t / 1e3), "gemm_tile_frac": gf,
+            # the same work as two calls: Algorithm 1 into a plan, then the errors
+            pl = gc.gc_decode_plan(Rd, ell, od, N, m, delta, pd, ws=wsP)
+            mse_a = torch.empty(npat, dtype=torch.float64, device=dev)
+            t_plan = _time_ms(torch, lambda: gc.gc_decode_plan(Rd, ell, od, N, m, delta, pd,
+                                                               plan=pl["plan"], ws=wsP), 3)
+            t_apply = _time_ms(torch, lambda: gc.gc_decode_apply(pl["plan"], ell, N, npat, G, Ghat=False,
+                                                                 grad_mse=mse_a, ws=wsA2), 3)
+            gc.gc_status(wsA2)
+            # useful flops of the quadratic forms: 2 nz^2 a row, nz = its non-zero entries
+            cs = pl["plan"][:2 * npat * ell * Kp * 2].view(torch.bfloat16).view(2, npat * ell, Kp)
+            v = (cs[0, :, :K].float() + cs[1, :, :K].float())
+            eye = (torch.arange(K, device=dev) % ell)[None, :] == (torch.arange(npat * ell, device=dev) % ell)[:, None]
+            nz = ((v - eye.float()) != 0).sum(dim=1).double()
+            form_flops = float(2.0 * (nz * nz).sum())
+            del cs, v, eye, nz
+            res[str(p)] = {"ms": t, "patterns/s": npat / (t / 1e3),
+                           "plan_ms": t_plan, "apply_ms": t_apply,
+                           "apply_tflops": (gram_flops + form_flops) / (t_apply / 1e3) / 1e12,
                            "mean_grad_mse": float(out["grad_mse"].mean()),
                            "mean_coef_err": float(out["coef_err"].mean()),
                            "mean_est": float(out["est"].mean())}
-            if gf > 0.99:
-                res[str(p)].update({"issued_tflops": issued / (t / 1e3) / 1e12,
-                                    "useful_tflops": useful / (t / 1e3) / 1e12})
             t_mse_tot += t
         t_mse = t_mse_tot / 3
-        t_dense = res["0.3"]["ms"]
+        r3 = res["0.3"]
         line.update({
             "metric": f"patterns/sec (MSE only, m=N=64, delta=8, d=65536, 10^5 patterns, l={ell})",
             "value": npat / (t_mse / 1e3), "unit": "patterns/s",
@@ -1186,15 +1173,18 @@ def extra_workload(args):
                             "frac_of_hbm": cfg.Ntil * d * 2 / (t_cg / 1e3) / 1e9 / hbm,
                             "TFLOP/s": 4.0 * cfg.Ntil * d / (t_cg / 1e3) / 1e12},
             "per_p": res,
-            "roofline": {"kernel": "k_combine_tc (MSE only; p = 0.3, whose row tiles are all on the GEMM)",
-                         "bound": "tensor", "unit": "TFLOP/s",
-                         "achieved": issued / (t_dense / 1e3) / 1e12, "peak": bf16s,
-                         "frac": issued / (t_dense / 1e3) / 1e12 / bf16s,
-                         "useful_tflops": useful / (t_dense / 1e3) / 1e12,
-                         "note": "issued = three bf16 MMAs per K step over the padded K; the timed gc_mse "
-                                 "includes Algorithm 1 for the 10^5 patterns; p = 0.5 and 0.7 take the "
-                                 "residual path (gemm_tile_frac per p)",
-                         "peak_source": f"{pk_src} bf16_tflops_sustained"},
+            "roofline": {"kernel": "gc_decode_apply errors only (k_gram_partial, k_gram_reduce, "
+                                   "k_mse_gram) at p = 0.3, the densest decode matrices",
+                         "bound": "alu", "unit": "TFLOP/s",
+                         "achieved": r3["apply_tflops"], "peak": fp32_peak,
+                         "frac": r3["apply_tflops"] / fp32_peak,
+                         "note": "each pattern's MSE is a quadratic form in the Gram matrix of the "
+                                 "N*l chunk blocks; flops = the Gram matrix's upper-triangle tiles "
+                                 "(2 * 64 * 64 * L each) + 2 nz^2 for every decode row with nz "
+                                 "non-zero entries of C - I; the sums read H from shared memory "
+                                 "(one load a multiply-add), which caps them near a quarter of the "
+                                 "FP32 rate; the timed gc_mse also runs Algorithm 1 (plan_ms)",
+                         "peak_source": f"derived: {sm_count} SMs x 128 FP32 lanes x 2 flops x 2.07 GHz"},
             "dtype": "bf16 X, f32 otherwise",
             "config": {"workload": f"sweep m=N=64 delta=8 d=65536 n_c=1024 bf16 npat=10^5 ell={ell}",
                        "l2": "inputs larger than L2 (X 8.6 GB)"}})

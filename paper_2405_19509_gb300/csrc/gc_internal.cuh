@@ -168,6 +168,11 @@ inline size_t plan_bytes(int N, int ell, int npat) {
 }
 // scratch of the GEMM side given the planes (G planes, sum of G, MSE partials)
 size_t apply_ws_bytes(int N, int ell, int npat, int d);
+// ---- gradient MSE through the Gram matrix of the chunk blocks (k_mse_gram.cu)
+bool mse_gram_applies(int N, int ell, int npat);
+size_t mse_gram_ws_bytes(int N, int ell, int d);
+int launch_mse_gram(const __nv_bfloat16* Cs, int Kp, const float* G, int N, int ell, int npat,
+                    int d, double* grad_mse, Carve& ws, cudaStream_t s);
 int launch_apply(const __nv_bfloat16* Cs, const float* G, int N, int ell, int npat, int d,
                  float* Ghat, double* grad_mse, Carve& ws, uint32_t* status, cudaStream_t s);
 // fp32 C (npat x ell x N*ell) -> planes

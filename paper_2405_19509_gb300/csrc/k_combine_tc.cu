@@ -683,8 +683,10 @@ size_t apply_ws_bytes(int N, int ell, int npat, int d) {
   const long long M = (long long)npat * ell;
   const int Kp = combine_kp(N, ell);
   const int nnt = (L + tc::BN - 1) / tc::BN;
-  return align_up((size_t)2 * L * Kp * 2, 256) + align_up((size_t)d * sizeof(float), 256) +
-         align_up((size_t)M * nnt * 2 * sizeof(float), 256) + resid_ws_bytes(N, ell, npat, d);
+  return std::max(align_up((size_t)2 * L * Kp * 2, 256) + align_up((size_t)d * sizeof(float), 256) +
+                      align_up((size_t)M * nnt * 2 * sizeof(float), 256) +
+                      resid_ws_bytes(N, ell, npat, d),
+                  mse_gram_ws_bytes(N, ell, d));
 }
 
 int launch_split_c(const float* C, int N, int ell, int npat, __nv_bfloat16* Cs, cudaStream_t s) {
@@ -709,13 +711,17 @@ int launch_apply(const __nv_bfloat16* Cs, const float* G, int N, int ell, int np
   const int K = N * ell;
   const int Kp = combine_kp(N, ell);  // every TMA row is one aligned 128-byte line
   if (M > (1LL << 31) - 1) return fail(GC_ERR_UNSUPPORTED, "npat*ell too large");
+  const int policy = decode_policy();
+  // errors only, and enough patterns to amortise one Gram matrix of the
+  // chunk blocks: each pattern's MSE is a quadratic form in it
+  if (!Ghat && grad_mse && policy == GC_DECODE_AUTO && mse_gram_applies(N, ell, npat))
+    return launch_mse_gram(Cs, Kp, G, N, ell, npat, d, grad_mse, ws, s);
   const int nmt = (int)((M + BM - 1) / BM), nnt = (L + BN - 1) / BN;
   __nv_bfloat16* Gs = ws.take<__nv_bfloat16>((size_t)2 * L * Kp);
   float* gsum = ws.take<float>((size_t)d);
   float* msep_mem = ws.take<float>((size_t)M * nnt * 2);
   float* msep = grad_mse ? msep_mem : nullptr;
   const ResidLists rl = carve_resid(ws, N, ell, npat, d, grad_mse != nullptr);
-  const int policy = decode_policy();
   // a residual tile may spend up to Kp / 64 corrections per pattern: about
   // what the three MMAs per 64-wide K block cost against reading the ell
   // blocks of one chunk gradient

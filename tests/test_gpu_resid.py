@@ -238,7 +238,9 @@ def test_combine_non_projector_matrix(gc):
     """gc_decode_combine with a decode matrix whose blocks, in one pattern in
     four, are near but not exactly I (every block of such a pattern differs
     from I): both paths against the plain product C . G in fp64 and against
-    each other; MSE-only as well."""
+    each other; MSE-only as well, and errors only under the automatic policy,
+    which forms each MSE as a quadratic form in the Gram matrix of the chunk
+    blocks."""
     N, ell, npat, d = 6, 2, 300, 1024
     rng = np.random.default_rng(17)
     C = np.tile(np.kron(np.ones((1, N)), np.eye(ell)), (npat, 1, 1))
@@ -271,6 +273,12 @@ def test_combine_non_projector_matrix(gc):
             assert_mse_close(float(res["grad_mse"][b]), mref[b], floor, f"{name} mse b={b}")
             assert_mse_close(float(mo[b]), mref[b], floor, f"{name} mse-only b={b}")
     assert np.max(np.abs(got["dense"] - got["residual"])) <= 1e-5 * np.max(np.abs(ref))
+    # errors only under the automatic policy: the quadratic forms in the Gram
+    # matrix of the chunk blocks (exact patterns give 0 exactly)
+    mg = to_np(gc.gc_decode_combine(Cd, ell, N, Gd, Ghat=False)["grad_mse"])
+    for b in range(npat):
+        assert_mse_close(float(mg[b]), mref[b], floor, f"gram mse-only b={b}")
+    assert np.all(mg[keep] == 0.0)
 
 
 @pytest.mark.parametrize("ell", [5, 8])
