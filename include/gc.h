@@ -122,9 +122,14 @@ int gc_inject_stall(int kernels);
  *                       the residual path.
  * Both paths give the same values up to fp32 rounding (the tests compare them
  * with each other and with the fp64 oracle); a pattern whose blocks are all
- * I_ell has grad_mse exactly 0 on the residual path.  Process-wide setting
- * (default GC_DECODE_AUTO) read at each launch; meant for tests and
- * measurements. */
+ * I_ell has grad_mse exactly 0 on the residual path.
+ * Errors only (Ghat = NULL) under GC_DECODE_AUTO, when npat*ell >= 2*N*ell
+ * and N*ell <= 256, take a third path: ghat_b - s = sum_a v_{b,k}[a] G_a with
+ * v = C - (1_N (x) I_ell) row by row, so ||ghat_b - s||^2 = sum_k v H v^T with
+ * H the (N*ell)^2 Gram matrix of the chunk blocks, formed once per call; each
+ * pattern then costs its non-zero entries squared instead of N*ell*L (exact
+ * patterns give 0 exactly).  Process-wide setting (default GC_DECODE_AUTO)
+ * read at each launch; meant for tests and measurements. */
 #define GC_DECODE_AUTO 0
 #define GC_DECODE_DENSE 1
 #define GC_DECODE_RESIDUAL 2
@@ -411,7 +416,8 @@ int gc_decode_combine(const float* C, int ell, int N, int npat, const float* G, 
 
 /* ---- error measures only (Sec. II-A eq. 7, Sec. IV) -------------------
  * gc_decode_batch with Ghat = NULL: coef_err, est and grad_mse per pattern;
- * the decoded gradients are reduced on chip and never written.
+ * the decoded gradients are never written (with enough patterns, grad_mse
+ * comes from the Gram matrix of the chunk blocks: see GC_DECODE_AUTO).
  */
 size_t gc_mse_workspace(int N, int m, int delta, int ell, int npat, int d);
 int gc_mse(const double* R, int ell, const int32_t* order, int N, int m, int delta,
