@@ -70,6 +70,9 @@ def parse():
                          "the 8.6 GB one; with --workload sweep: given chunk gradients instead of "
                          "X (the decode-combine alone, for profiler captures); with --workload "
                          "decode: 256 patterns per step (profiler captures)")
+    ap.add_argument("--decode-policy", default="auto", choices=["auto", "dense", "residual"],
+                    help="with --workload sweep: the batched decode's path (gc_set_decode_policy); "
+                         "dense forces the tensor-core GEMM for profiler captures of it")
     ap.add_argument("--shape", default=None,
                     help="with --workload chunkgrad: one case 'dtype,N,n_c,d' (dtype f32 or bf16) "
                          "timed over --steps calls after --warmup calls, instead of the table of "
@@ -1126,6 +1129,8 @@ def extra_workload(args):
         od = torch.from_numpy(order).to(dev)
         wsM = gc.Workspace(dev)
         wsP, wsA2 = gc.Workspace(dev), gc.Workspace(dev)
+        gc.gc_set_decode_policy({"auto": gc.GC_DECODE_AUTO, "dense": gc.GC_DECODE_DENSE,
+                                 "residual": gc.GC_DECODE_RESIDUAL}[args.decode_policy])
         res = {}
         t_mse_tot = 0.0
         L = -(-d // ell)
@@ -1166,6 +1171,31 @@ def extra_workload(args):
             t_mse_tot += t
         t_mse = t_mse_tot / 3
         r3 = res["0.3"]
+        roof = {"kernel": "gc_decode_apply errors only (k_gram_partial, k_gram_reduce, "
+                          "k_mse_gram) at p = 0.3, the densest decode matrices",
+                "bound": "alu", "unit": "TFLOP/s",
+                "achieved": r3["apply_tflops"], "peak": fp32_peak,
+                "frac": r3["apply_tflops"] / fp32_peak,
+                "note": "each pattern's MSE is a quadratic form in the Gram matrix of the "
+                        "N*l chunk blocks; flops = the Gram matrix's upper-triangle tiles "
+                        "(2 * 64 * 64 * L each) + 2 nz^2 for every decode row with nz "
+                        "non-zero entries of C - I; the sums read H from shared memory "
+                        "(one load a multiply-add), which caps them near a quarter of the "
+                        "FP32 rate; the timed gc_mse also runs Algorithm 1 (plan_ms)",
+                "peak_source": f"derived: {sm_count} SMs x 128 FP32 lanes x 2 flops x 2.07 GHz"}
+        if args.decode_policy == "dense":
+            # every row tile on the bf16x3 tensor-core GEMM: three MMAs per K step
+            issued = 3 * 2.0 * npat * ell * Kp * L
+            bf16s = float(pk.get("bf16_tflops_sustained", bf16))
+            roof = {"kernel": "gc_decode_apply errors only on the GEMM (k_split_gt, k_combine_tc) "
+                              "at p = 0.3", "bound": "tensor", "unit": "TFLOP/s",
+                    "achieved": issued / (r3["apply_ms"] / 1e3) / 1e12, "peak": bf16s,
+                    "frac": issued / (r3["apply_ms"] / 1e3) / 1e12 / bf16s,
+                    "useful_tflops": 2.0 * npat * ell * K * L / (r3["apply_ms"] / 1e3) / 1e12,
+                    "note": "issued = three bf16 MMAs per K step over the padded K "
+                            "(gc_set_decode_policy(DENSE)); apply_tflops per p assumes the "
+                            "Gram path and does not apply",
+                    "peak_source": f"{pk_src} bf16_tflops_sustained"}
         line.update({
             "metric": f"patterns/sec (MSE only, m=N=64, delta=8, d=65536, 10^5 patterns, l={ell})",
             "value": npat / (t_mse / 1e3), "unit": "patterns/s",
@@ -1173,21 +1203,12 @@ def extra_workload(args):
                             "frac_of_hbm": cfg.Ntil * d * 2 / (t_cg / 1e3) / 1e9 / hbm,
                             "TFLOP/s": 4.0 * cfg.Ntil * d / (t_cg / 1e3) / 1e12},
             "per_p": res,
-            "roofline": {"kernel": "gc_decode_apply errors only (k_gram_partial, k_gram_reduce, "
-                                   "k_mse_gram) at p = 0.3, the densest decode matrices",
-                         "bound": "alu", "unit": "TFLOP/s",
-                         "achieved": r3["apply_tflops"], "peak": fp32_peak,
-                         "frac": r3["apply_tflops"] / fp32_peak,
-                         "note": "each pattern's MSE is a quadratic form in the Gram matrix of the "
-                                 "N*l chunk blocks; flops = the Gram matrix's upper-triangle tiles "
-                                 "(2 * 64 * 64 * L each) + 2 nz^2 for every decode row with nz "
-                                 "non-zero entries of C - I; the sums read H from shared memory "
-                                 "(one load a multiply-add), which caps them near a quarter of the "
-                                 "FP32 rate; the timed gc_mse also runs Algorithm 1 (plan_ms)",
-                         "peak_source": f"derived: {sm_count} SMs x 128 FP32 lanes x 2 flops x 2.07 GHz"},
+            "roofline": roof,
             "dtype": "bf16 X, f32 otherwise",
             "config": {"workload": f"sweep m=N=64 delta=8 d=65536 n_c=1024 bf16 npat=10^5 ell={ell}",
+                       "decode_policy": args.decode_policy,
                        "l2": "inputs larger than L2 (X 8.6 GB)"}})
+        gc.gc_set_decode_policy(gc.GC_DECODE_AUTO)
     elif args.workload == "sgd":
         cfg = get("sgd")
         N, m, delta, d = cfg.N, cfg.m, cfg.delta, cfg.d

@@ -16,6 +16,7 @@
 //   compacted in shared memory and q = v H v^T is summed lane-parallel over
 //   the second index, then across the lanes and the ell rows in a fixed order.
 #include <algorithm>
+#include <type_traits>
 
 #include "gc_internal.cuh"
 
@@ -235,15 +236,22 @@ __global__ void __launch_bounds__(W * 32) k_mse_gram(const __nv_bfloat16* __rest
       v2[t] = e2 < nz ? s_val[e2] : 0.f;
       a2[t] = e2 < nz ? s_idx[e2] : 0;
     }
-    const int tmax = (nz + 31) / 32;  // the t with some lane in range
+    // only the t with some lane in range take part (no predicated-off work)
+    auto sweep = [&](auto tn) {
+      constexpr int TN = decltype(tn)::value;
 #pragma unroll 4
-    for (int e = 0; e < nz; ++e) {
-      const float ve = s_val[e];
-      const float* hr = Hm + (size_t)s_idx[e] * K;
+      for (int e = 0; e < nz; ++e) {
+        const float ve = s_val[e];
+        const float* hr = Hm + (size_t)s_idx[e] * K;
 #pragma unroll
-      for (int t = 0; t < KW; ++t)
-        if (t < tmax) uu[t] = fmaf(ve, hr[a2[t]], uu[t]);
-    }
+        for (int t = 0; t < TN; ++t) uu[t] = fmaf(ve, hr[a2[t]], uu[t]);
+      }
+    };
+    const int tmax = (nz + 31) / 32;
+    if (tmax <= 1)
+      sweep(std::integral_constant<int, 1>{});
+    else
+      sweep(std::integral_constant<int, KW>{});
     float q = 0.f;
 #pragma unroll
     for (int t = 0; t < KW; ++t) q = fmaf(v2[t], uu[t], q);
@@ -372,8 +380,7 @@ int launch_mse_gram(const __nv_bfloat16* Cs, int Kp, const float* G, int N, int 
     else if (kw <= 2) GC_MSEG(true, 2);
     else GC_MSEG(true, 4);
   } else {
-    if (kw <= 4) GC_MSEG(false, 4);
-    else GC_MSEG(false, 8);
+    GC_MSEG(false, 8);  // 128 < N*ell <= 256
   }
 #undef GC_MSEG
   if (e != cudaSuccess) return cuda_check(e, "cudaFuncSetAttribute(k_mse_gram)");
