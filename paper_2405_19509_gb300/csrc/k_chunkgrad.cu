@@ -31,36 +31,21 @@
 #include <type_traits>
 
 #include "gc_internal.cuh"
+#include "tc_ptx.cuh"
 
 namespace gc {
 
 namespace {
 
-__device__ __forceinline__ uint32_t smem_u32(const void* p) {
-  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
-}
-__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
-  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count)
-               : "memory");
-}
+// the CTA-local mbarrier wrappers are the shared ones (tc_ptx.cuh); the
+// cluster-scope ones below are this kernel's own
+using tcw::mbar_expect_tx;
+using tcw::mbar_init;
+using tcw::mbar_try_wait;
+using tcw::smem_u32;
+
 __device__ __forceinline__ void fence_mbar_init() {
   asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-}
-__device__ __forceinline__ void mbar_expect_tx(uint64_t* bar, uint32_t bytes) {
-  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)),
-               "r"(bytes)
-               : "memory");
-}
-__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
-  uint32_t ok;
-  asm volatile(
-      "{\n\t.reg .pred p;\n\t"
-      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
-      "selp.u32 %0, 1, 0, p;\n\t}"
-      : "=r"(ok)
-      : "r"(smem_u32(bar)), "r"(parity)
-      : "memory");
-  return ok != 0;
 }
 __device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t bytes,
                                          uint64_t* bar) {
@@ -159,9 +144,6 @@ struct CGArgs {
   uint32_t* status;
 };
 
-__device__ __forceinline__ void mbar_arrive_local(uint64_t* bar) {
-  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
-}
 // Arrive on the mbarrier at the same offset in cluster peer `rank`, releasing
 // this thread's prior shared::cluster stores to it.
 __device__ __forceinline__ void mbar_arrive_remote(uint64_t* bar, uint32_t rank) {
@@ -320,7 +302,7 @@ __device__ __forceinline__ void chunkgrad_body(const CGArgs& a) {
             st[(size_t)r * a.ld_s + c] = (c < a.Wc && col < a.d) ? src[col] : T(0.f);
           }
         }
-        mbar_arrive_local(&full[s]);
+        tcw::mbar_arrive(&full[s]);
       }
       issued = n + 1;
     }
@@ -394,7 +376,7 @@ __device__ __forceinline__ void chunkgrad_body(const CGArgs& a) {
     // hand a stage back to the producer (every lane of the warp is done reading it)
     auto release = [&](const Ring& g) {
       __syncwarp();
-      if (lane == 0) mbar_arrive_local(&empty[g.s]);
+      if (lane == 0) tcw::mbar_arrive(&empty[g.s]);
     };
     // Dot products of batch n, reduced over the CTA (warp butterfly, then
     // lane-parallel over (warp, row) pairs) and, with clusters, sent to every
