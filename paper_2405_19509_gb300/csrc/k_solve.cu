@@ -404,17 +404,34 @@ template <int ELL>
 __device__ __forceinline__ void write_planes(__nv_bfloat16* Cs, int Kp, int npat, int b, int i,
                                              const float (&Pf)[ELL][ELL]) {
   const size_t plane = (size_t)npat * ELL * Kp;
+  if constexpr (ELL % 2 == 0) {
+    // pairs of adjacent columns as one 4-byte store per plane (Kp and i*ELL
+    // even; plan buffers are 256-byte aligned)
 #pragma unroll
-  for (int a = 0; a < ELL; ++a)
+    for (int a = 0; a < ELL; ++a)
 #pragma unroll
-    for (int k = 0; k < ELL; ++k) {
-      const float v = Pf[a][k];
-      const __nv_bfloat16 hi = __float2bfloat16_rn(v);
-      const __nv_bfloat16 lo = __float2bfloat16_rn(v - __bfloat162float(hi));
-      const size_t idx = ((size_t)b * ELL + a) * Kp + (size_t)i * ELL + k;
-      Cs[idx] = hi;
-      Cs[plane + idx] = lo;
-    }
+      for (int k = 0; k < ELL; k += 2) {
+        const float v0 = Pf[a][k], v1 = Pf[a][k + 1 < ELL ? k + 1 : k];
+        const __nv_bfloat16 h0 = __float2bfloat16_rn(v0), h1 = __float2bfloat16_rn(v1);
+        const __nv_bfloat16 l0 = __float2bfloat16_rn(v0 - __bfloat162float(h0));
+        const __nv_bfloat16 l1 = __float2bfloat16_rn(v1 - __bfloat162float(h1));
+        const size_t idx = ((size_t)b * ELL + a) * Kp + (size_t)i * ELL + k;
+        *reinterpret_cast<__nv_bfloat162*>(Cs + idx) = __halves2bfloat162(h0, h1);
+        *reinterpret_cast<__nv_bfloat162*>(Cs + plane + idx) = __halves2bfloat162(l0, l1);
+      }
+  } else {
+#pragma unroll
+    for (int a = 0; a < ELL; ++a)
+#pragma unroll
+      for (int k = 0; k < ELL; ++k) {
+        const float v = Pf[a][k];
+        const __nv_bfloat16 hi = __float2bfloat16_rn(v);
+        const __nv_bfloat16 lo = __float2bfloat16_rn(v - __bfloat162float(hi));
+        const size_t idx = ((size_t)b * ELL + a) * Kp + (size_t)i * ELL + k;
+        Cs[idx] = hi;
+        Cs[plane + idx] = lo;
+      }
+  }
 }
 // Zero the padding columns [N*ell, Kp) of pattern b's rows (both planes);
 // thread t of the `run` threads owning the pattern takes entries t, t+run, ...
@@ -495,7 +512,16 @@ __global__ void __launch_bounds__(kPatThreads) k_patterns(const double* __restri
       auto emit = [&](int h, int k, double v) {
         if (E) E[(((size_t)b * m + hw[h]) * delta + hp[h]) * ELL + k] = v;
       };
-      if (TABLE && cnt <= tb.bits) {
+      if (!E && __popc(mask) >= ELL) {
+        // full row rank: the decode block is I exactly (Sec. II-A); no table
+        // read (the table holds the same I and 0 for these masks)
+        D = __popc(mask);
+#pragma unroll
+        for (int a = 0; a < ELL; ++a)
+#pragma unroll
+          for (int k = 0; k < ELL; ++k) Pf[a][k] = a == k ? 1.f : 0.f;
+        err = 0.0;
+      } else if (TABLE && cnt <= tb.bits) {
         const size_t e = ((size_t)i << tb.bits) | mask;
         const float* pi = tb.pi + e * ELL * ELL;
         if (ELL == 2) {  // one 16-byte load for the 2 x 2 block
@@ -518,14 +544,6 @@ __global__ void __launch_bounds__(kPatThreads) k_patterns(const double* __restri
 #pragma unroll
             for (int k = 0; k < ELL; ++k) emit(h, k, xp[h * ELL + k]);
         }
-      } else if (!E && __popc(mask) >= ELL) {
-        // full row rank: the decode block is I exactly (Sec. II-A)
-        D = __popc(mask);
-#pragma unroll
-        for (int a = 0; a < ELL; ++a)
-#pragma unroll
-          for (int k = 0; k < ELL; ++k) Pf[a][k] = a == k ? 1.f : 0.f;
-        err = 0.0;
       } else {
         double Pi[ELL][ELL];
         D = solve_block<ELL>(R, m, cnt, hw, mask, Pi, err, status, emit);
