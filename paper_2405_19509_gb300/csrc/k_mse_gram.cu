@@ -8,7 +8,11 @@
 //   ||ghat_b - s||^2 = sum_k v_{b,k} H v_{b,k}^T,   H[a][a'] = <G_a, G_a'>,
 // so one Gram matrix of the chunk blocks (N*ell x N*ell, formed once per call)
 // replaces the batch's (npat*ell) x (N*ell) x L product: each row costs at
-// most (N*ell)^2 multiply-adds, only over its non-zero entries.
+// most (N*ell)^2 multiply-adds, only over its non-zero entries.  When ell does
+// not divide d the last output block has only L_last = d - (ell-1) L columns,
+// so its rows take H_last, the same sums over the first L_last columns (the
+// other rows the full H); the slices are cut at L_last so that both come
+// from one pass.
 //
 // k_gram_partial: H over column slices, 64 x 64 tiles of the upper triangle,
 //   fp32 sums within a slice; k_gram_reduce adds the slices in order in fp64.
@@ -28,7 +32,7 @@ constexpr int kGramTile = 64;    // H tile edge
 constexpr int kGramCols = 32;    // columns staged per step
 constexpr int kGramMaxSplits = 128;
 constexpr int kGramMaxK = 256;   // N*ell beyond which the Gram path is not taken
-constexpr int kMseWarps = 32;    // warps of a k_mse_gram block
+constexpr int kMseWarps = 32;    // warps of a k_mse_gram block (H in shared memory)
 constexpr int kHSmemMaxK = 128;  // H staged in shared memory up to this N*ell
 
 // Upper-triangle tile t -> (ta, tb), ta <= tb, row-major over the triangle.
@@ -57,7 +61,7 @@ __device__ __forceinline__ void gram_load8(const float* __restrict__ G, int N, i
   const int i = a / ell, k = a - i * ell;
   const float* p = G + (size_t)i * d + (size_t)k * L;
   const long long lim = min((long long)c_hi, (long long)d - (long long)k * L);  // columns < lim exist
-  if (vec && c + 8 <= lim) {
+  if (vec && (c & 3) == 0 && c + 8 <= lim) {
     const float4 x = __ldg(reinterpret_cast<const float4*>(p + c));
     const float4 y = __ldg(reinterpret_cast<const float4*>(p + c + 4));
     v[0] = x.x; v[1] = x.y; v[2] = x.z; v[3] = x.w;
@@ -70,8 +74,8 @@ __device__ __forceinline__ void gram_load8(const float* __restrict__ G, int N, i
 }
 
 __global__ void __launch_bounds__(256) k_gram_partial(const float* __restrict__ G, int N, int ell,
-                                                      int d, int L, int slice, int vec,
-                                                      float* __restrict__ partial) {
+                                                      int d, int L, int slice, int nsa, int l_last,
+                                                      int vec, float* __restrict__ partial) {
   // staged column-major, sa[c][r], so that a thread reads 4 rows as one 16-byte load
   __shared__ __align__(16) float sa[kGramCols][kGramTile];
   __shared__ __align__(16) float sb[kGramCols][kGramTile];
@@ -79,7 +83,9 @@ __global__ void __launch_bounds__(256) k_gram_partial(const float* __restrict__ 
   int ta, tb;
   tri_tile(blockIdx.x, nt, ta, tb);
   const int z = blockIdx.y;
-  const int c_lo = z * slice, c_hi = min(L, c_lo + slice);
+  // slices z < nsa cover [0, l_last); slice nsa (when l_last < L) covers [l_last, L)
+  const int c_lo = z < nsa ? z * slice : l_last;
+  const int c_hi = z < nsa ? min(l_last, c_lo + slice) : L;
   const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;  // 4 x 4 outputs: rows 4 ty.., cols 4 tx..
   const int sr = threadIdx.x >> 2, sq = threadIdx.x & 3;    // staging: row sr, columns 8 sq .. 8 sq + 7
   float acc[4][4];
@@ -122,12 +128,14 @@ __global__ void __launch_bounds__(256) k_gram_partial(const float* __restrict__ 
         make_float4(acc[u][0], acc[u][1], acc[u][2], acc[u][3]);
 }
 
-// H[a][b] = H[b][a] = sum over the slices of the partials, in fp64: block
-// (tile t, part y) takes 32 of the tile's entries; thread (entry j, group g)
-// adds the slices z = g, g + 8, ... and the eight group sums are added in
-// order g = 0 .. 7.
+// H_last[a][b] = H_last[b][a] = sum over the slices z < nsa of the partials,
+// in fp64, and H = H_last + slice nsa when there is one: block (tile t, part y)
+// takes 32 of the tile's entries; thread (entry j, group g) adds the slices
+// z = g, g + 8, ... (< nsa) and the eight group sums are added in order
+// g = 0 .. 7.
 __global__ void __launch_bounds__(256) k_gram_reduce(const float* __restrict__ partial, int K,
-                                                     int nsplit, float* __restrict__ H) {
+                                                     int nsa, int nsplit, float* __restrict__ H,
+                                                     float* __restrict__ H_last) {
   __shared__ double s_part[8][32];
   const int nt = (K + kGramTile - 1) / kGramTile;
   int ta, tb;
@@ -137,14 +145,14 @@ __global__ void __launch_bounds__(256) k_gram_reduce(const float* __restrict__ p
   const float* src = partial + (size_t)blockIdx.x * nsplit * (kGramTile * kGramTile) + e;
   double sum = 0.0;
   int z = g;
-  for (; z + 56 < nsplit; z += 64) {  // eight slices of this group at a time
+  for (; z + 56 < nsa; z += 64) {  // eight slices of this group at a time
     float v[8];
 #pragma unroll
     for (int u = 0; u < 8; ++u) v[u] = src[(size_t)(z + 8 * u) * (kGramTile * kGramTile)];
 #pragma unroll
     for (int u = 0; u < 8; ++u) sum += (double)v[u];
   }
-  for (; z < nsplit; z += 8) sum += (double)src[(size_t)z * (kGramTile * kGramTile)];
+  for (; z < nsa; z += 8) sum += (double)src[(size_t)z * (kGramTile * kGramTile)];
   s_part[g][j] = sum;
   __syncthreads();
   if (g != 0) return;
@@ -154,6 +162,11 @@ __global__ void __launch_bounds__(256) k_gram_reduce(const float* __restrict__ p
   const int r = e / kGramTile, c = e % kGramTile;
   const int a = ta * kGramTile + r, b = tb * kGramTile + c;
   if (a >= K || b >= K) return;
+  if (nsplit > nsa) {  // a padded last block: H_last, then the full sums
+    H_last[(size_t)a * K + b] = (float)tot;
+    H_last[(size_t)b * K + a] = (float)tot;
+    tot += (double)src[(size_t)nsa * (kGramTile * kGramTile)];
+  }
   H[(size_t)a * K + b] = (float)tot;
   H[(size_t)b * K + a] = (float)tot;
 }
@@ -163,10 +176,11 @@ __global__ void __launch_bounds__(256) k_gram_reduce(const float* __restrict__ p
 // Lane l holds entries a = 32 u + l (u < KW) of a row; the warp's rows are
 // walked in order with the loads of the row two ahead issued before the
 // current row is summed, so the load latency hides behind two rows' work.
-template <bool HS, int KW, int W>
+template <bool HS, int KW, int W, bool PAD>
 __global__ void __launch_bounds__(W * 32) k_mse_gram(const __nv_bfloat16* __restrict__ Cs,
                                                              int Kp, int N, int ell, int npat,
                                                              const float* __restrict__ H,
+                                                             const float* __restrict__ H_last,
                                                              double inv_d,
                                                              double* __restrict__ grad_mse) {
   extern __shared__ float s_dyn[];
@@ -236,13 +250,16 @@ __global__ void __launch_bounds__(W * 32) k_mse_gram(const __nv_bfloat16* __rest
       v2[t] = e2 < nz ? s_val[e2] : 0.f;
       a2[t] = e2 < nz ? s_idx[e2] : 0;
     }
+    // the last output block of a padded d has its own Gram matrix (read
+    // through the cache)
+    const float* Hk = (PAD && k == ell - 1) ? H_last : Hm;
     // only the t with some lane in range take part (no predicated-off work)
     auto sweep = [&](auto tn) {
       constexpr int TN = decltype(tn)::value;
 #pragma unroll 4
       for (int e = 0; e < nz; ++e) {
         const float ve = s_val[e];
-        const float* hr = Hm + (size_t)s_idx[e] * K;
+        const float* hr = Hk + (size_t)s_idx[e] * K;
 #pragma unroll
         for (int t = 0; t < TN; ++t) uu[t] = fmaf(ve, hr[a2[t]], uu[t]);
       }
@@ -305,21 +322,22 @@ __global__ void __launch_bounds__(W * 32) k_mse_gram(const __nv_bfloat16* __rest
   }
 }
 
-template <bool HS, int KW, int W>
+template <bool HS, int KW, int W, bool PAD>
 cudaError_t launch_mse_gram_t(int blocks, size_t smem, const __nv_bfloat16* Cs, int Kp, int N,
-                              int ell, int npat, const float* H, double inv_d, double* grad_mse,
-                              cudaStream_t s) {
+                              int ell, int npat, const float* H, const float* H_last, double inv_d,
+                              double* grad_mse, cudaStream_t s) {
   if (HS) {
     static bool attr = false;
     if (!attr) {
       const cudaError_t e = cudaFuncSetAttribute(
-          k_mse_gram<HS, KW, W>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+          k_mse_gram<HS, KW, W, PAD>, cudaFuncAttributeMaxDynamicSharedMemorySize,
           (int)(((size_t)kHSmemMaxK * kHSmemMaxK + W * 2 * kHSmemMaxK) * sizeof(float)));
       if (e != cudaSuccess) return e;
       attr = true;
     }
   }
-  k_mse_gram<HS, KW, W><<<blocks, W * 32, smem, s>>>(Cs, Kp, N, ell, npat, H, inv_d, grad_mse);
+  k_mse_gram<HS, KW, W, PAD><<<blocks, W * 32, smem, s>>>(Cs, Kp, N, ell, npat, H, H_last,
+                                                           inv_d, grad_mse);
   return cudaSuccess;
 }
 
@@ -342,39 +360,44 @@ size_t mse_gram_ws_bytes(int N, int ell, int d) {
   const int L = (d + ell - 1) / ell;
   const int nt = (K + kGramTile - 1) / kGramTile;
   const size_t ntri = (size_t)nt * (nt + 1) / 2;
-  return align_up(ntri * gram_splits(L) * kGramTile * kGramTile * sizeof(float), 256) +
-         align_up((size_t)K * K * sizeof(float), 256);
+  return align_up(ntri * (gram_splits(L) + 1) * kGramTile * kGramTile * sizeof(float), 256) +
+         2 * align_up((size_t)K * K * sizeof(float), 256);
 }
 
 int launch_mse_gram(const __nv_bfloat16* Cs, int Kp, const float* G, int N, int ell, int npat,
                     int d, double* grad_mse, Carve& ws, cudaStream_t s) {
   const int K = N * ell;
   const int L = (d + ell - 1) / ell;
+  const int l_last = d - (ell - 1) * L;  // real columns of the last block, 0 < l_last <= L
   const int nt = (K + kGramTile - 1) / kGramTile;
   const int ntri = nt * (nt + 1) / 2;
-  const int nsplit = gram_splits(L);
-  const int slice = ((L + nsplit - 1) / nsplit + kGramCols - 1) / kGramCols * kGramCols;
+  const int nsa = gram_splits(l_last);                  // slices of [0, l_last)
+  const int nsplit = nsa + (l_last < L ? 1 : 0);        // + the last block's padding range
+  const int slice = ((l_last + nsa - 1) / nsa + kGramCols - 1) / kGramCols * kGramCols;
   float* partial = ws.take<float>((size_t)ntri * nsplit * kGramTile * kGramTile);
   float* H = ws.take<float>((size_t)K * K);
+  float* H_last = ws.take<float>((size_t)K * K);
   if (npat == 0) return GC_OK;
   const bool vec = d % 4 == 0 && L % 4 == 0 && reinterpret_cast<uintptr_t>(G) % 16 == 0;
-  k_gram_partial<<<dim3((unsigned)ntri, (unsigned)nsplit), 256, 0, s>>>(G, N, ell, d, L, slice,
-                                                                        vec ? 1 : 0, partial);
-  k_gram_reduce<<<dim3((unsigned)ntri, (kGramTile * kGramTile) / 32), 256, 0, s>>>(partial, K,
-                                                                                   nsplit, H);
+  k_gram_partial<<<dim3((unsigned)ntri, (unsigned)nsplit), 256, 0, s>>>(
+      G, N, ell, d, L, slice, nsa, l_last, vec ? 1 : 0, partial);
+  k_gram_reduce<<<dim3((unsigned)ntri, (kGramTile * kGramTile) / 32), 256, 0, s>>>(
+      partial, K, nsa, nsplit, H, H_last);
+  const float* hl = l_last < L ? H_last : nullptr;
   const bool hs = K <= kHSmemMaxK;
-  // H from shared memory: two blocks of 32 warps an SM (96 KB a block);
-  // from the cache (up to 8 entries a lane, more registers): blocks of 16 warps
-  const int W = hs ? kMseWarps : kMseWarps / 2;
+  // H from shared memory and no padded last block: blocks of 32 warps (96 KB,
+  // 64 registers a thread); otherwise blocks of 16 warps (up to 128 registers)
+  const int W = hs && !hl ? kMseWarps : kMseWarps / 2;
   const size_t smem = ((hs ? (size_t)K * K : 0) + (size_t)W * 2 * K) * sizeof(float);
   const int blocks = (int)std::min<long long>(((long long)npat + W - 1) / W,
                                               2LL * device_sm_count());
   const int kw = (K + 31) / 32;  // <= kGramMaxK / 32 = 8
   cudaError_t e = cudaSuccess;
 #define GC_MSEG(HSV, KWV)                                                                         \
-  e = launch_mse_gram_t<HSV, KWV, HSV ? kMseWarps : kMseWarps / 2>(blocks, smem, Cs, Kp, N, ell,  \
-                                                                    npat, H, 1.0 / (double)d,     \
-                                                                    grad_mse, s)
+  e = hl ? launch_mse_gram_t<HSV, KWV, kMseWarps / 2, true>(                                      \
+               blocks, smem, Cs, Kp, N, ell, npat, H, hl, 1.0 / (double)d, grad_mse, s)          \
+         : launch_mse_gram_t<HSV, KWV, HSV ? kMseWarps : kMseWarps / 2, false>(                  \
+               blocks, smem, Cs, Kp, N, ell, npat, H, hl, 1.0 / (double)d, grad_mse, s)
   if (hs) {
     if (kw <= 1) GC_MSEG(true, 1);
     else if (kw <= 2) GC_MSEG(true, 2);

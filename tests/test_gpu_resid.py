@@ -324,3 +324,36 @@ def test_large_ell_both_paths(gc, ell):
         for k, res in out.items():
             assert_grad_close(to_np(res["Ghat"][b]), r.ghat, f"{k} l={ell} b={b}")
             assert_mse_close(float(res["grad_mse"][b]), r.grad_mse, floor, f"{k} l={ell} mse b={b}")
+
+
+@pytest.mark.parametrize("N,delta,ell,d", [(10, 4, 3, 1001), (20, 8, 8, 997), (40, 6, 5, 1500)])
+def test_errors_only_gram_path(gc, N, delta, ell, d):
+    """Errors only under the automatic policy (npat * ell >= 2 N ell): each
+    pattern's gradient MSE as a quadratic form in the Gram matrix of the chunk
+    blocks, with a padded last block (l does not divide d), H in shared memory
+    (N l <= 128) or read through the cache (N l = 160, 200); against the
+    oracle's decoded gradients, against the residual/GEMM decode of the same
+    batch, and exactly 0 for exact patterns."""
+    m = N
+    rng = np.random.default_rng(50 + N + ell)
+    order = O.cyclic_order(N, m, delta)
+    R = rng.standard_normal((ell, m))
+    npat = 2 * N + 7
+    psi = rng.integers(0, delta + 1, size=(npat, m)).astype(np.int32)
+    psi[0] = delta                      # every worker done: exact
+    psi[1] = 0                          # none started
+    G = rng.standard_normal((N, d)).astype(np.float32)
+    Gref = G.astype(np.float64)
+    gsum = Gref.sum(axis=0)
+    floor = 1e-8 * float(gsum @ gsum) / d
+    Rd, od, pd = dev_tensors(R, order, psi)
+    Gd = torch.from_numpy(G).cuda()
+    res = gc.gc_mse(Rd, ell, od, N, m, delta, pd, Gd)               # the Gram path
+    full = gc.gc_decode_batch(Rd, ell, od, N, m, delta, pd, Gd)     # decoded gradients and MSE
+    torch.cuda.synchronize()
+    mg, mf = to_np(res["grad_mse"]), to_np(full["grad_mse"])
+    assert mg[0] == 0.0
+    for b in range(npat):
+        r = O.run_pattern(R, order, psi[b], N, Gref, want_transmit=False)
+        assert_mse_close(float(mg[b]), r.grad_mse, floor, f"gram b={b}")
+        assert_mse_close(float(mg[b]), float(mf[b]), floor, f"gram vs decode b={b}")
