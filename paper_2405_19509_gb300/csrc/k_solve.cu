@@ -626,10 +626,17 @@ size_t solve_table_bytes(int N, int ell, int bits) {
          align_up(ent * ell * ell * sizeof(float), 256) + align_up(ent * sizeof(double), 256);
 }
 
-// Lean variant for N <= 32 without coefficient output: one warp per pattern
-// (lane i = chunk i), grid-stride over patterns, sums by warp shuffles; no
-// shared memory or block barriers, so it runs well beside other kernels.
-template <int ELL, bool TABLE>
+// Lean variant without coefficient output for N <= 32 * CPL: one warp per
+// pattern, lane l takes chunks l, l + 32, ... (at most CPL of them), and
+// the warps stride over the patterns.  A lane's first eight holders of each
+// of its chunks (worker and slot) are read once, before the pattern loop, and
+// stay in registers; there is no shared memory and no block barrier, so the
+// kernel also runs well beside other kernels.  Per pattern the completion
+// masks of the lane's chunks are formed first (every psi load in flight),
+// then the blocks are produced one chunk at a time.  Each lane adds its
+// chunks' errors in chunk order starting from 0 and the lanes are summed by
+// a fixed xor tree: the same sums, in the same order, as k_patterns.
+template <int ELL, bool TABLE, int CPL>
 __global__ void __launch_bounds__(128) k_patterns_warp(const double* __restrict__ R,
                                                        const int32_t* __restrict__ psi,
                                                        Holders hd, int N, int m, int delta,
@@ -638,43 +645,110 @@ __global__ void __launch_bounds__(128) k_patterns_warp(const double* __restrict_
   const int lane = threadIdx.x & 31;
   const int gw = (int)((blockIdx.x * blockDim.x + threadIdx.x) >> 5);
   const int nw = (int)((gridDim.x * blockDim.x) >> 5);
-  const int i = lane;
-  const bool on = i < N;
-  const int cnt = on ? hd.cnt[i] : 0;
-  const int16_t* hw = hd.w + (size_t)(on ? i : 0) * GC_MAX_REPL;
-  const int8_t* hp = hd.p + (size_t)(on ? i : 0) * GC_MAX_REPL;
+  int cnt[CPL];
+  uint4 hw8[CPL];
+  uint2 hp8[CPL];
+#pragma unroll
+  for (int c = 0; c < CPL; ++c) {
+    const int i = lane + 32 * c;
+    cnt[c] = 0;
+    hw8[c] = make_uint4(0u, 0u, 0u, 0u);
+    hp8[c] = make_uint2(0u, 0u);
+    if (i < N) {
+      cnt[c] = hd.cnt[i];
+      hw8[c] = *reinterpret_cast<const uint4*>(hd.w + (size_t)i * GC_MAX_REPL);
+      hp8[c] = *reinterpret_cast<const uint2*>(hd.p + (size_t)i * GC_MAX_REPL);
+    }
+  }
+  const uint32_t udelta = (uint32_t)delta;
   for (int b = gw; b < npat; b += nw) {
+    const int32_t* ps = psi + (size_t)b * m;
+    // completion masks of the lane's chunks; psi outside [0, delta] counts as 0
+    uint32_t mask[CPL];
+    bool bad = false;
+#pragma unroll
+    for (int c = 0; c < CPL; ++c) {
+      uint32_t mk = 0;
+      const uint32_t ww[4] = {hw8[c].x, hw8[c].y, hw8[c].z, hw8[c].w};
+#pragma unroll
+      for (int q = 0; q < 8; ++q) {
+        if (q < cnt[c]) {
+          const int wq = (int)(int16_t)(ww[q >> 1] >> (16 * (q & 1)));
+          const int pq = (int)(int8_t)(((q < 4 ? hp8[c].x : hp8[c].y) >> (8 * (q & 3))) & 0xffu);
+          uint32_t v = (uint32_t)__ldg(ps + wq);
+          if (v > udelta) {
+            bad = true;
+            v = 0;
+          }
+          if (pq < (int)v) mk |= 1u << q;
+        }
+      }
+      // holders past the eighth (chunks with more than eight copies), eight a load
+      for (int h0 = 8; h0 < cnt[c]; h0 += 8) {
+        const size_t row = (size_t)(lane + 32 * c) * GC_MAX_REPL + h0;
+        const uint4 w8 = *reinterpret_cast<const uint4*>(hd.w + row);
+        const uint2 p8 = *reinterpret_cast<const uint2*>(hd.p + row);
+        const uint32_t wx[4] = {w8.x, w8.y, w8.z, w8.w};
+#pragma unroll
+        for (int q = 0; q < 8; ++q) {
+          if (h0 + q < cnt[c]) {
+            const int wq = (int)(int16_t)(wx[q >> 1] >> (16 * (q & 1)));
+            const int pq = (int)(int8_t)(((q < 4 ? p8.x : p8.y) >> (8 * (q & 3))) & 0xffu);
+            uint32_t v = (uint32_t)__ldg(ps + wq);
+            if (v > udelta) {
+              bad = true;
+              v = 0;
+            }
+            if (pq < (int)v) mk |= 1u << (h0 + q);
+          }
+        }
+      }
+      mask[c] = mk;
+    }
+    if (__any_sync(0xffffffffu, bad) && lane == 0) atomicOr(status, ST_BAD_PSI);
     double err = 0.0;
     int def = 0;
-    if (on) {
-      const int32_t* ps = psi + (size_t)b * m;
-      uint32_t mask = 0;
-      for (int h = 0; h < cnt; ++h) {
-        int v = __ldg(ps + hw[h]);
-        if (v < 0 || v > delta) {
-          atomicOr(status, ST_BAD_PSI);
-          v = 0;
+#pragma unroll 1
+    for (int c = 0; c < CPL; ++c) {
+      const int i = lane + 32 * c;
+      if (i >= N) break;
+      // this chunk's mask and holder count, selected without indexing the arrays
+      uint32_t mk = mask[0];
+      int cn = cnt[0];
+#pragma unroll
+      for (int q = 1; q < CPL; ++q)
+        if (c == q) {
+          mk = mask[q];
+          cn = cnt[q];
         }
-        if (hp[h] < v) mask |= 1u << h;
-      }
-      const int D = __popc(mask);
+      const int D = __popc(mk);
       float Pf[ELL][ELL];
+      double e_i = 0.0;
       if (D >= ELL) {  // full row rank: the decode block is I exactly (Sec. II-A)
 #pragma unroll
         for (int a = 0; a < ELL; ++a)
 #pragma unroll
           for (int k = 0; k < ELL; ++k) Pf[a][k] = a == k ? 1.f : 0.f;
-      } else if (TABLE && cnt <= tb.bits) {
-        const size_t e = ((size_t)i << tb.bits) | mask;
+      } else if (TABLE && cn <= tb.bits) {
+        const size_t e = ((size_t)i << tb.bits) | mk;
         const float* pi = tb.pi + e * ELL * ELL;
+        if (ELL == 2) {  // one 16-byte load for the 2 x 2 block
+          const float4 q = *reinterpret_cast<const float4*>(pi);
+          Pf[0][0] = q.x;
+          Pf[0][ELL - 1] = q.y;
+          Pf[ELL - 1][0] = q.z;
+          Pf[ELL - 1][ELL - 1] = q.w;
+        } else {
 #pragma unroll
-        for (int a = 0; a < ELL; ++a)
+          for (int a = 0; a < ELL; ++a)
 #pragma unroll
-          for (int k = 0; k < ELL; ++k) Pf[a][k] = pi[a * ELL + k];
-        err = tb.err[e];
+            for (int k = 0; k < ELL; ++k) Pf[a][k] = pi[a * ELL + k];
+        }
+        e_i = tb.err[e];
       } else {
         double Pi[ELL][ELL];
-        solve_block<ELL>(R, m, cnt, hw, mask, Pi, err, status, [](int, int, double) {});
+        solve_block<ELL>(R, m, cn, hd.w + (size_t)i * GC_MAX_REPL, mk, Pi, e_i, status,
+                         [](int, int, double) {});
 #pragma unroll
         for (int a = 0; a < ELL; ++a)
 #pragma unroll
@@ -690,12 +764,14 @@ __global__ void __launch_bounds__(128) k_patterns_warp(const double* __restrict_
       if (out.Cs) write_planes<ELL>(out.Cs, out.Kp, npat, b, i, Pf);
       if (out.delta_out) out.delta_out[(size_t)b * N + i] = (uint8_t)D;
       if (out.support) {
+        const int16_t* hw = hd.w + (size_t)i * GC_MAX_REPL;
         uint8_t* row = out.support + ((size_t)b * N + i) * m;
         for (int j = 0; j < m; ++j) row[j] = 0;
-        for (int h = 0; h < cnt; ++h)
-          if ((mask >> h) & 1u) row[hw[h]] = 1;
+        for (int h = 0; h < cn; ++h)
+          if ((mk >> h) & 1u) row[hw[h]] = 1;
       }
-      def = D < ELL ? ELL - D : 0;
+      err += e_i;
+      def += D < ELL ? ELL - D : 0;
     }
     if (out.Cs) zero_pad<ELL>(out.Cs, out.Kp, N, npat, b, lane, 32);
     // fixed xor tree over the 32 lanes (deterministic)
@@ -723,16 +799,33 @@ static void run_solve(const double* R, const int32_t* psi, Holders h, int N, int
     count_launches(1);
   }
   if (npat == 0) return;
-  if (!out.E && N <= 32) {
-    const int warps = 4;  // per 128-thread block
-    const int blocks = std::max(1, std::min((npat + warps - 1) / warps, 8 * device_sm_count()));
-    count_launches(1);
-    if (use_table)
-      k_patterns_warp<ELL, true><<<blocks, 128, 0, s>>>(R, psi, h, N, m, delta, npat, tb, out,
-                                                        status);
-    else
-      k_patterns_warp<ELL, false><<<blocks, 128, 0, s>>>(R, psi, h, N, m, delta, npat, tb, out,
-                                                         status);
+  // chunks a lane of the lean kernel takes: up to 4 for ell <= 4 (larger ell
+  // keep one, their solves fill the register file), else k_patterns below
+  const int cpl = N <= 32 ? 1 : (ELL <= 4 && N <= 64 ? 2 : (ELL <= 4 && N <= 128 ? 4 : 0));
+  if (!out.E && cpl > 0) {
+    // as many 128-thread blocks as are resident at once (all warps stride
+    // over the patterns, so a second partial wave would only add a tail)
+    auto go = [&](auto kern) {
+      int per_sm = 0;
+      if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, 128, 0) != cudaSuccess ||
+          per_sm < 1) {
+        cudaGetLastError();
+        per_sm = 1;
+      }
+      const int warps = 4;  // per 128-thread block
+      const int blocks =
+          std::max(1, std::min((npat + warps - 1) / warps, per_sm * device_sm_count()));
+      kern<<<blocks, 128, 0, s>>>(R, psi, h, N, m, delta, npat, tb, out, status);
+      count_launches(1);
+    };
+    if (cpl == 1) {
+      use_table ? go(k_patterns_warp<ELL, true, 1>) : go(k_patterns_warp<ELL, false, 1>);
+    } else if constexpr (ELL <= 4) {
+      if (cpl == 2)
+        use_table ? go(k_patterns_warp<ELL, true, 2>) : go(k_patterns_warp<ELL, false, 2>);
+      else
+        use_table ? go(k_patterns_warp<ELL, true, 4>) : go(k_patterns_warp<ELL, false, 4>);
+    }
     return;
   }
   int ppb = N <= kPatThreads ? kPatThreads / N : 0;

@@ -519,3 +519,74 @@ def test_maximum_delta_and_replication(gc):
     assert np.array_equal(out["T"].cpu().numpy(), Tn)
     assert np.array_equal(out["psi"].cpu().numpy(), psin)
     assert np.array_equal(out["T_full"].cpu().numpy(), TFn)
+
+
+# ------------------------------------------------------------------ the lean Algorithm 1 kernel
+@pytest.mark.parametrize("N,delta,ell,npat", [
+    (40, 4, 2, 300),     # two chunks a lane, the second group ragged (8 of 32 lanes)
+    (64, 8, 2, 400),     # the MSE sweep's shape, memo table (npat >= 2^delta)
+    (64, 8, 3, 9),       # direct solves (npat < 2^delta)
+    (100, 6, 4, 200),    # four chunks a lane, ragged
+    (128, 6, 1, 100),
+    (72, 12, 2, 5000),   # twelve holders a chunk: holders past the eighth, table of 2^12 masks
+    (48, 16, 2, 30),     # delta = 16: no table, sixteen holders a chunk
+])
+def test_lean_solve_matches_coefficient_path(gc, N, delta, ell, npat):
+    """Without E, Algorithm 1 for N <= 128 runs one warp per pattern with
+    several chunks a lane; it must give the Delta, supports, estimate, decode
+    blocks and coefficient error of the per-chunk-thread kernel that also
+    writes E (bit for bit where both solve; exactly I where that kernel
+    rounds a solved full-rank block), and the oracle's within tolerance; bad
+    psi entries are flagged and read as 0 on both paths."""
+    m = N
+    rng = np.random.default_rng(1000 + N + delta + ell)
+    order = O.cyclic_order(N, m, delta)
+    R = rng.standard_normal((ell, m))
+    psi = rng.integers(0, delta + 1, size=(npat, m)).astype(np.int32)
+    psi[0] = 0
+    psi[1 % npat] = delta
+    if npat > 3:
+        psi[2, ::3] = ell - 1   # chunks with fewer than ell finishers
+    Rd, od, pd = dev_tensors(R, order, psi)
+    full = gc.gc_find_encoding_coeff(Rd, ell, od, N, m, delta, pd, support=True)
+    lean = gc.gc_find_encoding_coeff(Rd, ell, od, N, m, delta, pd, E=False, support=True)
+    for k in ("delta", "support", "est"):
+        assert torch.equal(lean[k], full[k]), f"lean and coefficient kernels differ in {k}"
+    ce, est, D = to_np(lean["coef_err"]), to_np(lean["est"]), to_np(lean["delta"])
+    C = to_np(lean["C"])
+    # blocks of chunks with Delta >= ell: exactly I on the lean path (Sec. II-A),
+    # I to rounding where E is also wanted (that path solves them); the
+    # others come from the same solve on both paths, bit for bit
+    Cf = to_np(full["C"]).reshape(npat, ell, N, ell)
+    Cl = C.reshape(npat, ell, N, ell)
+    full_rank = (D >= ell)[:, None, :, None]
+    eye = np.broadcast_to(np.eye(ell, dtype=np.float32)[None, :, None, :], Cl.shape)
+    assert np.array_equal(np.where(full_rank, Cl, eye), eye)
+    assert np.max(np.abs(np.where(full_rank, Cf, eye) - eye)) <= 1e-6
+    assert np.array_equal(np.where(full_rank, 0, Cl), np.where(full_rank, 0, Cf))
+    assert np.all(np.abs(ce - to_np(full["coef_err"])) <= 1e-12 * np.maximum(1.0, ce))
+    for b in sorted({0, 1 % npat, 2 % npat, npat - 1}):
+        r = O.run_pattern(R, order, psi[b], N)
+        assert np.array_equal(D[b], r.Delta), b
+        assert np.max(np.abs(C[b] - r.C)) <= 2e-6, b
+        assert abs(ce[b] - r.coef_err) <= 1e-9 * max(1.0, r.coef_err), b
+        assert est[b] == r.est, b
+    # out-of-range entries: flagged, and read as 0 by both kernels
+    bad = psi[:4].copy()
+    bad[0, 0], bad[1 % 4, m - 1] = delta + 1, -2
+    Rd, od, bd = dev_tensors(R, order, bad)
+    outs = []
+    for want_E in (True, False):
+        ws = gc.Workspace()
+        outs.append(gc.gc_find_encoding_coeff(Rd, ell, od, N, m, delta, bd, E=want_E, ws=ws))
+        with pytest.raises(gc.GCError) as ei:
+            gc.gc_status(ws)
+        assert ei.value.code == -7 and "psi" in str(ei.value)
+    zeroed = bad.copy()
+    zeroed[(zeroed < 0) | (zeroed > delta)] = 0
+    Rd, od, zd = dev_tensors(R, order, zeroed)
+    ref = gc.gc_find_encoding_coeff(Rd, ell, od, N, m, delta, zd, E=False)
+    for k in ("delta", "est"):
+        assert torch.equal(outs[1][k], outs[0][k]) and torch.equal(outs[1][k], ref[k]), k
+    for k in ("C", "coef_err"):
+        assert torch.equal(outs[1][k], ref[k]), k
