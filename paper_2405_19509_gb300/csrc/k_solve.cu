@@ -770,15 +770,20 @@ __global__ void __launch_bounds__(128) k_patterns_warp(const double* __restrict_
         for (int h = 0; h < cn; ++h)
           if ((mk >> h) & 1u) row[hw[h]] = 1;
       }
-      err += e_i;
+      // GB300's fp64 pipe retires 2 operations a clock per SM, so the
+      // additions of +0 (every block with Delta >= ell) are skipped: adding
+      // +0 to a sum that starts at +0 leaves its bits unchanged
+      if (__double_as_longlong(e_i) != 0) err += e_i;
       def += D < ELL ? ELL - D : 0;
     }
     if (out.Cs) zero_pad<ELL>(out.Cs, out.Kp, N, npat, b, lane, 32);
-    // fixed xor tree over the 32 lanes (deterministic)
+    // fixed xor tree over the 32 lanes (deterministic); when every lane's
+    // sum is +0 (an exactly decodable pattern) so is the total
 #pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-      err += __shfl_xor_sync(0xffffffffu, err, o);
-      def += __shfl_xor_sync(0xffffffffu, def, o);
+    for (int o = 16; o > 0; o >>= 1) def += __shfl_xor_sync(0xffffffffu, def, o);
+    if (__any_sync(0xffffffffu, __double_as_longlong(err) != 0)) {
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) err += __shfl_xor_sync(0xffffffffu, err, o);
     }
     if (lane == 0) {
       if (out.coef_err) out.coef_err[b] = err;
