@@ -42,9 +42,15 @@ ROOT = os.path.dirname(os.path.abspath(__file__))
 if ROOT not in sys.path:
     sys.path.insert(0, ROOT)
 
-METRIC = ("decoded gradients/sec (decode-dominated batch: m=N=256, delta=16, d=2^20, "
-          "4096 straggler patterns per step, l=2)")
-METRIC_LOGISTIC = "decoded gradients/sec (logistic m=N=20, delta=4, d=4096, 10^4 realizations, l=2)"
+def metric_decode(ell: int) -> str:
+    return ("decoded gradients/sec (decode-dominated batch: m=N=256, delta=16, d=2^20, "
+            f"4096 straggler patterns per step, l={ell})")
+
+
+def metric_logistic(ell: int) -> str:
+    return f"decoded gradients/sec (logistic m=N=20, delta=4, d=4096, 10^4 realizations, l={ell})"
+
+
 UNIT = "decoded gradients/s"
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 
@@ -221,7 +227,7 @@ def reference_arm(args, rank, world):
     value = statistics.median(rates)
     cores = os.cpu_count()
     line = {
-        "impl": "reference", "metric": METRIC_LOGISTIC, "value": value, "unit": UNIT, "n_gpus": world,
+        "impl": "reference", "metric": metric_logistic(args.ell), "value": value, "unit": UNIT, "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * cfg.npat / value,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
         "data": "synthetic",
@@ -319,7 +325,7 @@ def reference_decode(args, world):
     wall = time.perf_counter() - t_all
     value = 1.0 / statistics.median(per)
     line = {
-        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
+        "impl": "reference", "metric": metric_decode(ell), "value": value, "unit": UNIT, "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * cfg.npat / value,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
         "data": "synthetic",
@@ -568,7 +574,7 @@ def decode_arm(args, rank, world, local_rank):
                               "gc_decode_apply": achieved},
                 "serial_ms": {"gc_decode_plan": serial_ms[0], "gc_decode_apply": serial_ms[1]}}
     line = {
-        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K,
+        "metric": metric_decode(ell), "value": value, "unit": UNIT, "n_gpus": world, "steps": K,
         "warmup": args.warmup, "ms_per_step": total_ms / K, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f32 (Algorithm 1 in f64)",
         "data": "synthetic",
@@ -1014,7 +1020,7 @@ def logistic_arm(args, rank, world, local_rank):
                                       for i in (0, 2)}}
 
     line = {
-        "metric": METRIC_LOGISTIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K,
+        "metric": metric_logistic(ell), "value": value, "unit": UNIT, "n_gpus": world, "steps": K,
         "warmup": args.warmup, "ms_per_step": total_ms / K, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
         "config": {"workload": "logistic m=N=20 delta=4 d=4096 n_c=512 npat=10000 ell=%d" % ell,
