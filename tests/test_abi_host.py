@@ -160,3 +160,23 @@ def test_batched_chunk_grads_validation():
     assert L.gc_chunk_grads_batched(nul, nul, nul, 2, 100, 256, 32, 0, nul, nul, 0, nul) == -3
     assert L.gc_chunk_grads_batched(nul, nul, nul, 2, 128, 256, 32, 0, nul, nul, 0, nul) == -1
     assert L.gc_chunk_grads_batched_workspace(2, 128, 256, 32) > 256
+
+
+def test_binding_without_library_raises(tmp_path):
+    """The package has no CPU fallback: a copy of its Python files without
+    libgc.so beside them refuses to import, naming the missing library."""
+    import shutil
+    import subprocess
+    import sys
+    pkg = os.path.join(ROOT, "paper_2405_19509_gb300")
+    dst = tmp_path / "paper_2405_19509_gb300"
+    dst.mkdir()
+    for name in os.listdir(pkg):
+        if name.endswith(".py"):
+            shutil.copy(os.path.join(pkg, name), dst / name)
+    assert not (dst / "libgc.so").exists()
+    r = subprocess.run([sys.executable, "-c", "import paper_2405_19509_gb300"], cwd=tmp_path,
+                       capture_output=True, text=True, timeout=300,
+                       env={**os.environ, "PYTHONPATH": str(tmp_path)})
+    assert r.returncode != 0
+    assert "ImportError" in r.stderr and "libgc.so is missing" in r.stderr
